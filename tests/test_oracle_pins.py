@@ -1,0 +1,362 @@
+"""Pins of the CPU oracle to facts fixed outside it: hand-worked index sets from Eq. 2,
+closed forms, an independent fmaf (the C library's), library routines (scipy cosine,
+torch scaled_dot_product_attention), exact integer arithmetic, brute-force enumeration
+and invariants.  CPU only."""
+import ctypes
+import ctypes.util
+import itertools
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+import workloads as W
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _rng(seed=0):
+    return np.random.default_rng(seed)
+
+
+def _bf16(x):
+    return W.bf16_bits_to_f32(W.to_bf16_bits(np.asarray(x, dtype=np.float64)))
+
+
+def _parse_range(s):
+    s = s.strip()
+    if s == "-":
+        return ()
+    out = []
+    for part in s.split(","):
+        if "-" in part:
+            a, b = part.split("-")
+            out += list(range(int(a), int(b) + 1))
+        else:
+            out.append(int(part))
+    return tuple(out)
+
+
+# ---------------------------------------------------------------- frame bookkeeping
+def test_frame_roles_golden():
+    n = 0
+    for line in open(os.path.join(GOLDEN, "frame_roles.txt")):
+        if line.startswith("#") or not line.strip():
+            continue
+        cols = [c.strip() for c in line.split("|")]
+        nh, S, Wn = map(int, cols[0].split())
+        r = O.frame_roles(nh, S, Wn)
+        assert r.sink == _parse_range(cols[1]), line
+        assert r.window == _parse_range(cols[2]), line
+        anchor = None if cols[3] == "-" else int(cols[3])
+        assert r.anchor == anchor, line
+        assert r.scoreable == _parse_range(cols[4]), line
+        n += 1
+    assert n >= 8
+
+
+def test_eq2_static_tokens_golden():
+    lines = [l for l in open(os.path.join(GOLDEN, "eq2_static_tokens.txt")) if not l.startswith("#")]
+    params = dict(kv.split("=") for kv in lines[0].split())
+    C, F, S, i = (int(params[k]) for k in ("C", "F", "S", "i"))
+    expected = [int(x) for x in lines[1].split()]
+    roles = O.frame_roles(i * C, S, 0)
+    got = O.static_key_tokens(roles, F, range(i * C, (i + 1) * C))
+    assert got == expected
+
+
+def test_segment_ranges_partition_frame():
+    for F, n in [(60, 1), (60, 6), (1560, 6), (8160, 6), (12, 4)]:
+        rs = [O.segment_range(F, n, j) for j in range(n)]
+        assert rs[0][0] == 0 and rs[-1][1] == F
+        assert all(a[1] == b[0] for a, b in zip(rs, rs[1:]))
+        assert len({hi - lo for lo, hi in rs}) == 1
+    with pytest.raises(ValueError):
+        O.segment_range(10, 3, 0)
+
+
+def test_keep_count_floor():
+    assert O.keep_count(700, 6) == 4      # b = 1 - r = 0.7 with r = 0.3, n = 6 (App. H)
+    assert O.keep_count(600, 6) == 3
+    assert O.keep_count(500, 6) == 3
+    assert O.keep_count(500, 1) == 0
+    assert O.keep_count(1000, 6) == 6
+    assert O.keep_count(0, 6) == 0
+    assert O.keep_count(300, 6) == 1      # Eq. 3 literally: floor(r n) with r = 0.3
+
+
+# ---------------------------------------------------------------- Eq. 3 scores
+def test_fmaf_emulation_matches_c_library():
+    libm = ctypes.CDLL(ctypes.util.find_library("m"))
+    libm.fmaf.restype = ctypes.c_float
+    libm.fmaf.argtypes = [ctypes.c_float] * 3
+    rng = _rng(1)
+    a = _bf16(rng.standard_normal(4000) * np.exp2(rng.integers(-20, 20, 4000)))
+    b = _bf16(rng.standard_normal(4000) * np.exp2(rng.integers(-20, 20, 4000)))
+    c = (rng.standard_normal(4000) * np.exp2(rng.integers(-40, 40, 4000))).astype(np.float32)
+    got = O.fmaf_bf16(a, b, c)
+    ref = np.array([libm.fmaf(float(x), float(y), float(z)) for x, y, z in zip(a, b, c)],
+                   dtype=np.float32)
+    assert np.array_equal(got.view(np.uint32), ref.view(np.uint32))
+
+
+@pytest.mark.parametrize("D", [64, 128])
+def test_token_dot_exact_on_small_integers(D):
+    rng = _rng(D)
+    A = rng.integers(-8, 9, size=(300, D)).astype(np.float32)
+    B = rng.integers(-8, 9, size=(300, D)).astype(np.float32)
+    exact = (A.astype(np.int64) * B.astype(np.int64)).sum(axis=1)
+    assert np.array_equal(O.token_dots_contract(A, B).astype(np.int64), exact)
+
+
+@pytest.mark.parametrize("D", [64, 128])
+def test_token_dot_within_fp32_error_bound(D):
+    # an fma chain of 8 then log2(D/8) butterfly adds: error <= (8 + log2(D/8)) u sum|ab|
+    rng = _rng(D + 1)
+    A = _bf16(rng.standard_normal((2000, D)) * 3)
+    B = _bf16(rng.standard_normal((2000, D)) * 3)
+    exact = (A.astype(np.float64) * B.astype(np.float64)).sum(axis=1)
+    bound = (8 + math.log2(D // 8)) * 2.0 ** -24 * np.abs(A.astype(np.float64) * B).sum(axis=1)
+    err = np.abs(O.token_dots_contract(A, B).astype(np.float64) - exact)
+    assert (err <= bound * 1.0001 + 1e-30).all()
+
+
+def test_fixed_point_truncates_toward_zero():
+    x = np.array([1.5, -1.5, 2.0 ** -25, -(2.0 ** -25), 3.0, 0.0], dtype=np.float64) * 2.0 ** -24
+    assert O.fixed_point(x).tolist() == [1, -1, 0, 0, 3, 0]
+    assert O.fixed_point(np.float32(2.0 ** 23)).item() == 2 ** 47
+
+
+def test_score_closed_forms():
+    rng = _rng(3)
+    a = _bf16(rng.standard_normal((260, 128)))
+    assert O.segment_score_contract(a, a) == np.float32(1.0)
+    assert O.segment_score_contract(a, -a) == np.float32(-1.0)
+    # disjoint channel support in every token: orthogonal segments
+    b = a.copy()
+    a2 = a.copy()
+    a2[:, 64:] = 0
+    b[:, :64] = 0
+    assert O.segment_score_contract(a2, b) == np.float32(0.0)
+    assert O.segment_score_contract(np.zeros_like(a), a) == np.float32(0.0)
+    assert O.cosine_fp64(a2, b) == 0.0
+    assert abs(O.cosine_fp64(a, -a) + 1.0) < 1e-15
+
+
+def test_cosine_matches_scipy_and_contract():
+    from scipy.spatial.distance import cosine as scipy_cosine
+    rng = _rng(4)
+    for rho in (0.0, 0.5, 0.9, 0.99):
+        x = _bf16(rng.standard_normal((260, 128)) * 1.7)
+        y = _bf16(rho * x + math.sqrt(1 - rho * rho) * rng.standard_normal((260, 128)) * 1.7)
+        ref = 1.0 - scipy_cosine(x.astype(np.float64).ravel(), y.astype(np.float64).ravel())
+        assert abs(O.cosine_fp64(x, y) - ref) < 1e-12
+        assert abs(float(O.segment_score_contract(x, y)) - ref) <= 1e-6
+
+
+def test_contract_scores_token_permutation_invariant():
+    rng = _rng(5)
+    x = _bf16(rng.standard_normal((260, 128)))
+    y = _bf16(0.9 * x + 0.4 * rng.standard_normal((260, 128)))
+    p = rng.permutation(260)
+    s0 = O.segment_score_contract(x, y)
+    s1 = O.segment_score_contract(x[p], y[p])
+    assert s0.view(np.uint32) == s1.view(np.uint32)
+
+
+def test_cosine_scale_invariant_fp64():
+    rng = _rng(6)
+    x = _bf16(rng.standard_normal((100, 64)))
+    y = _bf16(rng.standard_normal((100, 64)) + x)
+    for m in (-3, 2, 5):
+        assert abs(O.cosine_fp64(x * 2.0 ** m, y) - O.cosine_fp64(x, y)) < 1e-14
+
+
+def test_score_precondition_enforced():
+    a = np.full((4, 128), 300.0, dtype=np.float32)   # n_p = 128 * 90000 > 2^23
+    with pytest.raises(ValueError):
+        O.segment_score_contract(a, a)
+
+
+# ---------------------------------------------------------------- Eq. 3 BottomK
+def _brute_force_keep(scores, k):
+    """The unique size-k subset whose members all precede every non-member in (score, index)."""
+    n = len(scores)
+    key = [(float(s), i) for i, s in enumerate(scores)]
+    hits = []
+    for sub in itertools.combinations(range(n), k):
+        rest = [i for i in range(n) if i not in sub]
+        if all(key[a] < key[b] for a in sub for b in rest):
+            hits.append(sorted(sub))
+    assert len(hits) == 1
+    return hits[0]
+
+
+def test_bottom_k_brute_force_with_ties():
+    rng = _rng(7)
+    for trial in range(300):
+        n = int(rng.integers(1, 8))
+        s = rng.choice(np.array([0.1, 0.5, 0.5, 0.9, -0.2, 0.5], dtype=np.float32), size=n)
+        for k in range(n + 1):
+            assert O.bottom_k(s, range(n), k) == _brute_force_keep(s, k)
+
+
+def test_bottom_k_keeps_lowest_similarity():
+    s = np.array([0.99, 0.2, 0.95, 0.1, 0.97, 0.5], dtype=np.float32)
+    # evict the highest-similarity segments, keep floor(0.7 * 6) = 4 (Sec. 4.3)
+    assert O.bottom_k(s, range(6), 4) == [1, 2, 3, 5]
+
+
+def test_bottom_k_ties_go_to_lower_index():
+    s = np.float32([0.5] * 6)
+    assert O.bottom_k(s, range(6), 3) == [0, 1, 2]
+
+
+# ---------------------------------------------------------------- Eq. 3/4 on constructed frames
+def _constructed_oracle(static_map, n_hist=5, S=1, C=2, F=12, n=4, D=64, budget=500, seed=8):
+    """Frames whose segments j in `same[t]` are copied from frame t into frame t+1."""
+    rng = _rng(seed)
+    H = len(static_map)
+    frames = [rng.standard_normal((F, H, D))]
+    same = {}
+    for t in range(1, n_hist + C):
+        f = rng.standard_normal((F, H, D))
+        pick = rng.choice(n, size=n - O.keep_count(budget, n), replace=False)
+        same[t - 1] = sorted(pick.tolist())
+        for j in pick:
+            lo, hi = O.segment_range(F, n, j)
+            f[lo:hi] = frames[-1][lo:hi]
+        frames.append(f)
+    bits = W.to_bf16_bits(np.concatenate(frames))
+    orc = O.ForcingKVOracle(n_layers=1, n_heads=H, head_dim=D, tokens_per_frame=F,
+                            frames_per_chunk=C, n_sink_frames=S, window_frames=0, n_segments=n,
+                            keep_budget_permille=budget, head_is_static=[static_map])
+    orc.append_frames(0, bits[:n_hist * F], bits[:n_hist * F])
+    orc.append_chunk(0, bits[n_hist * F:], bits[n_hist * F:])
+    return orc, same
+
+
+def test_kept_segments_are_the_changed_ones():
+    orc, same = _constructed_oracle([0, 0])
+    n = 4
+    for h in range(2):
+        sc = orc.scores(0, h)
+        kept = orc.kept(0, h)
+        for t in orc.roles(0).scoreable:
+            for j in same[t]:
+                assert sc[t][j] == np.float32(1.0)       # t compared with t+1, not t-1
+            expect = [t * n + j for j in range(n) if j not in same[t]]
+            assert [s for s in kept if s // n == t] == expect
+
+
+def test_dynamic_set_full_budget_is_full_window():
+    orc, _ = _constructed_oracle([0, 1], budget=1000)
+    total = (orc.nh[0] + orc.C) * orc.F
+    assert sorted(orc.key_tokens(0, 0)) == list(range(total))
+
+
+def test_dynamic_set_zero_budget_is_static_set():
+    orc, _ = _constructed_oracle([0, 1], budget=0)
+    assert orc.key_tokens(0, 0) == orc.key_tokens(0, 1)
+    roles = orc.roles(0)
+    assert orc.key_tokens(0, 1) == O.static_key_tokens(roles, orc.F, orc.current_frames(0))
+
+
+def test_pooled_selection_brute_force():
+    w = W.TINY
+    hk, hv, ck, cv, q = W.snapshot_inputs(w)
+    orc = O.ForcingKVOracle.from_workload(w, W.head_map(w))
+    orc.append_frames(0, hk, hv)
+    orc.append_chunk(0, ck, cv)
+    for h in (2, 3):
+        sc = orc.scores(0, h)
+        flat = np.array([sc[t][0] for t in sorted(sc)])
+        assert len(flat) == 6
+        assert orc.kept(0, h) == _brute_force_keep(flat, 3)
+
+
+def test_layer0_pooled_score_is_cosine_over_heads():
+    w = W.TINY_PER_FRAME.with_(score_source="layer0_pooled", n_layers=2)
+    fs = W.FrameStream(w, 0)
+    hk, hv = fs.frames(w.n_history_frames)
+    orc = O.ForcingKVOracle.from_workload(w, W.head_map(w))
+    orc.append_frames(0, hk, hv)
+    sc = orc.scores(1, 2)  # a layer-1 dynamic head is scored with layer-0 keys of all heads
+    K = W.bf16_bits_to_f32(hk).reshape(w.n_history_frames, w.tokens_per_frame, w.n_heads, w.head_dim)
+    for t in sc:
+        for j in range(w.n_segments):
+            lo, hi = O.segment_range(w.tokens_per_frame, w.n_segments, j)
+            ref = O.cosine_fp64(K[t, lo:hi], K[t + 1, lo:hi])
+            assert abs(float(sc[t][j]) - ref) <= 1e-6
+
+
+# ---------------------------------------------------------------- attention
+def _sdpa64(Q, K, V):
+    q = torch.from_numpy(np.asarray(Q, np.float64))[None, None]
+    k = torch.from_numpy(np.asarray(K, np.float64))[None, None]
+    v = torch.from_numpy(np.asarray(V, np.float64))[None, None]
+    return torch.nn.functional.scaled_dot_product_attention(q, k, v)[0, 0].numpy()
+
+
+def test_attention_matches_torch_sdpa():
+    rng = _rng(9)
+    Q, K, V = (rng.standard_normal((300, 64)), rng.standard_normal((777, 64)) * 2,
+               rng.standard_normal((777, 64)))
+    assert np.abs(O.attention_fp64(Q, K, V, row_block=64) - _sdpa64(Q, K, V)).max() < 1e-12
+
+
+def test_attention_closed_forms():
+    rng = _rng(10)
+    Q = rng.standard_normal((5, 32))
+    K1, V1 = rng.standard_normal((1, 32)), rng.standard_normal((1, 32))
+    assert np.allclose(O.attention_fp64(Q, K1, V1), np.repeat(V1, 5, 0), atol=1e-15)
+    Ks = np.repeat(rng.standard_normal((1, 32)), 40, 0)
+    V = rng.standard_normal((40, 32))
+    assert np.allclose(O.attention_fp64(Q, Ks, V), V.mean(0, keepdims=True), atol=1e-13)
+
+
+def test_oracle_full_budget_equals_full_attention():
+    w = W.TINY_PER_FRAME.with_(keep_budget_permille=1000)
+    hk, hv, ck, cv, q = W.snapshot_inputs(w)
+    orc = O.ForcingKVOracle.from_workload(w, W.head_map(w))
+    orc.append_frames(0, hk, hv)
+    orc.append_chunk(0, ck, cv)
+    out = orc.attend(0, q)
+    Kall = W.bf16_bits_to_f32(np.concatenate([hk, ck]))
+    Vall = W.bf16_bits_to_f32(np.concatenate([hv, cv]))
+    Qf = W.bf16_bits_to_f32(q)
+    for h in (2, 3):   # dynamic heads: full window
+        ref = _sdpa64(Qf[:, h], Kall[:, h], Vall[:, h])
+        assert np.abs(out[:, h] - ref).max() < 1e-12
+    F = w.tokens_per_frame
+    for h in (0, 1):   # static heads: Eq. 2 only (no sink in this case: anchor + chunk)
+        idx = np.r_[6 * F:7 * F, 7 * F:10 * F]
+        ref = _sdpa64(Qf[:, h], Kall[idx, h], Vall[idx, h])
+        assert np.abs(out[:, h] - ref).max() < 1e-12
+
+
+def test_view_lengths_match_paper_sizes():
+    # 480P single layer: static = sink + anchor + chunk, dynamic adds 17 frames x 4 x 260 tokens
+    w = W.P480_LAYER
+    roles = O.frame_roles(w.n_history_frames, w.n_sink_frames, w.window_frames)
+    F = w.tokens_per_frame
+    cur = range(19, 22)
+    assert len(O.static_key_tokens(roles, F, cur)) == 7800
+    kept = [t * 6 + j for t in roles.scoreable for j in range(4)]
+    assert len(O.dynamic_key_tokens(roles, F, 6, kept, cur)) == 25480
+
+
+def test_window_drops_old_frames():
+    w = W.ROLLING.with_(tokens_per_frame=12, n_heads=2, head_dim=16, n_chunks=8)
+    orc = O.ForcingKVOracle.from_workload(w, [[1, 0]])
+    fs = W.FrameStream(w, 0)
+    for c in range(8):
+        k, v = fs.frames(3)
+        orc.append_chunk(0, k, v)
+    r = orc.roles(0)
+    assert orc.nh[0] == 21 and r.window == tuple(range(9, 21)) and r.sink == (0,)
+    assert sorted(orc.frames[0]) == [0] + list(range(9, 21))
+    assert len(orc.kept(0, 1)) == 11 * 3

@@ -1,0 +1,283 @@
+"""Seeded synthetic workloads for the Forcing-KV hot path.
+
+This module holds the workload definitions (shapes, schedules and value models
+shaped like the paper's 480P / 1080P Self Forcing and LongLive settings, Sec. 5
+and App. H) and one counter-based random generator.  The CPU oracle and the
+CUDA path are both fed from here, byte for byte.  Nothing in this module
+computes any part of the method: no scores, no selection, no attention.
+
+Generator (fixed recipe, independent of platform):
+  * SplitMix64 (Steele, Lea & Flood, OOPSLA 2014) over a 64-bit counter,
+  * Box-Muller in fp64 on the two 24-bit halves of each 64-bit draw,
+  * fp64 -> fp32 (round to nearest) -> bf16 (round to nearest even).
+
+Value model (per layer, per head, per token, per channel):
+  * keys   K_f = s_h * x_f, x_f = rho_k * x_{f-1} + sqrt(1 - rho_k^2) * e_f,
+    x_0 = e_0, and x_f = e_f at a scene-cut frame;  s_h ~ U[scale_lo, scale_hi];
+  * values the same AR(1) recursion with rho_v and no head scale;
+  * queries iid N(0, 1).
+"""
+from __future__ import annotations
+
+import math
+from dataclasses import dataclass, field, replace
+from typing import Iterator
+
+import numpy as np
+
+__all__ = [
+    "Workload", "TINY", "TINY_PER_FRAME", "P480_LAYER", "P480_STACK", "ROLLING",
+    "P1080_LAYER", "WORKLOADS", "normals", "uniforms", "to_bf16_bits", "bf16_bits_to_f32",
+    "head_map", "FrameStream", "snapshot_inputs", "queries", "step_kv", "stream_key",
+]
+
+_U64 = np.uint64
+
+
+def _splitmix64(x: np.ndarray) -> np.ndarray:
+    with np.errstate(over="ignore"):
+        z = x + _U64(0x9E3779B97F4A7C15)
+        z = (z ^ (z >> _U64(30))) * _U64(0xBF58476D1CE4E5B9)
+        z = (z ^ (z >> _U64(27))) * _U64(0x94D049BB133111EB)
+        return z ^ (z >> _U64(31))
+
+
+def stream_key(*tags: int) -> int:
+    """Fold integer tags (seed, tensor kind, layer, frame, ...) into one 64-bit key."""
+    k = np.array([0x51ED2701F00DCAFE], dtype=np.uint64)
+    for t in tags:
+        with np.errstate(over="ignore"):
+            k = _splitmix64(k ^ np.array([t & 0xFFFFFFFFFFFFFFFF], dtype=np.uint64))
+    return int(k[0])
+
+
+def normals(key: int, n: int) -> np.ndarray:
+    """n standard normal draws (fp64) of stream `key`."""
+    m = (n + 1) // 2
+    with np.errstate(over="ignore"):
+        z = _splitmix64(_U64(key) + np.arange(m, dtype=np.uint64))
+    u1 = ((z >> _U64(40)).astype(np.float64) + 1.0) * (1.0 / 16777216.0)        # (0, 1]
+    u2 = ((z >> _U64(16)) & _U64(0xFFFFFF)).astype(np.float64) * (1.0 / 16777216.0)  # [0, 1)
+    r = np.sqrt(-2.0 * np.log(u1))
+    out = np.empty(2 * m, dtype=np.float64)
+    out[0::2] = r * np.cos(2.0 * math.pi * u2)
+    out[1::2] = r * np.sin(2.0 * math.pi * u2)
+    return out[:n]
+
+
+def uniforms(key: int, n: int) -> np.ndarray:
+    """n uniform draws in [0, 1) (fp64) of stream `key`."""
+    with np.errstate(over="ignore"):
+        z = _splitmix64(_U64(key) + np.arange(n, dtype=np.uint64))
+    return (z >> _U64(11)).astype(np.float64) * (1.0 / 9007199254740992.0)
+
+
+def to_bf16_bits(x: np.ndarray) -> np.ndarray:
+    """fp64/fp32 -> fp32 (nearest) -> bf16 bit pattern (nearest even), as uint16."""
+    b = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32)
+    with np.errstate(over="ignore"):
+        r = (b + np.uint32(0x7FFF) + ((b >> np.uint32(16)) & np.uint32(1))) >> np.uint32(16)
+    return r.astype(np.uint16)
+
+
+def bf16_bits_to_f32(bits: np.ndarray) -> np.ndarray:
+    """bf16 bit pattern (uint16) -> exact fp32 value."""
+    return (np.asarray(bits, dtype=np.uint16).astype(np.uint32) << np.uint32(16)).view(np.float32)
+
+
+# tensor-kind tags of the generator streams
+_K, _V, _Q, _SCALE, _MAP, _KSTEP, _VSTEP = 1, 2, 3, 4, 5, 6, 7
+
+
+@dataclass(frozen=True)
+class Workload:
+    """One synthetic workload: cache/attention shapes plus its driving schedule.
+
+    schedule "snapshot": `n_history_frames` frames are loaded as history, then one
+    chunk of C frames is the current chunk (single-layer cases).
+    schedule "stream": `n_chunks` chunks are appended one by one; after each append
+    the cache is compressed and the chunk is attended `denoise_steps` times.
+    """
+    name: str
+    n_layers: int
+    n_heads: int
+    head_dim: int
+    tokens_per_frame: int
+    frames_per_chunk: int
+    n_sink_frames: int
+    window_frames: int            # non-sink history frames kept (0 = unbounded)
+    n_segments: int
+    keep_budget_permille: int
+    select_scope: str = "per_frame"      # "per_frame" | "pooled"
+    score_source: str = "per_head"       # "per_head" | "layer0_pooled"
+    incremental: bool = False
+    schedule: str = "snapshot"
+    n_history_frames: int = 0
+    n_chunks: int = 0
+    denoise_steps: int = 1
+    rho_k: float = 0.9
+    rho_v: float = 0.9
+    scale_lo: float = 0.5
+    scale_hi: float = 2.0
+    scene_cut_every_chunks: int = 0
+    static_heads: tuple = ()             # fixed static heads (empty = seeded map)
+    static_fraction: float = 0.5
+    exact_half_static: bool = True       # seeded permutation with exactly H/2 static
+    seed: int = 0
+    description: str = ""
+
+    # ---- derived sizes ----
+    @property
+    def seg_len(self) -> int:
+        return self.tokens_per_frame // self.n_segments
+
+    @property
+    def n_queries(self) -> int:
+        return self.frames_per_chunk * self.tokens_per_frame
+
+    def max_history_frames(self) -> int:
+        if self.schedule == "snapshot":
+            return self.n_history_frames
+        return self.n_chunks * self.frames_per_chunk
+
+    def scene_cut(self, frame: int) -> bool:
+        e = self.scene_cut_every_chunks
+        return e > 0 and frame > 0 and frame % (e * self.frames_per_chunk) == 0
+
+    def with_(self, **kw) -> "Workload":
+        return replace(self, **kw)
+
+
+TINY = Workload(
+    name="tiny", n_layers=1, n_heads=4, head_dim=64, tokens_per_frame=60, frames_per_chunk=3,
+    n_sink_frames=0, window_frames=0, n_segments=1, keep_budget_permille=500,
+    select_scope="pooled", schedule="snapshot", n_history_frames=7,
+    rho_k=0.8, rho_v=0.0, scale_lo=1.0, scale_hi=1.0, static_heads=(0, 1), seed=0,
+    description="tiny correctness case: 1 layer, 4 heads (0-1 static), D=64, 60 tokens/frame, "
+                "3-frame chunk, 7 history frames, one segment per frame, 50% budget pooled")
+
+TINY_PER_FRAME = TINY.with_(
+    name="tiny_per_frame", n_segments=6, select_scope="per_frame",
+    description="tiny case with 6 segments (grid rows) per frame, 3 of 6 kept per frame")
+
+P480_LAYER = Workload(
+    name="480p_layer", n_layers=1, n_heads=12, head_dim=128, tokens_per_frame=1560,
+    frames_per_chunk=3, n_sink_frames=1, window_frames=0, n_segments=6, keep_budget_permille=700,
+    schedule="snapshot", n_history_frames=19, seed=1,
+    description="480P single layer: 12 heads (6 static seeded), D=128, 1560 tokens/frame (30x52), "
+                "4680 queries, 1 sink + 18 history frames, 70% dynamic budget")
+
+P480_STACK = Workload(
+    name="480p_stack", n_layers=30, n_heads=12, head_dim=128, tokens_per_frame=1560,
+    frames_per_chunk=3, n_sink_frames=1, window_frames=0, n_segments=6, keep_budget_permille=700,
+    score_source="layer0_pooled", incremental=True, schedule="stream", n_chunks=7, denoise_steps=4,
+    exact_half_static=False, seed=2,
+    description="480P stack: 30 layers x 12 heads, 7 chunks of 3 frames, 4 denoising steps, "
+                "compression after each append, layer-0 pooled scoring")
+
+ROLLING = Workload(
+    name="rolling", n_layers=1, n_heads=12, head_dim=128, tokens_per_frame=1560,
+    frames_per_chunk=3, n_sink_frames=1, window_frames=12, n_segments=6, keep_budget_permille=600,
+    incremental=True, schedule="stream", n_chunks=60, denoise_steps=1,
+    rho_k=0.95, rho_v=0.95, scene_cut_every_chunks=20, seed=3,
+    description="rolling cache: 12 heads, D=128, 1 sink + 12-frame window, 60 chunks, 60% budget, "
+                "rho=0.95 drift with a scene cut every 20 chunks")
+
+P1080_LAYER = Workload(
+    name="1080p_layer", n_layers=1, n_heads=12, head_dim=128, tokens_per_frame=8160,
+    frames_per_chunk=3, n_sink_frames=1, window_frames=0, n_segments=6, keep_budget_permille=700,
+    schedule="snapshot", n_history_frames=10, seed=4,
+    description="1080P single layer: 12 heads, D=128, 8160 tokens/frame (68x120), 24480 queries, "
+                "1 sink + 9 history frames, 70% dynamic budget")
+
+WORKLOADS = {w.name: w for w in (TINY, TINY_PER_FRAME, P480_LAYER, P480_STACK, ROLLING, P1080_LAYER)}
+
+
+def head_map(w: Workload) -> np.ndarray:
+    """uint8 [n_layers, n_heads]: 1 = static head, 0 = dynamic head (seeded)."""
+    m = np.zeros((w.n_layers, w.n_heads), dtype=np.uint8)
+    for layer in range(w.n_layers):
+        if w.static_heads:
+            m[layer, list(w.static_heads)] = 1
+        elif w.exact_half_static:
+            u = uniforms(stream_key(w.seed, _MAP, layer), w.n_heads)
+            m[layer, np.argsort(u, kind="stable")[: w.n_heads // 2]] = 1
+        else:
+            u = uniforms(stream_key(w.seed, _MAP, layer), w.n_heads)
+            m[layer] = (u < w.static_fraction).astype(np.uint8)
+    return m
+
+
+def _head_scales(w: Workload, layer: int) -> np.ndarray:
+    u = uniforms(stream_key(w.seed, _SCALE, layer), w.n_heads)
+    return w.scale_lo + (w.scale_hi - w.scale_lo) * u
+
+
+class FrameStream:
+    """Sequential AR(1) key/value frames of one layer, as bf16 bits [F, H, D]."""
+
+    def __init__(self, w: Workload, layer: int):
+        self.w, self.layer, self.next = w, layer, 0
+        self._xk = None
+        self._xv = None
+        self._scale = _head_scales(w, layer)[None, :, None]
+
+    def _step(self, x, rho, kind, f):
+        w = self.w
+        e = normals(stream_key(w.seed, kind, self.layer, f),
+                    w.tokens_per_frame * w.n_heads * w.head_dim)
+        e = e.reshape(w.tokens_per_frame, w.n_heads, w.head_dim)
+        if x is None or w.scene_cut(f):
+            return e
+        return rho * x + math.sqrt(max(0.0, 1.0 - rho * rho)) * e
+
+    def next_frame(self) -> tuple[np.ndarray, np.ndarray]:
+        f = self.next
+        self._xk = self._step(self._xk, self.w.rho_k, _K, f)
+        self._xv = self._step(self._xv, self.w.rho_v, _V, f)
+        self.next += 1
+        return to_bf16_bits(self._scale * self._xk), to_bf16_bits(self._xv)
+
+    def frames(self, n: int) -> tuple[np.ndarray, np.ndarray]:
+        """The next n frames, concatenated token-major: [n*F, H, D] each."""
+        ks, vs = zip(*(self.next_frame() for _ in range(n))) if n else ((), ())
+        w = self.w
+        shape = (0, w.n_heads, w.head_dim)
+        return (np.concatenate(ks) if n else np.zeros(shape, np.uint16),
+                np.concatenate(vs) if n else np.zeros(shape, np.uint16))
+
+    def chunks(self) -> Iterator[tuple[np.ndarray, np.ndarray]]:
+        while True:
+            yield self.frames(self.w.frames_per_chunk)
+
+
+def snapshot_inputs(w: Workload, layer: int = 0):
+    """(history K, history V [n_hist*F, H, D], current K, current V [C*F, H, D], Q [C*F, H, D])."""
+    fs = FrameStream(w, layer)
+    hk, hv = fs.frames(w.n_history_frames)
+    ck, cv = fs.frames(w.frames_per_chunk)
+    q = queries(w, layer, 0, 0)
+    return hk, hv, ck, cv, q
+
+
+def queries(w: Workload, layer: int, chunk: int, step: int) -> np.ndarray:
+    """Queries of one chunk at one denoising step: iid N(0,1) bf16 bits [C*F, H, D]."""
+    n = w.n_queries * w.n_heads * w.head_dim
+    q = normals(stream_key(w.seed, _Q, layer, chunk, step), n)
+    return to_bf16_bits(q).reshape(w.n_queries, w.n_heads, w.head_dim)
+
+
+def step_kv(w: Workload, layer: int, chunk: int, step: int, clean_k: np.ndarray,
+            clean_v: np.ndarray) -> tuple[np.ndarray, np.ndarray]:
+    """Current-chunk K/V at denoising step `step`: the clean chunk on the last step,
+    earlier steps add seeded noise of decreasing weight (a stand-in for noisy latents)."""
+    last = w.denoise_steps - 1
+    if step >= last:
+        return clean_k, clean_v
+    a = 0.5 * (last - step) / max(1, last)
+    n = clean_k.size
+    ek = normals(stream_key(w.seed, _KSTEP, layer, chunk, step), n).reshape(clean_k.shape)
+    ev = normals(stream_key(w.seed, _VSTEP, layer, chunk, step), n).reshape(clean_v.shape)
+    k = bf16_bits_to_f32(clean_k).astype(np.float64) + a * ek
+    v = bf16_bits_to_f32(clean_v).astype(np.float64) + a * ev
+    return to_bf16_bits(k), to_bf16_bits(v)
