@@ -1,0 +1,194 @@
+/*
+ * fk.h -- C ABI of the Forcing-KV hot path (hybrid KV-cache compression plus chunk
+ * attention over the compressed cache) on one NVIDIA GB300 (sm_103a).
+ *
+ * The operations follow the paper's statement of the method:
+ *   - static heads attend to [sink frames, transition-anchor frame, current chunk]
+ *     (Sec. 4.2, Eq. 2);
+ *   - dynamic heads score each history frame t against frame t+1 segment by segment
+ *     with a cosine similarity, keep the floor(b*n) lowest-similarity segments of the
+ *     n equal segments of each frame (BottomK, Sec. 4.3, Eq. 3; b = 1 - r, the keep
+ *     budget, App. H) and attend to [sink, kept segments, anchor frame, current chunk]
+ *     (Sec. 4.3, Eq. 4; the anchor is kept because the dynamic-head cache subsumes the
+ *     static portion, Sec. 5.3);
+ *   - compression starts once adjacent history frames exist (App. H); sink frames are
+ *     never scored or evicted.
+ *
+ * Conventions shared by every call:
+ *   - Tensors K, V, Q, O are bf16, token-major [tokens][n_heads][head_dim], row-major
+ *     and contiguous ("the [seq, heads, dim] layout"), 16-byte aligned.
+ *   - A tensor pointer may be device memory or host memory (pinned or pageable).  Host
+ *     inputs are copied into library-owned device staging buffers on `stream`; a host
+ *     output is written by an asynchronous device-to-host copy on `stream`, so the
+ *     caller synchronizes `stream` before reading it.  Caller-owned device inputs must
+ *     stay valid until the work queued on `stream` by the call has run.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = the legacy default stream).
+ *   - Frames are numbered globally from 0 in append order.  The history is every frame
+ *     appended before the current chunk; the current chunk is frames nh..nh+C-1, where
+ *     nh is the number of history frames.  Segment id of segment j of frame t is t*n+j.
+ *   - Every call returns a status code.  The library never aborts, traps or prints.
+ *     Conditions found on the device (the scoring precondition, an expired bounded
+ *     wait) are recorded in a device status word and reported by fk_sync_status.
+ *   - The library owns all of its device memory; it is allocated in fk_create and
+ *     released in fk_destroy.  No other call allocates.
+ *   - A handle is not thread-safe: calls on one handle are made from one host thread.
+ */
+#ifndef FK_H
+#define FK_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define FK_API __attribute__((visibility("default")))
+#else
+#define FK_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum fk_status {
+  FK_OK = 0,
+  FK_ERR_CONFIG = 1,   /* invalid configuration (see fk_config)                         */
+  FK_ERR_ARG = 2,      /* null or misaligned pointer, layer/head out of range, short buffer */
+  FK_ERR_STATE = 3,    /* call out of order: attend before compress, no current chunk,
+                          layers out of step under layer-0 pooled scoring               */
+  FK_ERR_FULL = 4,     /* unbounded window and max_history_frames would be exceeded      */
+  FK_ERR_RANGE = 5,    /* scoring precondition violated: a token's squared key norm > 2^23 */
+  FK_ERR_TIMEOUT = 6,  /* a bounded wait inside a kernel expired; outputs are undefined   */
+  FK_ERR_CUDA = 7,     /* a CUDA runtime/driver call failed (no device, launch failure)   */
+  FK_ERR_NOMEM = 8     /* device memory for the cache could not be allocated             */
+} fk_status;
+
+/* Selection scope of BottomK (Eq. 3). */
+enum {
+  FK_SCOPE_PER_FRAME = 0, /* keep floor(b*n) segments of every scoreable frame            */
+  FK_SCOPE_POOLED = 1     /* keep floor(b*|T|*n) segments over all scoreable frames T      */
+};
+
+/* Which keys score the dynamic heads (Eq. 3). */
+enum {
+  FK_SCORE_PER_HEAD = 0,      /* each dynamic head scores its own keys                     */
+  FK_SCORE_LAYER0_POOLED = 1  /* keys of every head of layer 0, pooled, score every dynamic
+                                 head of every layer ("the first block ... as a proxy",
+                                 Sec. 4.3); one kept set is shared by all dynamic heads     */
+};
+
+typedef struct fk_config {
+  int32_t n_layers;             /* 1..256                                                  */
+  int32_t n_heads;              /* 1..128                                                  */
+  int32_t head_dim;             /* 64 or 128                                               */
+  int32_t tokens_per_frame;     /* F >= 1, a multiple of n_segments                        */
+  int32_t frames_per_chunk;     /* C >= 1                                                  */
+  int32_t n_sink_frames;        /* S >= 0: frames 0..S-1 are sinks, never evicted          */
+  int32_t window_frames;        /* W >= 0 non-sink history frames kept, anchor included;
+                                   0 = unbounded (capacity max_history_frames)            */
+  int32_t n_segments;           /* n >= 1 contiguous equal segments per frame              */
+  int32_t keep_budget_permille; /* b*1000 in [0, 1000]; k = floor(b*n) kept per frame      */
+  int32_t select_scope;         /* FK_SCOPE_*                                              */
+  int32_t score_source;         /* FK_SCORE_*                                              */
+  int32_t incremental;          /* 1: fk_compress scores only frame pairs not scored yet
+                                   (a frame's pairs never change once both frames exist);
+                                   0: every fk_compress rescores the whole window         */
+  int32_t max_history_frames;   /* history capacity in frames, sinks included, when W = 0 */
+  int32_t device;               /* CUDA device ordinal                                     */
+  const uint8_t* head_is_static;/* host [n_layers*n_heads]: 1 = static head, 0 = dynamic;
+                                   copied by fk_create                                     */
+} fk_config;
+
+typedef struct fk_handle fk_handle;
+
+/* Host-only validation of a configuration (no CUDA call).  FK_OK or FK_ERR_CONFIG /
+ * FK_ERR_ARG.  fk_create runs the same checks first. */
+FK_API fk_status fk_validate_config(const fk_config* cfg);
+
+/* Create a cache on cfg->device and allocate all of its device memory.
+ * *out receives the handle (NULL on failure). */
+FK_API fk_status fk_create(const fk_config* cfg, fk_handle** out);
+
+/* Release the handle and its device memory (synchronizes the device first). NULL is a no-op. */
+FK_API void fk_destroy(fk_handle* h);
+
+/* Append n_frames frames to the history of `layer` (e.g. loading sink and history
+ * frames).  If a current chunk exists it first joins the history, and afterwards no
+ * current chunk exists.  K, V: [n_frames*F][H][D].  Static heads keep only sink frames
+ * and the newest non-sink frame (the anchor); dynamic heads keep every window frame
+ * for scoring.  Marks the layer for fk_compress.  FK_ERR_FULL if the history would
+ * exceed max_history_frames with W = 0. */
+FK_API fk_status fk_append_frames(fk_handle* h, int layer, const void* K, const void* V, int n_frames,
+                           void* stream);
+
+/* Start AR step: the current chunk (if any) joins the history and K, V [C*F][H][D]
+ * become the current chunk of `layer` (Eq. 2 and Eq. 4 K_{iCF:(i+1)CF}).  Marks the
+ * layer for fk_compress. */
+FK_API fk_status fk_append_chunk(fk_handle* h, int layer, const void* K, const void* V, void* stream);
+
+/* Overwrite the current chunk's K, V [C*F][H][D] of `layer` (next denoising step of
+ * the same AR step), or set it when none exists.  The history is unchanged. */
+FK_API fk_status fk_set_current(fk_handle* h, int layer, const void* K, const void* V, void* stream);
+
+/* Compress every layer marked by an append: score the new (or, with incremental = 0,
+ * all) adjacent frame pairs of the window segment by segment (Eq. 3), select the kept
+ * segments (BottomK, ties to the lower segment id) and compact each dynamic head's
+ * keys and values into its packed view [current chunk | sink | kept segments | anchor].
+ * With no scoreable frame it only rebuilds the views.  Asynchronous on `stream`;
+ * FK_ERR_STATE when layer-0 pooled scoring finds layers with different histories. */
+FK_API fk_status fk_compress(fk_handle* h, void* stream);
+
+/* O [C*F][H][D] = per head softmax(Q K^T / sqrt(D)) V over the head's key set: Eq. 2
+ * for static heads, Eq. 4 plus the anchor frame for dynamic heads.  Q: [C*F][H][D].
+ * FK_ERR_STATE if `layer` has no current chunk or was appended to since the last
+ * fk_compress. */
+FK_API fk_status fk_attend(fk_handle* h, int layer, const void* Q, void* O, void* stream);
+
+/* Bytes of device memory currently holding live cache state: retained history pages,
+ * the used part of every packed view (current chunk included), scores and kept lists. */
+FK_API size_t fk_cache_bytes(const fk_handle* h);
+
+/* Bytes of device memory the handle allocated (all buffers, live or not). */
+FK_API size_t fk_reserved_bytes(const fk_handle* h);
+
+/* Number of keys head (layer, head) attends to at the current state (host-known). */
+FK_API fk_status fk_key_count(const fk_handle* h, int layer, int head, int* n_keys);
+
+/* Kept segment ids (t*n + j, ascending) of dynamic head (layer, head) after the last
+ * fk_compress; *n_out = 0 for a static head.  Synchronizes `stream`.  FK_ERR_ARG if
+ * capacity is too small (then *n_out holds the required count). */
+FK_API fk_status fk_get_kept(fk_handle* h, int layer, int head, int32_t* out, int capacity, int* n_out,
+                      void* stream);
+
+/* Segment scores s_t^(j) (fp32, Eq. 3 under the score contract) of the scoreable
+ * frames of dynamic head (layer, head): out[(t - *first_frame)*n + j] for the
+ * *n_frames frames t = *first_frame .. .  Synchronizes `stream`. */
+FK_API fk_status fk_get_scores(fk_handle* h, int layer, int head, float* out, int capacity,
+                        int* first_frame, int* n_frames, void* stream);
+
+/* Synchronize `stream` and report (then clear) device-side conditions:
+ * FK_ERR_RANGE, FK_ERR_TIMEOUT, or FK_OK. */
+FK_API fk_status fk_sync_status(fk_handle* h, void* stream);
+
+/* Kernel timing: when enabled, every kernel launch is bracketed by CUDA events on its
+ * stream.  fk_profile_read synchronizes and returns, per kernel kind, the total device
+ * milliseconds and the number of launches since the last reset. */
+enum { FK_KERNEL_APPEND = 0, FK_KERNEL_SCORE = 1, FK_KERNEL_SELECT = 2, FK_KERNEL_COMPACT = 3,
+       FK_KERNEL_ATTEND = 4, FK_KERNEL_KINDS = 5 };
+FK_API fk_status fk_profile_enable(fk_handle* h, int on);
+FK_API fk_status fk_profile_read(fk_handle* h, int kind, double* total_ms, int64_t* launches);
+FK_API fk_status fk_profile_reset(fk_handle* h);
+
+/* Kernels launched by this handle since creation (all kinds). */
+FK_API int64_t fk_launch_count(const fk_handle* h);
+
+/* Static text for a status code. */
+FK_API const char* fk_status_str(fk_status s);
+
+/* ABI version of this header: 1. */
+FK_API int fk_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* FK_H */

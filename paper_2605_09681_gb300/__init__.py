@@ -1,0 +1,189 @@
+"""Forcing-KV hot path on GB300: hybrid KV-cache compression (static structural pruning,
+segment-similarity pruning) and chunk attention over the compressed cache.
+
+Every step runs in the CUDA kernels of libfk.so behind the C ABI of include/fk.h; this
+module only marshals arguments (torch tensors for device memory and streams).
+"""
+from __future__ import annotations
+
+import ctypes
+
+import numpy as np
+
+from . import _lib as L
+from ._lib import FkError, KERNEL_KINDS, STATUS_NAMES
+
+__all__ = ["ForcingKVCache", "FkError", "KERNEL_KINDS", "STATUS_NAMES", "load_library"]
+
+
+def load_library():
+    return L.load()
+
+
+def _check(status: int, call: str) -> None:
+    if status != L.FK_OK:
+        raise FkError(status, call)
+
+
+def _ptr(x) -> int:
+    """Address of a bf16 tensor (torch, any device) or a uint16 numpy array of bf16 bits."""
+    import torch
+    if isinstance(x, torch.Tensor):
+        if x.dtype != torch.bfloat16 or not x.is_contiguous():
+            raise ValueError("expected a contiguous torch.bfloat16 tensor")
+        return x.data_ptr()
+    if isinstance(x, np.ndarray):
+        if x.dtype != np.uint16 or not x.flags["C_CONTIGUOUS"]:
+            raise ValueError("expected a C-contiguous uint16 array of bf16 bit patterns")
+        return x.ctypes.data
+    raise TypeError("unsupported tensor type %r" % type(x))
+
+
+def _numel(x) -> int:
+    return x.numel() if hasattr(x, "numel") and not isinstance(x, np.ndarray) else x.size
+
+
+def _stream(stream) -> int | None:
+    if stream is None:
+        import torch
+        if torch.cuda.is_available():
+            return torch.cuda.current_stream().cuda_stream
+        return None
+    return getattr(stream, "cuda_stream", stream)
+
+
+class ForcingKVCache:
+    """One Forcing-KV cache (all layers of a model) on one GPU.
+
+    Tensors are bf16 [tokens, n_heads, head_dim]; device or host memory.  Calls are
+    asynchronous on `stream` (default: torch's current stream)."""
+
+    def __init__(self, *, n_layers, n_heads, head_dim, tokens_per_frame, frames_per_chunk,
+                 n_sink_frames, window_frames, n_segments, keep_budget_permille,
+                 head_is_static, select_scope="per_frame", score_source="per_head",
+                 incremental=False, max_history_frames=64, device=0):
+        self._lib = L.load()
+        self._h = ctypes.c_void_p()
+        hm = np.ascontiguousarray(np.asarray(head_is_static, dtype=np.uint8).reshape(-1))
+        if hm.size != n_layers * n_heads:
+            raise ValueError("head_is_static must have n_layers * n_heads entries")
+        self._map = hm
+        self.cfg = L.FkConfig(
+            n_layers, n_heads, head_dim, tokens_per_frame, frames_per_chunk, n_sink_frames,
+            window_frames, n_segments, keep_budget_permille,
+            {"per_frame": L.FK_SCOPE_PER_FRAME, "pooled": L.FK_SCOPE_POOLED}[select_scope],
+            {"per_head": L.FK_SCORE_PER_HEAD, "layer0_pooled": L.FK_SCORE_LAYER0_POOLED}[score_source],
+            1 if incremental else 0, max_history_frames, device,
+            hm.ctypes.data_as(ctypes.POINTER(ctypes.c_uint8)))
+        self.n_layers, self.n_heads, self.head_dim = n_layers, n_heads, head_dim
+        self.F, self.C, self.n_segments = tokens_per_frame, frames_per_chunk, n_segments
+        self.device = device
+        _check(self._lib.fk_create(ctypes.byref(self.cfg), ctypes.byref(self._h)), "fk_create")
+
+    @classmethod
+    def from_workload(cls, w, head_is_static, device=0, **over):
+        kw = dict(n_layers=w.n_layers, n_heads=w.n_heads, head_dim=w.head_dim,
+                  tokens_per_frame=w.tokens_per_frame, frames_per_chunk=w.frames_per_chunk,
+                  n_sink_frames=w.n_sink_frames, window_frames=w.window_frames,
+                  n_segments=w.n_segments, keep_budget_permille=w.keep_budget_permille,
+                  head_is_static=head_is_static, select_scope=w.select_scope,
+                  score_source=w.score_source, incremental=w.incremental,
+                  max_history_frames=max(1, w.max_history_frames()), device=device)
+        kw.update(over)
+        return cls(**kw)
+
+    # ---- lifetime
+    def close(self):
+        if getattr(self, "_h", None) and self._h.value:
+            self._lib.fk_destroy(self._h)
+            self._h = ctypes.c_void_p()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.close()
+
+    # ---- cache updates
+    def append_frames(self, layer, K, V, stream=None):
+        nf = _numel(K) // (self.F * self.n_heads * self.head_dim)
+        _check(self._lib.fk_append_frames(self._h, layer, _ptr(K), _ptr(V), nf, _stream(stream)),
+               "fk_append_frames")
+
+    def append_chunk(self, layer, K, V, stream=None):
+        _check(self._lib.fk_append_chunk(self._h, layer, _ptr(K), _ptr(V), _stream(stream)),
+               "fk_append_chunk")
+
+    def set_current(self, layer, K, V, stream=None):
+        _check(self._lib.fk_set_current(self._h, layer, _ptr(K), _ptr(V), _stream(stream)),
+               "fk_set_current")
+
+    def compress(self, stream=None):
+        _check(self._lib.fk_compress(self._h, _stream(stream)), "fk_compress")
+
+    def attend(self, layer, Q, O=None, stream=None):
+        if O is None:
+            import torch
+            O = torch.empty_like(Q)
+        _check(self._lib.fk_attend(self._h, layer, _ptr(Q), _ptr(O), _stream(stream)), "fk_attend")
+        return O
+
+    # ---- inspection
+    def kept(self, layer, head, stream=None) -> list:
+        n = ctypes.c_int(0)
+        st = self._lib.fk_get_kept(self._h, layer, head, None, 0, ctypes.byref(n), _stream(stream))
+        if n.value == 0:
+            _check(st, "fk_get_kept")
+            return []
+        buf = (ctypes.c_int32 * n.value)()
+        _check(self._lib.fk_get_kept(self._h, layer, head, buf, n.value, ctypes.byref(n),
+                                     _stream(stream)), "fk_get_kept")
+        return list(buf)
+
+    def scores(self, layer, head, stream=None):
+        """(first_frame, fp32 array [n_frames, n_segments]) of the scoreable frames."""
+        first, nfr = ctypes.c_int(0), ctypes.c_int(0)
+        cap = 1 << 16
+        buf = np.zeros(cap, dtype=np.float32)
+        _check(self._lib.fk_get_scores(self._h, layer, head,
+                                       buf.ctypes.data_as(ctypes.POINTER(ctypes.c_float)), cap,
+                                       ctypes.byref(first), ctypes.byref(nfr), _stream(stream)),
+               "fk_get_scores")
+        return first.value, buf[: nfr.value * self.n_segments].reshape(nfr.value, self.n_segments).copy()
+
+    def key_count(self, layer, head) -> int:
+        n = ctypes.c_int(0)
+        _check(self._lib.fk_key_count(self._h, layer, head, ctypes.byref(n)), "fk_key_count")
+        return n.value
+
+    def cache_bytes(self) -> int:
+        return int(self._lib.fk_cache_bytes(self._h))
+
+    def reserved_bytes(self) -> int:
+        return int(self._lib.fk_reserved_bytes(self._h))
+
+    def sync_status(self, stream=None) -> int:
+        """Synchronize and return the device status (FK_OK, FK_ERR_RANGE, FK_ERR_TIMEOUT)."""
+        return int(self._lib.fk_sync_status(self._h, _stream(stream)))
+
+    # ---- timing
+    def profile_enable(self, on=True):
+        _check(self._lib.fk_profile_enable(self._h, 1 if on else 0), "fk_profile_enable")
+
+    def profile_reset(self):
+        _check(self._lib.fk_profile_reset(self._h), "fk_profile_reset")
+
+    def profile_read(self, kind: str):
+        ms, n = ctypes.c_double(0), ctypes.c_int64(0)
+        _check(self._lib.fk_profile_read(self._h, KERNEL_KINDS[kind], ctypes.byref(ms),
+                                         ctypes.byref(n)), "fk_profile_read")
+        return ms.value, n.value
+
+    def launch_count(self) -> int:
+        return int(self._lib.fk_launch_count(self._h))

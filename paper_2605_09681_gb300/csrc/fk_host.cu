@@ -1,0 +1,957 @@
+// Host side of the Forcing-KV library: configuration checks, device-memory layout,
+// frame bookkeeping (sink / window / anchor / scoreable frames, Sec. 4.2-4.3, App. H)
+// and the C ABI declared in fk.h.  All arithmetic of the method runs in the kernels
+// of fk_copy.cu, fk_score.cu and fk_attn.cu; this file only decides what to launch.
+//
+// Device memory (allocated once in fk_create, zero-initialised):
+//   view arenas  K and V, [rows][D] bf16 each; head (l, h) owns rows
+//                [row_base, row_base + view_rows), padded to whole 128-key tiles.
+//                Static head view:  [current chunk C*F | sink S*F | anchor F]
+//                Dynamic head view: [current chunk C*F | sink | kept segments | anchor F]
+//   page rings   K and V, [ring_slots][F][D] per head that keeps history for scoring
+//                (dynamic heads; every head of layer 0 under layer-0 pooled scoring);
+//                frame f lives in slot f (f < S) or S + (f - S) mod cap_nonsink.
+//   scores       fp32 [target][ring_slots][n]; kept lists int32 [target][kmax];
+//                scoring partials int64 (scratch); status word; host-input staging.
+#include <algorithm>
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <new>
+#include <vector>
+
+#include <cudaTypedefs.h>
+
+#include "fk_internal.h"
+
+using namespace fk;
+
+namespace {
+
+struct HeadBuf {
+  bool is_static = false;
+  bool retains = false;   // owns a page ring
+  bf16* pageK = nullptr;
+  bf16* pageV = nullptr;
+  bf16* viewK = nullptr;
+  bf16* viewV = nullptr;
+  int64_t row_base = 0;
+  int view_rows = 0;
+  int target = -1;        // selection target (dynamic heads)
+};
+
+struct LayerState {
+  int nh = 0;             // history frames appended
+  bool has_current = false;
+  bool dirty = false;     // appended since the last fk_compress
+  int scored_upto = 0;    // pairs (t, t+1) with t < scored_upto are scored
+  int n_keep = 0;         // kept segments of each dynamic head (after fk_compress)
+  int len_static = 0;     // keys of a static head
+  int len_dynamic = 0;    // keys of a dynamic head
+};
+
+struct ProfRec {
+  int kind;
+  cudaEvent_t a, b;
+};
+
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+std::once_flag g_encode_once;
+
+bool get_encode() {
+  std::call_once(g_encode_once, [] {
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  });
+  return g_encode != nullptr;
+}
+
+int64_t round_up(int64_t x, int64_t m) { return (x + m - 1) / m * m; }
+
+}  // namespace
+
+struct fk_handle {
+  fk_config cfg{};
+  std::vector<uint8_t> static_map;
+  int L = 0, H = 0, D = 0, F = 0, C = 0, S = 0, W = 0, n = 0, b = 0;
+  int scope = 0, source = 0, incremental = 0, max_hist = 0, dev = 0;
+  int seg = 0, CF = 0;
+  int cap_nonsink = 0, ring_slots = 0, k_frame = 0, kmax = 0, chunks = 0;
+  std::vector<HeadBuf> heads;      // [L*H]
+  std::vector<LayerState> layers;  // [L]
+  // device memory
+  std::vector<void*> allocs;
+  size_t reserved = 0;
+  bf16* viewK = nullptr;
+  bf16* viewV = nullptr;
+  int64_t view_rows_total = 0;
+  float* scores = nullptr;
+  int* kept = nullptr;
+  long long* partials = nullptr;
+  int* status = nullptr;
+  bf16* stage_q = nullptr;
+  bf16* stage_o = nullptr;
+  bf16* stage_k = nullptr;
+  bf16* stage_v = nullptr;
+  int64_t stage_frames = 0;        // frames one K/V staging buffer holds
+  ScoreItem* d_score_items = nullptr;
+  SelectTarget* d_targets = nullptr;
+  CompactItem* d_compact_items = nullptr;
+  std::vector<ScoreItem> score_items;
+  std::vector<SelectTarget> targets;
+  std::vector<int> target_layer;
+  std::vector<CompactItem> compact_items;
+  int max_run = 0;
+  CUtensorMap tmK{}, tmV{};
+  const void* q_cached = nullptr;
+  CUtensorMap tmQ{};
+  // profiling
+  bool prof = false;
+  std::vector<ProfRec> prof_pending;
+  std::vector<cudaEvent_t> ev_free;
+  double prof_ms[FK_KERNEL_KINDS] = {};
+  int64_t prof_n[FK_KERNEL_KINDS] = {};
+  int64_t launches = 0;
+};
+
+namespace {
+
+fk_status cuda_fail(cudaError_t e) {
+  return e == cudaErrorMemoryAllocation ? FK_ERR_NOMEM : FK_ERR_CUDA;
+}
+
+#define FK_CUDA(x)                                  \
+  do {                                              \
+    cudaError_t e_ = (x);                           \
+    if (e_ != cudaSuccess) return cuda_fail(e_);    \
+  } while (0)
+
+bool is_device_ptr(const void* p) {
+  cudaPointerAttributes at{};
+  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+int ring_slot(const fk_handle* h, int f) {
+  return f < h->S ? f : h->S + (f - h->S) % h->cap_nonsink;
+}
+
+struct Roles {
+  int n_sink;       // sink frames present
+  int lo;           // first window frame
+  int anchor;       // -1 = none
+  int t_lo;         // first scoreable frame
+  int n_scoreable;  // scoreable frames t_lo .. t_lo + n - 1
+};
+
+Roles roles_of(const fk_handle* h, int nh) {
+  Roles r{};
+  r.n_sink = std::min(h->S, nh);
+  r.lo = h->W > 0 ? std::max(h->S, nh - h->W) : h->S;
+  r.anchor = nh - 1 >= r.lo ? nh - 1 : -1;
+  r.t_lo = r.lo;
+  r.n_scoreable = r.anchor >= 0 ? r.anchor - r.lo : 0;
+  return r;
+}
+
+int keep_total(const fk_handle* h, int n_scoreable) {
+  if (h->scope == FK_SCOPE_PER_FRAME) return n_scoreable * h->k_frame;
+  return (int)(((int64_t)h->b * n_scoreable * h->n) / 1000);
+}
+
+void update_lengths(fk_handle* h, int l) {
+  LayerState& ls = h->layers[l];
+  const Roles r = roles_of(h, ls.nh);
+  const int base = h->CF + r.n_sink * h->F + (r.anchor >= 0 ? h->F : 0);
+  ls.len_static = base;
+  ls.len_dynamic = base + ls.n_keep * h->seg;
+}
+
+// ---- profiling and launch accounting
+void prof_begin(fk_handle* h, cudaStream_t s, cudaEvent_t* ev) {
+  *ev = nullptr;
+  if (!h->prof || h->ev_free.size() < 2) return;
+  *ev = h->ev_free.back();
+  h->ev_free.pop_back();
+  cudaEventRecord(*ev, s);
+}
+
+void prof_end(fk_handle* h, cudaStream_t s, int kind, cudaEvent_t ev0) {
+  h->launches++;
+  if (!ev0) return;
+  cudaEvent_t ev1 = h->ev_free.back();
+  h->ev_free.pop_back();
+  cudaEventRecord(ev1, s);
+  h->prof_pending.push_back({kind, ev0, ev1});
+}
+
+fk_status prof_collect(fk_handle* h) {
+  for (auto& r : h->prof_pending) {
+    FK_CUDA(cudaEventSynchronize(r.b));
+    float ms = 0.f;
+    FK_CUDA(cudaEventElapsedTime(&ms, r.a, r.b));
+    h->prof_ms[r.kind] += ms;
+    h->prof_n[r.kind] += 1;
+    h->ev_free.push_back(r.a);
+    h->ev_free.push_back(r.b);
+  }
+  h->prof_pending.clear();
+  return FK_OK;
+}
+
+template <class F>
+fk_status launch(fk_handle* h, cudaStream_t s, int kind, F&& f) {
+  cudaEvent_t ev0;
+  if (h->prof && h->ev_free.size() < 4) prof_collect(h);
+  prof_begin(h, s, &ev0);
+  f();
+  cudaError_t e = cudaGetLastError();
+  prof_end(h, s, kind, ev0);
+  return e == cudaSuccess ? FK_OK : FK_ERR_CUDA;
+}
+
+fk_status dev_alloc(fk_handle* h, size_t bytes, void** out) {
+  *out = nullptr;
+  if (bytes == 0) return FK_OK;
+  void* p = nullptr;
+  cudaError_t e = cudaMalloc(&p, bytes);
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    return cuda_fail(e);
+  }
+  h->allocs.push_back(p);
+  h->reserved += bytes;
+  e = cudaMemset(p, 0, bytes);
+  if (e != cudaSuccess) return FK_ERR_CUDA;
+  *out = p;
+  return FK_OK;
+}
+
+// Copy host input [rows][H][D] into staging when needed; returns the device pointer to use.
+fk_status stage_input(fk_handle* h, const void* src, bf16* stage, size_t bytes, cudaStream_t s,
+                      const bf16** out) {
+  if (is_device_ptr(src)) {
+    *out = static_cast<const bf16*>(src);
+    return FK_OK;
+  }
+  FK_CUDA(cudaMemcpyAsync(stage, src, bytes, cudaMemcpyHostToDevice, s));
+  *out = stage;
+  return FK_OK;
+}
+
+fk_status encode_2d(CUtensorMap* m, void* base, int64_t rows, int D) {
+  const cuuint64_t dims[2] = {(cuuint64_t)D, (cuuint64_t)rows};
+  const cuuint64_t strides[1] = {(cuuint64_t)D * 2};
+  const cuuint32_t box[2] = {64, (cuuint32_t)kAttnBN};
+  const cuuint32_t es[2] = {1, 1};
+  CUresult r = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, dims, strides, box, es,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? FK_OK : FK_ERR_CUDA;
+}
+
+fk_status encode_q(CUtensorMap* m, const void* q, int Nq, int H, int D) {
+  const cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)H, (cuuint64_t)Nq};
+  const cuuint64_t strides[2] = {(cuuint64_t)D * 2, (cuuint64_t)H * D * 2};
+  const cuuint32_t box[3] = {64, 1, (cuuint32_t)kAttnBM};
+  const cuuint32_t es[3] = {1, 1, 1};
+  CUresult r = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(q), dims,
+                        strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? FK_OK : FK_ERR_CUDA;
+}
+
+// Move frames of `layer` into history.  K/V sources are per-head row-major views
+// (src_per_head = true: headK[h] + i*F*D) or token-major [nf*F][H][D] device buffers.
+fk_status push_history(fk_handle* h, int layer, const bf16* const* headK, const bf16* const* headV,
+                       const bf16* tokK, const bf16* tokV, int nf, cudaStream_t s) {
+  LayerState& ls = h->layers[layer];
+  const int nh0 = ls.nh, nh1 = ls.nh + nf;
+  const int lo1 = h->W > 0 ? std::max(h->S, nh1 - h->W) : h->S;   // window after the push
+  const int64_t frame_elems = (int64_t)h->F * h->D;
+  CopyJobs jobs;
+  jobs.n = 0;
+  auto flush = [&]() -> fk_status {
+    fk_status st = launch(h, s, FK_KERNEL_APPEND, [&] { launch_copy_jobs(jobs, s); });
+    jobs.n = 0;
+    return st;
+  };
+  for (int i = 0; i < nf; ++i) {
+    const int f = nh0 + i;
+    const bool sink = f < h->S;
+    const bool in_window = sink || f >= lo1;        // frames overwritten within this push are skipped
+    const bool is_anchor = !sink && f == nh1 - 1;
+    if (!in_window) continue;
+    if (tokK) {
+      ScatterArgs pa{}, va{};
+      pa.srcK = tokK + (int64_t)i * h->F * h->H * h->D;
+      pa.srcV = tokV + (int64_t)i * h->F * h->H * h->D;
+      pa.rows = h->F;
+      pa.heads = h->H;
+      pa.head_dim = h->D;
+      va = pa;
+      bool any_p = false, any_v = false;
+      for (int hd = 0; hd < h->H; ++hd) {
+        const HeadBuf& hb = h->heads[layer * h->H + hd];
+        if (hb.retains) {
+          pa.dstK[hd] = hb.pageK + ring_slot(h, f) * frame_elems;
+          pa.dstV[hd] = hb.pageV + ring_slot(h, f) * frame_elems;
+          any_p = true;
+        }
+        if (hb.is_static && (sink || is_anchor)) {
+          const int64_t row = h->CF + (int64_t)(sink ? f : h->S) * h->F;
+          va.dstK[hd] = hb.viewK + row * h->D;
+          va.dstV[hd] = hb.viewV + row * h->D;
+          any_v = true;
+        }
+      }
+      if (any_p) {
+        fk_status st = launch(h, s, FK_KERNEL_APPEND, [&] { launch_scatter(pa, s); });
+        if (st != FK_OK) return st;
+      }
+      if (any_v) {
+        fk_status st = launch(h, s, FK_KERNEL_APPEND, [&] { launch_scatter(va, s); });
+        if (st != FK_OK) return st;
+      }
+    } else {
+      for (int hd = 0; hd < h->H; ++hd) {
+        const HeadBuf& hb = h->heads[layer * h->H + hd];
+        const bf16* sk = headK[hd] + i * frame_elems;
+        const bf16* sv = headV[hd] + i * frame_elems;
+        auto add = [&](bf16* dk, bf16* dv) -> fk_status {
+          if (jobs.n + 2 > kMaxCopyJobs) {
+            fk_status st = flush();
+            if (st != FK_OK) return st;
+          }
+          jobs.job[jobs.n++] = {sk, dk, frame_elems * 2};
+          jobs.job[jobs.n++] = {sv, dv, frame_elems * 2};
+          return FK_OK;
+        };
+        if (hb.retains) {
+          fk_status st = add(hb.pageK + ring_slot(h, f) * frame_elems,
+                             hb.pageV + ring_slot(h, f) * frame_elems);
+          if (st != FK_OK) return st;
+        }
+        if (hb.is_static && (sink || is_anchor)) {
+          const int64_t row = h->CF + (int64_t)(sink ? f : h->S) * h->F;
+          fk_status st = add(hb.viewK + row * h->D, hb.viewV + row * h->D);
+          if (st != FK_OK) return st;
+        }
+      }
+    }
+  }
+  if (jobs.n) {
+    fk_status st = flush();
+    if (st != FK_OK) return st;
+  }
+  ls.nh = nh1;
+  ls.dirty = true;
+  update_lengths(h, layer);
+  return FK_OK;
+}
+
+// The current chunk (view fronts) joins the history.
+fk_status retire_current(fk_handle* h, int layer, cudaStream_t s) {
+  LayerState& ls = h->layers[layer];
+  if (!ls.has_current) return FK_OK;
+  if (h->W == 0 && ls.nh + h->C > h->max_hist) return FK_ERR_FULL;
+  std::vector<const bf16*> hk(h->H), hv(h->H);
+  for (int hd = 0; hd < h->H; ++hd) {
+    hk[hd] = h->heads[layer * h->H + hd].viewK;
+    hv[hd] = h->heads[layer * h->H + hd].viewV;
+  }
+  fk_status st = push_history(h, layer, hk.data(), hv.data(), nullptr, nullptr, h->C, s);
+  if (st != FK_OK) return st;
+  ls.has_current = false;
+  return FK_OK;
+}
+
+fk_status write_current(fk_handle* h, int layer, const void* K, const void* V, cudaStream_t s) {
+  const size_t bytes = (size_t)h->CF * h->H * h->D * 2;
+  const bf16 *k, *v;
+  fk_status st = stage_input(h, K, h->stage_k, bytes, s, &k);
+  if (st != FK_OK) return st;
+  st = stage_input(h, V, h->stage_v, bytes, s, &v);
+  if (st != FK_OK) return st;
+  ScatterArgs a{};
+  a.srcK = k;
+  a.srcV = v;
+  a.rows = h->CF;
+  a.heads = h->H;
+  a.head_dim = h->D;
+  for (int hd = 0; hd < h->H; ++hd) {
+    a.dstK[hd] = h->heads[layer * h->H + hd].viewK;
+    a.dstV[hd] = h->heads[layer * h->H + hd].viewV;
+  }
+  st = launch(h, s, FK_KERNEL_APPEND, [&] { launch_scatter(a, s); });
+  if (st != FK_OK) return st;
+  h->layers[layer].has_current = true;
+  update_lengths(h, layer);
+  return FK_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int fk_abi_version(void) { return 1; }
+
+const char* fk_status_str(fk_status s) {
+  switch (s) {
+    case FK_OK: return "ok";
+    case FK_ERR_CONFIG: return "invalid configuration";
+    case FK_ERR_ARG: return "invalid argument";
+    case FK_ERR_STATE: return "call out of order";
+    case FK_ERR_FULL: return "history capacity exceeded";
+    case FK_ERR_RANGE: return "scoring precondition violated (token squared key norm > 2^23)";
+    case FK_ERR_TIMEOUT: return "bounded device wait expired";
+    case FK_ERR_CUDA: return "CUDA error";
+    case FK_ERR_NOMEM: return "out of device memory";
+  }
+  return "unknown status";
+}
+
+fk_status fk_validate_config(const fk_config* c) {
+  if (!c || !c->head_is_static) return FK_ERR_ARG;
+  if (c->n_layers < 1 || c->n_layers > kMaxLayers) return FK_ERR_CONFIG;
+  if (c->n_heads < 1 || c->n_heads > kMaxHeads) return FK_ERR_CONFIG;
+  if (c->head_dim != 64 && c->head_dim != 128) return FK_ERR_CONFIG;
+  if (c->tokens_per_frame < 1 || c->n_segments < 1 || c->tokens_per_frame % c->n_segments)
+    return FK_ERR_CONFIG;
+  if (c->frames_per_chunk < 1 || c->n_sink_frames < 0 || c->window_frames < 0) return FK_ERR_CONFIG;
+  if (c->keep_budget_permille < 0 || c->keep_budget_permille > 1000) return FK_ERR_CONFIG;
+  if (c->select_scope != FK_SCOPE_PER_FRAME && c->select_scope != FK_SCOPE_POOLED) return FK_ERR_CONFIG;
+  if (c->score_source != FK_SCORE_PER_HEAD && c->score_source != FK_SCORE_LAYER0_POOLED)
+    return FK_ERR_CONFIG;
+  if (c->incremental != 0 && c->incremental != 1) return FK_ERR_CONFIG;
+  if (c->window_frames == 0 && c->max_history_frames < 1) return FK_ERR_CONFIG;
+  const int64_t cf = (int64_t)c->frames_per_chunk * c->tokens_per_frame;
+  if (cf > (1 << 24) || (int64_t)c->tokens_per_frame * c->head_dim > (1 << 28)) return FK_ERR_CONFIG;
+  const int64_t cap = c->window_frames > 0 ? c->window_frames
+                                           : std::max(0, c->max_history_frames - c->n_sink_frames);
+  if (cap > 4096 || c->n_sink_frames > 4096) return FK_ERR_CONFIG;
+  return FK_OK;
+}
+
+fk_status fk_create(const fk_config* cfg, fk_handle** out) {
+  if (!out) return FK_ERR_ARG;
+  *out = nullptr;
+  fk_status st = fk_validate_config(cfg);
+  if (st != FK_OK) return st;
+  fk_handle* h = new (std::nothrow) fk_handle();
+  if (!h) return FK_ERR_NOMEM;
+  h->cfg = *cfg;
+  h->L = cfg->n_layers;
+  h->H = cfg->n_heads;
+  h->D = cfg->head_dim;
+  h->F = cfg->tokens_per_frame;
+  h->C = cfg->frames_per_chunk;
+  h->S = cfg->n_sink_frames;
+  h->W = cfg->window_frames;
+  h->n = cfg->n_segments;
+  h->b = cfg->keep_budget_permille;
+  h->scope = cfg->select_scope;
+  h->source = cfg->score_source;
+  h->incremental = cfg->incremental;
+  h->max_hist = cfg->max_history_frames;
+  h->dev = cfg->device;
+  h->seg = h->F / h->n;
+  h->CF = h->C * h->F;
+  h->static_map.assign(cfg->head_is_static, cfg->head_is_static + (size_t)h->L * h->H);
+  h->cfg.head_is_static = h->static_map.data();
+  h->cap_nonsink = h->W > 0 ? h->W : std::max(0, h->max_hist - h->S);
+  if (h->cap_nonsink < 1) h->cap_nonsink = 1;
+  h->ring_slots = h->S + h->cap_nonsink;
+  h->k_frame = (h->b * h->n) / 1000;
+  h->kmax = std::max(1, keep_total(h, h->cap_nonsink - 1));
+  h->chunks = (h->seg + kScoreTokens - 1) / kScoreTokens;
+  h->max_run = h->cap_nonsink;
+  h->heads.resize((size_t)h->L * h->H);
+  h->layers.resize(h->L);
+
+  auto fail = [&](fk_status s) {
+    fk_destroy(h);
+    return s;
+  };
+  if (cudaSetDevice(h->dev) != cudaSuccess) {
+    cudaGetLastError();
+    return fail(FK_ERR_CUDA);
+  }
+  if (!get_encode()) return fail(FK_ERR_CUDA);
+  if (attention_prepare(h->D) != cudaSuccess) return fail(FK_ERR_CUDA);
+
+  // heads: roles, view rows, targets
+  int n_dynamic = 0;
+  for (int l = 0; l < h->L; ++l)
+    for (int hd = 0; hd < h->H; ++hd) {
+      HeadBuf& hb = h->heads[l * h->H + hd];
+      hb.is_static = h->static_map[l * h->H + hd] != 0;
+      hb.retains = !hb.is_static || (h->source == FK_SCORE_LAYER0_POOLED && l == 0);
+      const int64_t rows = hb.is_static
+                               ? (int64_t)h->CF + (int64_t)h->S * h->F + h->F
+                               : (int64_t)h->CF + (int64_t)h->S * h->F + (int64_t)h->kmax * h->seg + h->F;
+      hb.view_rows = (int)round_up(rows, kViewAlignRows);
+      hb.row_base = h->view_rows_total;
+      h->view_rows_total += hb.view_rows;
+      n_dynamic += !hb.is_static;
+    }
+  if (h->view_rows_total >= (int64_t)1 << 31) return fail(FK_ERR_CONFIG);
+  if (h->source == FK_SCORE_LAYER0_POOLED) {
+    h->targets.push_back({0, 0, h->H});
+    h->target_layer.push_back(0);
+    for (int hd = 0; hd < h->H; ++hd) h->score_items.push_back({nullptr, 0, 0});
+    for (auto& hb : h->heads)
+      if (!hb.is_static) hb.target = 0;
+  } else {
+    for (int l = 0; l < h->L; ++l)
+      for (int hd = 0; hd < h->H; ++hd) {
+        HeadBuf& hb = h->heads[l * h->H + hd];
+        if (hb.is_static) continue;
+        hb.target = (int)h->targets.size();
+        h->targets.push_back({l, (int)h->score_items.size(), 1});
+        h->target_layer.push_back(l);
+        h->score_items.push_back({nullptr, l, hb.target});
+      }
+  }
+
+  // allocations
+  void* p = nullptr;
+  const size_t view_bytes = (size_t)h->view_rows_total * h->D * 2;
+  if ((st = dev_alloc(h, view_bytes, &p)) != FK_OK) return fail(st);
+  h->viewK = static_cast<bf16*>(p);
+  if ((st = dev_alloc(h, view_bytes, &p)) != FK_OK) return fail(st);
+  h->viewV = static_cast<bf16*>(p);
+  size_t n_ret = 0;
+  for (auto& hb : h->heads) n_ret += hb.retains;
+  const size_t ring_elems = (size_t)h->ring_slots * h->F * h->D;
+  bf16* pages = nullptr;
+  if (n_ret) {
+    if ((st = dev_alloc(h, n_ret * ring_elems * 2 * 2, &p)) != FK_OK) return fail(st);
+    pages = static_cast<bf16*>(p);
+  }
+  size_t ri = 0;
+  for (auto& hb : h->heads) {
+    hb.viewK = h->viewK + hb.row_base * h->D;
+    hb.viewV = h->viewV + hb.row_base * h->D;
+    if (hb.retains) {
+      hb.pageK = pages + (2 * ri) * ring_elems;
+      hb.pageV = pages + (2 * ri + 1) * ring_elems;
+      ++ri;
+    }
+  }
+  const size_t nt = std::max<size_t>(1, h->targets.size());
+  if ((st = dev_alloc(h, nt * h->ring_slots * h->n * sizeof(float), &p)) != FK_OK) return fail(st);
+  h->scores = static_cast<float*>(p);
+  if ((st = dev_alloc(h, nt * h->kmax * sizeof(int), &p)) != FK_OK) return fail(st);
+  h->kept = static_cast<int*>(p);
+  const size_t n_items = std::max<size_t>(1, h->score_items.size());
+  if ((st = dev_alloc(h, n_items * h->max_run * h->n * h->chunks * 2 * sizeof(long long), &p)) != FK_OK)
+    return fail(st);
+  h->partials = static_cast<long long*>(p);
+  if ((st = dev_alloc(h, 256, &p)) != FK_OK) return fail(st);
+  h->status = static_cast<int*>(p);
+  const size_t chunk_bytes = (size_t)h->CF * h->H * h->D * 2;
+  if ((st = dev_alloc(h, chunk_bytes, &p)) != FK_OK) return fail(st);
+  h->stage_q = static_cast<bf16*>(p);
+  if ((st = dev_alloc(h, chunk_bytes, &p)) != FK_OK) return fail(st);
+  h->stage_o = static_cast<bf16*>(p);
+  if ((st = dev_alloc(h, chunk_bytes, &p)) != FK_OK) return fail(st);
+  h->stage_k = static_cast<bf16*>(p);
+  if ((st = dev_alloc(h, chunk_bytes, &p)) != FK_OK) return fail(st);
+  h->stage_v = static_cast<bf16*>(p);
+  h->stage_frames = h->C;
+
+  // static device tables
+  if (h->source == FK_SCORE_LAYER0_POOLED) {
+    for (int hd = 0; hd < h->H; ++hd) h->score_items[hd].pagesK = h->heads[hd].pageK;
+  } else {
+    for (auto& si : h->score_items) {
+      for (int hd = 0; hd < h->H; ++hd) {
+        const HeadBuf& hb = h->heads[si.layer * h->H + hd];
+        if (hb.target == si.target) si.pagesK = hb.pageK;
+      }
+    }
+  }
+  for (int l = 0; l < h->L; ++l)
+    for (int hd = 0; hd < h->H; ++hd) {
+      const HeadBuf& hb = h->heads[l * h->H + hd];
+      if (hb.is_static) continue;
+      h->compact_items.push_back({hb.pageK, hb.pageV, hb.viewK, hb.viewV, l, hb.target});
+    }
+  auto upload = [&](const void* src, size_t bytes, void** dst) -> fk_status {
+    fk_status s2 = dev_alloc(h, std::max<size_t>(bytes, 16), dst);
+    if (s2 != FK_OK) return s2;
+    if (bytes && cudaMemcpy(*dst, src, bytes, cudaMemcpyHostToDevice) != cudaSuccess) return FK_ERR_CUDA;
+    return FK_OK;
+  };
+  if ((st = upload(h->score_items.data(), h->score_items.size() * sizeof(ScoreItem), &p)) != FK_OK)
+    return fail(st);
+  h->d_score_items = static_cast<ScoreItem*>(p);
+  if ((st = upload(h->targets.data(), h->targets.size() * sizeof(SelectTarget), &p)) != FK_OK)
+    return fail(st);
+  h->d_targets = static_cast<SelectTarget*>(p);
+  if ((st = upload(h->compact_items.data(), h->compact_items.size() * sizeof(CompactItem), &p)) != FK_OK)
+    return fail(st);
+  h->d_compact_items = static_cast<CompactItem*>(p);
+
+  if ((st = encode_2d(&h->tmK, h->viewK, h->view_rows_total, h->D)) != FK_OK) return fail(st);
+  if ((st = encode_2d(&h->tmV, h->viewV, h->view_rows_total, h->D)) != FK_OK) return fail(st);
+  if (cudaDeviceSynchronize() != cudaSuccess) return fail(FK_ERR_CUDA);
+  for (int l = 0; l < h->L; ++l) update_lengths(h, l);
+  *out = h;
+  return FK_OK;
+}
+
+void fk_destroy(fk_handle* h) {
+  if (!h) return;
+  cudaSetDevice(h->dev);
+  cudaDeviceSynchronize();
+  for (auto& r : h->prof_pending) {
+    cudaEventDestroy(r.a);
+    cudaEventDestroy(r.b);
+  }
+  for (auto e : h->ev_free) cudaEventDestroy(e);
+  for (void* p : h->allocs) cudaFree(p);
+  cudaGetLastError();
+  delete h;
+}
+
+static fk_status check_layer(const fk_handle* h, int layer) {
+  if (!h) return FK_ERR_ARG;
+  if (layer < 0 || layer >= h->L) return FK_ERR_ARG;
+  return FK_OK;
+}
+
+fk_status fk_append_frames(fk_handle* h, int layer, const void* K, const void* V, int n_frames,
+                           void* stream) {
+  fk_status st = check_layer(h, layer);
+  if (st != FK_OK) return st;
+  if (n_frames < 0 || (n_frames > 0 && (!K || !V))) return FK_ERR_ARG;
+  if (n_frames > 0 && (!aligned16(K) || !aligned16(V))) return FK_ERR_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  FK_CUDA(cudaSetDevice(h->dev));
+  LayerState& ls = h->layers[layer];
+  const int extra = ls.has_current ? h->C : 0;
+  if (h->W == 0 && ls.nh + extra + n_frames > h->max_hist) return FK_ERR_FULL;
+  if ((st = retire_current(h, layer, s)) != FK_OK) return st;
+  const bool dev_in = n_frames > 0 && is_device_ptr(K) && is_device_ptr(V);
+  const size_t frame_bytes = (size_t)h->F * h->H * h->D * 2;
+  for (int f0 = 0; f0 < n_frames;) {
+    const int nf = dev_in ? n_frames : (int)std::min<int64_t>(h->stage_frames, n_frames - f0);
+    const bf16* k = static_cast<const bf16*>(K) + (size_t)f0 * frame_bytes / 2;
+    const bf16* v = static_cast<const bf16*>(V) + (size_t)f0 * frame_bytes / 2;
+    if (!dev_in) {
+      FK_CUDA(cudaMemcpyAsync(h->stage_k, k, nf * frame_bytes, cudaMemcpyHostToDevice, s));
+      FK_CUDA(cudaMemcpyAsync(h->stage_v, v, nf * frame_bytes, cudaMemcpyHostToDevice, s));
+      k = h->stage_k;
+      v = h->stage_v;
+    }
+    if ((st = push_history(h, layer, nullptr, nullptr, k, v, nf, s)) != FK_OK) return st;
+    f0 += nf;
+  }
+  ls.dirty = true;
+  return FK_OK;
+}
+
+fk_status fk_append_chunk(fk_handle* h, int layer, const void* K, const void* V, void* stream) {
+  fk_status st = check_layer(h, layer);
+  if (st != FK_OK) return st;
+  if (!K || !V || !aligned16(K) || !aligned16(V)) return FK_ERR_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  FK_CUDA(cudaSetDevice(h->dev));
+  if ((st = retire_current(h, layer, s)) != FK_OK) return st;
+  if ((st = write_current(h, layer, K, V, s)) != FK_OK) return st;
+  h->layers[layer].dirty = true;
+  return FK_OK;
+}
+
+fk_status fk_set_current(fk_handle* h, int layer, const void* K, const void* V, void* stream) {
+  fk_status st = check_layer(h, layer);
+  if (st != FK_OK) return st;
+  if (!K || !V || !aligned16(K) || !aligned16(V)) return FK_ERR_ARG;
+  FK_CUDA(cudaSetDevice(h->dev));
+  return write_current(h, layer, K, V, static_cast<cudaStream_t>(stream));
+}
+
+fk_status fk_compress(fk_handle* h, void* stream) {
+  if (!h) return FK_ERR_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  FK_CUDA(cudaSetDevice(h->dev));
+  bool any = false;
+  for (auto& ls : h->layers) any |= ls.dirty;
+  if (!any) return FK_OK;
+  const bool pooled_src = h->source == FK_SCORE_LAYER0_POOLED;
+  if (pooled_src) {
+    for (int l = 1; l < h->L; ++l)
+      if (h->layers[l].nh != h->layers[0].nh) return FK_ERR_STATE;
+  }
+  ScoreArgs sa{};
+  SelectArgs se{};
+  CompactArgs ca{};
+  bool any_run = false, any_select = false, any_compact = false;
+  for (int l = 0; l < h->L; ++l) {
+    LayerState& ls = h->layers[l];
+    const Roles r = roles_of(h, ls.nh);
+    const int keep = keep_total(h, r.n_scoreable);
+    // scoring run of the layer whose keys score (every layer per head; layer 0 pooled)
+    const bool scores_here = pooled_src ? l == 0 : true;
+    if (ls.dirty && scores_here) {
+      int t_first = h->incremental ? std::max(r.t_lo, ls.scored_upto) : r.t_lo;
+      const int last_t = r.t_lo + r.n_scoreable - 1;
+      if (r.n_scoreable > 0 && t_first <= last_t) {
+        sa.run[l] = {t_first, last_t + 2 - t_first};
+        any_run = true;
+      }
+      ls.scored_upto = r.anchor >= 0 ? r.anchor : ls.scored_upto;
+    }
+    se.run[l] = sa.run[l];
+    se.t_lo[l] = r.t_lo;
+    se.n_scoreable[l] = r.n_scoreable;
+    se.n_keep[l] = keep;
+    if (ls.dirty && r.n_scoreable > 0 && scores_here) any_select = true;
+    ca.n_sink_present[l] = r.n_sink;
+    ca.n_keep[l] = keep;
+    ca.anchor[l] = r.anchor;
+    ca.active[l] = ls.dirty ? 1 : 0;
+    const int units = r.n_sink * h->n + keep + (r.anchor >= 0 ? h->n : 0);
+    ca.max_units = std::max(ca.max_units, ls.dirty ? units : 0);
+  }
+  for (const auto& ci : h->compact_items) any_compact |= ca.active[ci.layer] != 0;
+  fk_status st;
+  if (any_run) {
+    sa.items = h->d_score_items;
+    sa.n_items = (int)h->score_items.size();
+    sa.F = h->F;
+    sa.D = h->D;
+    sa.n_seg = h->n;
+    sa.seg_len = h->seg;
+    sa.chunks = h->chunks;
+    sa.S = h->S;
+    sa.cap_nonsink = h->cap_nonsink;
+    sa.max_run = h->max_run;
+    sa.partials = h->partials;
+    sa.status = h->status;
+    if ((st = launch(h, s, FK_KERNEL_SCORE, [&] { launch_score(sa, s); })) != FK_OK) return st;
+  }
+  if (any_select && !h->targets.empty()) {
+    se.targets = h->d_targets;
+    se.n_targets = (int)h->targets.size();
+    se.n_seg = h->n;
+    se.chunks = h->chunks;
+    se.max_run = h->max_run;
+    se.S = h->S;
+    se.cap_nonsink = h->cap_nonsink;
+    se.ring_slots = h->ring_slots;
+    se.scope = h->scope;
+    se.k_frame = h->k_frame;
+    se.kmax = h->kmax;
+    se.partials = h->partials;
+    se.scores = h->scores;
+    se.kept = h->kept;
+    if ((st = launch(h, s, FK_KERNEL_SELECT, [&] { launch_select(se, s); })) != FK_OK) return st;
+  }
+  if (any_compact && ca.max_units > 0) {
+    ca.items = h->d_compact_items;
+    ca.n_items = (int)h->compact_items.size();
+    ca.F = h->F;
+    ca.D = h->D;
+    ca.n_seg = h->n;
+    ca.seg_len = h->seg;
+    ca.CF = h->CF;
+    ca.S = h->S;
+    ca.cap_nonsink = h->cap_nonsink;
+    ca.kmax = h->kmax;
+    ca.kept = h->kept;
+    if ((st = launch(h, s, FK_KERNEL_COMPACT, [&] { launch_compact(ca, s); })) != FK_OK) return st;
+  }
+  for (int l = 0; l < h->L; ++l) {
+    LayerState& ls = h->layers[l];
+    if (!ls.dirty) continue;
+    ls.n_keep = ca.n_keep[l];
+    ls.dirty = false;
+    update_lengths(h, l);
+  }
+  return FK_OK;
+}
+
+fk_status fk_attend(fk_handle* h, int layer, const void* Q, void* O, void* stream) {
+  fk_status st = check_layer(h, layer);
+  if (st != FK_OK) return st;
+  if (!Q || !O || !aligned16(Q) || !aligned16(O)) return FK_ERR_ARG;
+  const LayerState& ls = h->layers[layer];
+  if (!ls.has_current || ls.dirty) return FK_ERR_STATE;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  FK_CUDA(cudaSetDevice(h->dev));
+  const size_t bytes = (size_t)h->CF * h->H * h->D * 2;
+  const bf16* q;
+  if ((st = stage_input(h, Q, h->stage_q, bytes, s, &q)) != FK_OK) return st;
+  const bool dev_out = is_device_ptr(O);
+  bf16* o = dev_out ? static_cast<bf16*>(O) : h->stage_o;
+  if (q != h->q_cached) {
+    if ((st = encode_q(&h->tmQ, q, h->CF, h->H, h->D)) != FK_OK) return st;
+    h->q_cached = q;
+  }
+  AttnArgs a{};
+  a.O = o;
+  a.Nq = h->CF;
+  a.H = h->H;
+  a.n_qtiles = (h->CF + kAttnBM - 1) / kAttnBM;
+  a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)h->D));
+  a.status = h->status;
+  std::vector<int> order(h->H);
+  for (int hd = 0; hd < h->H; ++hd) {
+    const HeadBuf& hb = h->heads[layer * h->H + hd];
+    a.row_base[hd] = (int)hb.row_base;
+    a.n_keys[hd] = hb.is_static ? ls.len_static : ls.len_dynamic;
+    order[hd] = hd;
+  }
+  std::stable_sort(order.begin(), order.end(),
+                   [&](int x, int y) { return a.n_keys[x] > a.n_keys[y]; });
+  for (int i = 0; i < h->H; ++i) a.head_of[i] = order[i];
+  const int D = h->D;
+  if ((st = launch(h, s, FK_KERNEL_ATTEND,
+                   [&] { launch_attention(D, h->tmQ, h->tmK, h->tmV, a, s); })) != FK_OK)
+    return st;
+  if (!dev_out) FK_CUDA(cudaMemcpyAsync(O, o, bytes, cudaMemcpyDeviceToHost, s));
+  return FK_OK;
+}
+
+size_t fk_cache_bytes(const fk_handle* h) {
+  if (!h) return 0;
+  size_t bytes = 0;
+  const size_t frame_bytes = (size_t)h->F * h->D * 2 * 2;   // K and V
+  for (int l = 0; l < h->L; ++l) {
+    const LayerState& ls = h->layers[l];
+    const Roles r = roles_of(h, ls.nh);
+    const int live_frames = r.n_sink + (ls.nh - r.lo > 0 ? ls.nh - r.lo : 0);
+    for (int hd = 0; hd < h->H; ++hd) {
+      const HeadBuf& hb = h->heads[l * h->H + hd];
+      if (hb.retains) bytes += (size_t)live_frames * frame_bytes;
+      const int rows = hb.is_static ? ls.len_static : ls.len_dynamic;
+      bytes += (size_t)rows * h->D * 2 * 2;
+    }
+  }
+  bytes += h->targets.size() * ((size_t)h->ring_slots * h->n * sizeof(float) + h->kmax * sizeof(int));
+  return bytes;
+}
+
+size_t fk_reserved_bytes(const fk_handle* h) { return h ? h->reserved : 0; }
+
+fk_status fk_key_count(const fk_handle* h, int layer, int head, int* n_keys) {
+  fk_status st = check_layer(h, layer);
+  if (st != FK_OK) return st;
+  if (head < 0 || head >= h->H || !n_keys) return FK_ERR_ARG;
+  const LayerState& ls = h->layers[layer];
+  *n_keys = h->heads[layer * h->H + head].is_static ? ls.len_static : ls.len_dynamic;
+  return FK_OK;
+}
+
+fk_status fk_get_kept(fk_handle* h, int layer, int head, int32_t* out, int capacity, int* n_out,
+                      void* stream) {
+  fk_status st = check_layer(h, layer);
+  if (st != FK_OK) return st;
+  if (head < 0 || head >= h->H || !n_out) return FK_ERR_ARG;
+  const HeadBuf& hb = h->heads[layer * h->H + head];
+  if (hb.is_static) {
+    *n_out = 0;
+    return FK_OK;
+  }
+  const int n = h->layers[layer].n_keep;
+  *n_out = n;
+  if (capacity < n || (n > 0 && !out)) return FK_ERR_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  FK_CUDA(cudaSetDevice(h->dev));
+  if (n > 0)
+    FK_CUDA(cudaMemcpyAsync(out, h->kept + (size_t)hb.target * h->kmax, n * sizeof(int),
+                            cudaMemcpyDeviceToHost, s));
+  FK_CUDA(cudaStreamSynchronize(s));
+  return FK_OK;
+}
+
+fk_status fk_get_scores(fk_handle* h, int layer, int head, float* out, int capacity,
+                        int* first_frame, int* n_frames, void* stream) {
+  fk_status st = check_layer(h, layer);
+  if (st != FK_OK) return st;
+  if (head < 0 || head >= h->H || !first_frame || !n_frames) return FK_ERR_ARG;
+  const HeadBuf& hb = h->heads[layer * h->H + head];
+  const int sl = h->source == FK_SCORE_LAYER0_POOLED ? 0 : layer;
+  const Roles r = roles_of(h, h->layers[sl].nh);
+  *first_frame = r.t_lo;
+  *n_frames = hb.is_static ? 0 : r.n_scoreable;
+  if (hb.is_static || r.n_scoreable == 0) return FK_OK;
+  if (!out || capacity < r.n_scoreable * h->n) return FK_ERR_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  FK_CUDA(cudaSetDevice(h->dev));
+  std::vector<float> all((size_t)h->ring_slots * h->n);
+  FK_CUDA(cudaMemcpyAsync(all.data(), h->scores + (size_t)hb.target * h->ring_slots * h->n,
+                          all.size() * sizeof(float), cudaMemcpyDeviceToHost, s));
+  FK_CUDA(cudaStreamSynchronize(s));
+  for (int i = 0; i < r.n_scoreable; ++i) {
+    const int slot = ring_slot(h, r.t_lo + i);
+    std::memcpy(out + (size_t)i * h->n, all.data() + (size_t)slot * h->n, h->n * sizeof(float));
+  }
+  return FK_OK;
+}
+
+fk_status fk_sync_status(fk_handle* h, void* stream) {
+  if (!h) return FK_ERR_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  FK_CUDA(cudaSetDevice(h->dev));
+  int word = 0;
+  FK_CUDA(cudaMemcpyAsync(&word, h->status, sizeof(int), cudaMemcpyDeviceToHost, s));
+  FK_CUDA(cudaStreamSynchronize(s));
+  if (word) FK_CUDA(cudaMemset(h->status, 0, sizeof(int)));
+  if (word & kStatusTimeout) return FK_ERR_TIMEOUT;
+  if (word & kStatusRange) return FK_ERR_RANGE;
+  return FK_OK;
+}
+
+fk_status fk_profile_enable(fk_handle* h, int on) {
+  if (!h) return FK_ERR_ARG;
+  FK_CUDA(cudaSetDevice(h->dev));
+  if (on && h->ev_free.empty() && h->prof_pending.empty()) {
+    for (int i = 0; i < 1024; ++i) {
+      cudaEvent_t e;
+      FK_CUDA(cudaEventCreate(&e));
+      h->ev_free.push_back(e);
+    }
+  }
+  h->prof = on != 0;
+  return FK_OK;
+}
+
+fk_status fk_profile_read(fk_handle* h, int kind, double* total_ms, int64_t* launches) {
+  if (!h || kind < 0 || kind >= FK_KERNEL_KINDS || !total_ms || !launches) return FK_ERR_ARG;
+  FK_CUDA(cudaSetDevice(h->dev));
+  fk_status st = prof_collect(h);
+  if (st != FK_OK) return st;
+  *total_ms = h->prof_ms[kind];
+  *launches = h->prof_n[kind];
+  return FK_OK;
+}
+
+fk_status fk_profile_reset(fk_handle* h) {
+  if (!h) return FK_ERR_ARG;
+  fk_status st = prof_collect(h);
+  if (st != FK_OK) return st;
+  for (int k = 0; k < FK_KERNEL_KINDS; ++k) {
+    h->prof_ms[k] = 0;
+    h->prof_n[k] = 0;
+  }
+  return FK_OK;
+}
+
+int64_t fk_launch_count(const fk_handle* h) { return h ? h->launches : 0; }
+
+}  // extern "C"

@@ -1,0 +1,105 @@
+"""CPU-side checks of the C ABI: the library builds for sm_103a, loads, exports every
+symbol include/fk.h declares, and validates configurations on the host.  No kernel runs."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2605_09681_gb300 import build, _lib
+    build.build()
+    return _lib.load()
+
+
+def _declared():
+    text = open(os.path.join(ROOT, "include", "fk.h")).read()
+    return re.findall(r"FK_API\s+[\w\s\*]+?\b(fk_\w+)\s*\(", text)
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = _declared()
+    assert len(names) >= 20
+    raw = ctypes.CDLL(os.path.join(ROOT, "paper_2605_09681_gb300", "libfk.so"))
+    for n in names:
+        assert hasattr(raw, n), n
+    from paper_2605_09681_gb300 import _lib
+    assert sorted(names) == sorted(_lib.EXPORTS)
+
+
+def _cfg(**kw):
+    from paper_2605_09681_gb300._lib import FkConfig
+    hm = np.zeros(kw.get("n_layers", 1) * kw.get("n_heads", 4), dtype=np.uint8)
+    base = dict(n_layers=1, n_heads=4, head_dim=64, tokens_per_frame=60, frames_per_chunk=3,
+                n_sink_frames=1, window_frames=0, n_segments=6, keep_budget_permille=700,
+                select_scope=0, score_source=0, incremental=0, max_history_frames=8, device=0)
+    base.update(kw)
+    c = FkConfig(**base)
+    c.head_is_static = hm.ctypes.data_as(ctypes.POINTER(ctypes.c_uint8))
+    return c, hm
+
+
+def test_config_struct_layout():
+    from paper_2605_09681_gb300._lib import FkConfig
+    assert ctypes.sizeof(FkConfig) == 64
+    assert FkConfig.head_is_static.offset == 56
+
+
+@pytest.mark.parametrize("bad", [
+    dict(head_dim=96), dict(head_dim=0), dict(n_heads=0), dict(n_heads=129), dict(n_layers=0),
+    dict(n_layers=257), dict(tokens_per_frame=61), dict(n_segments=0), dict(frames_per_chunk=0),
+    dict(keep_budget_permille=1001), dict(keep_budget_permille=-1), dict(select_scope=2),
+    dict(score_source=5), dict(incremental=2), dict(window_frames=-1), dict(n_sink_frames=-1),
+    dict(window_frames=0, max_history_frames=0),
+])
+def test_validate_rejects_bad_configs(lib, bad):
+    c, _keep = _cfg(**bad)
+    assert lib.fk_validate_config(ctypes.byref(c)) == 1   # FK_ERR_CONFIG
+
+
+def test_validate_accepts_paper_configs(lib):
+    for kw in [dict(), dict(head_dim=128, n_heads=12, tokens_per_frame=1560),
+               dict(head_dim=128, n_heads=12, tokens_per_frame=8160, max_history_frames=10),
+               dict(window_frames=12, keep_budget_permille=600),
+               dict(n_segments=1, select_scope=1, keep_budget_permille=500, n_sink_frames=0),
+               dict(n_layers=30, n_heads=12, score_source=1, incremental=1, max_history_frames=21)]:
+        c, _keep = _cfg(**kw)
+        assert lib.fk_validate_config(ctypes.byref(c)) == 0, kw
+
+
+def test_null_config_and_status_strings(lib):
+    assert lib.fk_validate_config(None) == 2
+    for s in range(9):
+        assert lib.fk_status_str(s)
+    assert lib.fk_abi_version() == 1
+
+
+@pytest.mark.skipif(os.path.exists("/dev/nvidia0"), reason="checks the no-GPU error path")
+def test_create_without_gpu_fails_cleanly(lib):
+    c, _keep = _cfg()
+    h = ctypes.c_void_p()
+    st = lib.fk_create(ctypes.byref(c), ctypes.byref(h))
+    assert st == 7 and not h.value          # FK_ERR_CUDA, no handle
+
+
+def test_missing_library_fails_loudly(tmp_path):
+    from paper_2605_09681_gb300 import _lib
+    saved = _lib._lib
+    _lib._lib = None
+    try:
+        with pytest.raises(ImportError):
+            _lib.load(str(tmp_path / "libfk.so"))
+    finally:
+        _lib._lib = saved
+
+
+def test_null_handle_calls_are_rejected(lib):
+    assert lib.fk_compress(None, None) == 2
+    assert lib.fk_attend(None, 0, None, None, None) == 2
+    assert lib.fk_cache_bytes(None) == 0
+    lib.fk_destroy(None)

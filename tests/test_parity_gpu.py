@@ -1,0 +1,227 @@
+"""GPU parity of the CUDA path (through the C ABI) against the CPU oracle, on seeded inputs:
+kept sets and scores bit-exact, attention within max abs 2e-2 / mean abs 2e-3."""
+import numpy as np
+import pytest
+
+import oracle as O
+import workloads as W
+from fkharness import (ATOL_MAX, ATOL_MEAN, compare_layer, run_snapshot, sample_rows, snapshot,
+                       to_dev, to_f64)
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _library():
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    from paper_2605_09681_gb300 import build, load_library
+    build.build()
+    load_library()
+
+
+def _small(**kw):
+    base = dict(name="small", n_layers=1, n_heads=4, head_dim=64, tokens_per_frame=60,
+                frames_per_chunk=3, n_sink_frames=1, window_frames=0, n_segments=6,
+                keep_budget_permille=500, schedule="snapshot", n_history_frames=7,
+                static_heads=(0, 2), seed=11)
+    base.update(kw)
+    return W.Workload(**base)
+
+
+# ------------------------------------------------------------------ small cases, every row
+def test_tiny_pooled():
+    run_snapshot(W.TINY)
+
+
+def test_tiny_per_frame():
+    run_snapshot(W.TINY_PER_FRAME)
+
+
+@pytest.mark.parametrize("D", [64, 128])
+@pytest.mark.parametrize("budget", [0, 333, 500, 1000])
+def test_budgets_and_head_dims(D, budget):
+    run_snapshot(_small(head_dim=D, keep_budget_permille=budget, seed=D + budget))
+
+
+@pytest.mark.parametrize("S,nh", [(0, 1), (1, 1), (1, 2), (2, 5), (3, 3), (0, 0)])
+def test_degenerate_histories(S, nh):
+    # no history, sink-only history, a lone anchor, more sinks than history
+    run_snapshot(_small(n_sink_frames=S, n_history_frames=nh, seed=100 + 7 * S + nh),
+                 max_history_frames=max(1, nh))
+
+
+def test_ragged_tiles_d128():
+    # 200 tokens/frame: 600 queries (4 full q tiles + 88), segment 50, ragged key tiles
+    run_snapshot(_small(head_dim=128, tokens_per_frame=200, n_segments=4, n_history_frames=9,
+                        keep_budget_permille=750, seed=5))
+
+
+def test_single_segment_per_frame_per_frame_scope():
+    run_snapshot(_small(n_segments=1, keep_budget_permille=1000))
+
+
+def test_identical_adjacent_frames_tie_break():
+    # frames 1..4 identical: every score is exactly 1; ties keep the lower segment id
+    w = _small(n_history_frames=6, keep_budget_permille=500)
+    hk, hv, ck, cv, q = W.snapshot_inputs(w)
+    F = w.tokens_per_frame
+    for f in range(2, 5):
+        hk[f * F:(f + 1) * F] = hk[F:2 * F]
+    run_snapshot(w, inputs=(hk, hv, ck, cv, q))
+
+
+def test_host_pointers_match_device():
+    from paper_2605_09681_gb300 import ForcingKVCache
+    w = _small(head_dim=128, tokens_per_frame=120, n_history_frames=6)
+    hk, hv, ck, cv, q = W.snapshot_inputs(w)
+    hm = W.head_map(w)
+    outs = []
+    for host in (False, True):
+        with ForcingKVCache.from_workload(w, hm) as c:
+            conv = (lambda a: a) if host else to_dev
+            c.append_frames(0, conv(hk), conv(hv))
+            c.set_current(0, conv(ck), conv(cv))
+            c.compress()
+            if host:
+                qh = torch.from_numpy(q.view(np.int16)).view(torch.bfloat16).pin_memory()
+                oh = torch.empty_like(qh).pin_memory()
+                c.attend(0, qh, oh)
+                torch.cuda.synchronize()
+                outs.append(oh.float().numpy())
+            else:
+                outs.append(c.attend(0, to_dev(q)).float().cpu().numpy())
+    assert np.array_equal(outs[0], outs[1])
+
+
+# ------------------------------------------------------------------ streaming (window, incremental)
+def _stream(w, track_layers=(0,), compare_every=1, step_filter=None, layer_data=None):
+    """Drive a streaming workload through the library and the oracle; compare tracked layers."""
+    from paper_2605_09681_gb300 import ForcingKVCache
+    hm = W.head_map(w)
+    orc = O.ForcingKVOracle.from_workload(w, hm, track_layers=list(track_layers))
+    streams = {l: W.FrameStream(w, l) for l in orc.layers}
+    n_cmp = 0
+    with ForcingKVCache.from_workload(w, hm) as cache:
+        for c in range(w.n_chunks):
+            clean = {l: streams[l].frames(w.frames_per_chunk) for l in orc.layers}
+            for d in range(w.denoise_steps):
+                kv = {l: W.step_kv(w, l, c, d, *clean[l]) for l in orc.layers}
+                dev = {l: (to_dev(kv[l][0]), to_dev(kv[l][1])) for l in orc.layers}
+                for l in range(w.n_layers):
+                    src = l if l in dev else orc.layers[0]
+                    if d == 0:
+                        cache.append_chunk(l, *dev[src])
+                    else:
+                        cache.set_current(l, *dev[src])
+                for l in orc.layers:
+                    (orc.append_chunk if d == 0 else orc.set_current)(l, *kv[l])
+                if d == 0:
+                    cache.compress()
+                check = (c % compare_every == 0 or c == w.n_chunks - 1) and (
+                    step_filter is None or d in step_filter)
+                for l in orc.layers:
+                    q = W.queries(w, l, c, d)
+                    Od = cache.attend(l, to_dev(q))
+                    if check:
+                        torch.cuda.synchronize()
+                        rows = sample_rows(q.shape[0], 48, seed=c) if q.shape[0] > 1024 else None
+                        compare_layer(cache, orc, l, q, Od, rows=rows, label="%s c%d d%d" % (w.name, c, d))
+                        n_cmp += 1
+        assert cache.sync_status() == 0
+    return n_cmp
+
+
+def test_stream_window_small():
+    w = W.ROLLING.with_(name="rolling_small", head_dim=64, tokens_per_frame=48, n_heads=4,
+                        window_frames=5, n_chunks=12, scene_cut_every_chunks=4)
+    assert _stream(w) == 12
+
+
+def test_stream_incremental_matches_rescore():
+    from paper_2605_09681_gb300 import ForcingKVCache
+    w = W.ROLLING.with_(name="inc", head_dim=64, tokens_per_frame=60, n_heads=4, window_frames=6,
+                        n_chunks=6)
+    hm = W.head_map(w)
+    got = []
+    for inc in (True, False):
+        fs = W.FrameStream(w, 0)
+        with ForcingKVCache.from_workload(w, hm, incremental=inc) as cache:
+            res = []
+            for c in range(w.n_chunks):
+                k, v = fs.frames(3)
+                cache.append_chunk(0, to_dev(k), to_dev(v))
+                cache.compress()
+                res.append([(cache.kept(0, h), cache.scores(0, h)[1].tobytes()) for h in range(4)])
+            got.append(res)
+    assert got[0] == got[1]
+
+
+def test_stream_layer0_pooled_small():
+    w = W.P480_STACK.with_(name="stack_small", n_layers=3, n_heads=4, head_dim=64,
+                           tokens_per_frame=60, n_chunks=5, denoise_steps=2)
+    assert _stream(w, track_layers=(0, 1, 2)) == 5 * 2 * 3
+
+
+# ------------------------------------------------------------------ error paths (host-side)
+def test_state_errors():
+    from paper_2605_09681_gb300 import ForcingKVCache, FkError
+    w = _small(n_history_frames=3)
+    hk, hv, ck, cv, q = W.snapshot_inputs(w)
+    with ForcingKVCache.from_workload(w, W.head_map(w), max_history_frames=3) as c:
+        with pytest.raises(FkError) as e:
+            c.attend(0, to_dev(q))
+        assert e.value.name == "FK_ERR_STATE"          # no current chunk
+        c.append_frames(0, to_dev(hk), to_dev(hv))
+        c.set_current(0, to_dev(ck), to_dev(cv))
+        with pytest.raises(FkError) as e:
+            c.attend(0, to_dev(q))
+        assert e.value.name == "FK_ERR_STATE"          # appended, not compressed
+        c.compress()
+        c.attend(0, to_dev(q))
+        with pytest.raises(FkError) as e:
+            c.append_chunk(0, to_dev(ck), to_dev(cv))  # history would exceed 3 frames
+        assert e.value.name == "FK_ERR_FULL"
+        with pytest.raises(FkError) as e:
+            c.attend(7, to_dev(q))
+        assert e.value.name == "FK_ERR_ARG"
+        assert c.sync_status() == 0
+
+
+def test_range_precondition_reported():
+    from paper_2605_09681_gb300 import ForcingKVCache, STATUS_NAMES
+    w = _small(n_history_frames=4)
+    hk, hv, ck, cv, q = W.snapshot_inputs(w)
+    big = W.to_bf16_bits(np.full(hk.shape, 400.0))      # n_p = 64 * 400^2 > 2^23
+    with ForcingKVCache.from_workload(w, W.head_map(w)) as c:
+        c.append_frames(0, to_dev(big), to_dev(hv))
+        c.set_current(0, to_dev(ck), to_dev(cv))
+        c.compress()
+        assert STATUS_NAMES[c.sync_status()] == "FK_ERR_RANGE"
+        assert c.sync_status() == 0                     # the status word is cleared
+
+
+# ------------------------------------------------------------------ full-size workloads (sampled rows)
+def test_480p_layer():
+    w = W.P480_LAYER
+    st = run_snapshot(w, rows=sample_rows(w.n_queries, 96))
+    print("480p", st)
+
+
+def test_1080p_layer():
+    w = W.P1080_LAYER
+    st = run_snapshot(w, rows=sample_rows(w.n_queries, 64))
+    print("1080p", st)
+
+
+def test_rolling_full():
+    w = W.ROLLING
+    assert _stream(w, compare_every=10) >= 6
+
+
+def test_480p_stack_full():
+    # all 30 layers are appended and compressed; layers 0, 13, 29 carry their own seeded
+    # data and are attended and compared (the other layers replay layer 0's inputs)
+    w = W.P480_STACK
+    assert _stream(w, track_layers=(0, 13, 29), compare_every=3, step_filter=(0, 3)) > 0

@@ -20,6 +20,8 @@ Value model (per layer, per head, per token, per channel):
 from __future__ import annotations
 
 import math
+import os
+from concurrent.futures import ThreadPoolExecutor
 from dataclasses import dataclass, field, replace
 from typing import Iterator
 
@@ -32,6 +34,7 @@ __all__ = [
 ]
 
 _U64 = np.uint64
+_THREADS = max(1, min(16, os.cpu_count() or 1))
 
 
 def _splitmix64(x: np.ndarray) -> np.ndarray:
@@ -222,29 +225,40 @@ class FrameStream:
         self._xv = None
         self._scale = _head_scales(w, layer)[None, :, None]
 
-    def _step(self, x, rho, kind, f):
+    def _noise(self, kind, f):
         w = self.w
         e = normals(stream_key(w.seed, kind, self.layer, f),
                     w.tokens_per_frame * w.n_heads * w.head_dim)
-        e = e.reshape(w.tokens_per_frame, w.n_heads, w.head_dim)
-        if x is None or w.scene_cut(f):
+        return e.reshape(w.tokens_per_frame, w.n_heads, w.head_dim)
+
+    def _advance(self, x, rho, e, f):
+        if x is None or self.w.scene_cut(f):
             return e
         return rho * x + math.sqrt(max(0.0, 1.0 - rho * rho)) * e
 
     def next_frame(self) -> tuple[np.ndarray, np.ndarray]:
-        f = self.next
-        self._xk = self._step(self._xk, self.w.rho_k, _K, f)
-        self._xv = self._step(self._xv, self.w.rho_v, _V, f)
-        self.next += 1
-        return to_bf16_bits(self._scale * self._xk), to_bf16_bits(self._xv)
+        k, v = self.frames(1)
+        return k, v
 
     def frames(self, n: int) -> tuple[np.ndarray, np.ndarray]:
         """The next n frames, concatenated token-major: [n*F, H, D] each."""
-        ks, vs = zip(*(self.next_frame() for _ in range(n))) if n else ((), ())
         w = self.w
-        shape = (0, w.n_heads, w.head_dim)
-        return (np.concatenate(ks) if n else np.zeros(shape, np.uint16),
-                np.concatenate(vs) if n else np.zeros(shape, np.uint16))
+        F = w.tokens_per_frame
+        K = np.empty((n * F, w.n_heads, w.head_dim), np.uint16)
+        V = np.empty((n * F, w.n_heads, w.head_dim), np.uint16)
+        if n == 0:
+            return K, V
+        fs = list(range(self.next, self.next + n))
+        jobs = [(_K, f) for f in fs] + [(_V, f) for f in fs]
+        with ThreadPoolExecutor(max_workers=min(len(jobs), _THREADS)) as ex:
+            noise = dict(zip(jobs, ex.map(lambda kf: self._noise(*kf), jobs)))
+        for i, f in enumerate(fs):
+            self._xk = self._advance(self._xk, w.rho_k, noise[(_K, f)], f)
+            self._xv = self._advance(self._xv, w.rho_v, noise[(_V, f)], f)
+            K[i * F:(i + 1) * F] = to_bf16_bits(self._scale * self._xk)
+            V[i * F:(i + 1) * F] = to_bf16_bits(self._xv)
+        self.next += n
+        return K, V
 
     def chunks(self) -> Iterator[tuple[np.ndarray, np.ndarray]]:
         while True:
