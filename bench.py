@@ -1,0 +1,433 @@
+#!/usr/bin/env python
+"""Benchmark of the Forcing-KV hot path on GB300 (one JSON line on stdout).
+
+A step is one pass of the whole hot path over one chunk: the new chunk's K/V join the
+cache (append), the window is scored segment by segment, BottomK-selected and compacted
+(compress), and the chunk's queries attend over every head's key set (attend).  The
+default workload is the 480P single-layer case: 12 heads (6 static), head_dim 128, 1560
+tokens/frame, 3-frame chunks (4680 queries), 1 sink + 18 history frames, 70% dynamic
+budget.  Chunks stream through an 18-frame window so that every step sees exactly that
+cache; each step rescores the whole window.
+
+value   : compressed chunk-attention TFLOP/s over the whole step (algorithmic attention
+          FLOPs sum_h 4*Nq*Nk_h*D divided by the step time), inputs resident in HBM;
+e2e     : the same through the C ABI with pinned host buffers (Q, K, V in; O out) copied
+          inside every timed step;
+roofline: the attention kernel (tensor bound) against the measured bf16 peak, plus the
+          scoring and compaction kernels (HBM bound) against the measured copy bandwidth.
+
+--impl reference times the CPU oracle (the plain restatement of the paper) on the host
+cores for the same workload, metric and unit.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "compressed chunk-attention TFLOP/s + compaction GB/s (% roofline); attn frames/s"
+DIT_LAYERS, DENOISE_STEPS = 30, 4      # attention calls per generated chunk in the 30-block, 4-step DiT
+L2_FLUSH_BYTES = 512 << 20
+
+
+def _peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return {"hbm_gbs": d["hbm_gbs"], "bf16_tflops": d["bf16_tflops"],
+                "bf16_tflops_sustained": d.get("bf16_tflops_sustained"), "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+            "source": "fallback"}
+
+
+def _workload(name: str):
+    import workloads as W
+    w = W.WORKLOADS[name]
+    if w.schedule != "snapshot":
+        raise SystemExit("bench workloads are the single-layer cases: 480p_layer, 1080p_layer, tiny")
+    # stream chunks through a window holding exactly the snapshot's history
+    return w.with_(window_frames=max(1, w.n_history_frames - w.n_sink_frames), incremental=False)
+
+
+def _algorithmic(w, key_counts):
+    """Per-step algorithmic work: attention FLOPs and kernel bytes (the design doc lists the formulas)."""
+    import oracle as O
+    D, F, H = w.head_dim, w.tokens_per_frame, w.n_heads
+    nq = w.n_queries
+    flops = sum(4.0 * nq * nk * D for nk in key_counts)
+    roles = O.frame_roles(w.n_history_frames, w.n_sink_frames, w.window_frames)
+    n_dyn = sum(1 for nk, st in zip(key_counts, _workload_static(w)) if not st)
+    run_frames = len(roles.scoreable) + 1 if roles.scoreable else 0
+    score_bytes = n_dyn * run_frames * F * D * 2
+    n_keep = len(roles.scoreable) * O.keep_count(w.keep_budget_permille, w.n_segments)
+    units_tokens = len(roles.sink) * F + n_keep * (F // w.n_segments) + (F if roles.anchor is not None else 0)
+    compact_bytes = n_dyn * 2 * 2 * units_tokens * D * 2
+    append_bytes = 2 * 2 * nq * H * D * 2 + sum(
+        2 * 2 * w.frames_per_chunk * F * D * 2 if not st else 2 * 2 * F * D * 2
+        for st in _workload_static(w))
+    return dict(attn_flops=flops, score_bytes=score_bytes, compact_bytes=compact_bytes,
+                append_bytes=append_bytes)
+
+
+def _workload_static(w):
+    import workloads as W
+    return [bool(x) for x in W.head_map(w)[0]]
+
+
+class Clocks:
+    """nvidia-smi sampling during the timed region."""
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index, self.proc = index, None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.FIELDS,
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *exc):
+        self.out = ""
+        if self.proc:
+            time.sleep(0.2)
+            self.proc.terminate()
+            try:
+                self.out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in (self.out or "").splitlines():
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[4:8]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        loaded = [s for s in sm if s > 0.5 * max(sm)] or sm
+        return {"sm_mhz": statistics.median(loaded), "sm_max_mhz": max(mx),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def _dist():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    if ws > 1:
+        import torch.distributed as dist
+        if not dist.is_initialized():
+            dist.init_process_group("gloo")
+        return dist.get_rank(), ws, int(os.environ.get("LOCAL_RANK", "0"))
+    return 0, 1, 0
+
+
+def reduce_max(x: float, world: int) -> float:
+    """Maximum of a host float over all ranks (gloo, host side only)."""
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world: int) -> None:
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def run_fk(args, rank, world, local_rank):
+    import numpy as np
+    import torch
+
+    import workloads as W
+    from paper_2605_09681_gb300 import ForcingKVCache, build
+
+    build.build()
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    w = _workload(args.workload)
+    hm = W.head_map(w)
+    fs = W.FrameStream(w, 0)
+    hk, hv = fs.frames(w.n_history_frames)
+    n_pool = 4
+    chunks = [fs.frames(w.frames_per_chunk) for _ in range(n_pool)]
+    qs = [W.queries(w, 0, c, 0) for c in range(n_pool)]
+    to_t = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16)
+    dK = [to_t(k).to(dev) for k, _ in chunks]
+    dV = [to_t(v).to(dev) for _, v in chunks]
+    dQ = [to_t(q).to(dev) for q in qs]
+    dO = torch.empty_like(dQ[0])
+    hK = [to_t(k).pin_memory() for k, _ in chunks]
+    hV = [to_t(v).pin_memory() for _, v in chunks]
+    hQ = [to_t(q).pin_memory() for q in qs]
+    hO = torch.empty(dQ[0].shape, dtype=torch.bfloat16).pin_memory()
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    cache = ForcingKVCache.from_workload(w, hm, device=local_rank)
+    cache.append_frames(0, to_t(hk).to(dev), to_t(hv).to(dev))
+    cache.set_current(0, dK[0], dV[0])
+    cache.compress()
+
+    def step(i, host=False):
+        j = i % n_pool
+        if host:
+            cache.append_chunk(0, hK[j], hV[j])
+            cache.compress()
+            cache.attend(0, hQ[j], hO)
+        else:
+            cache.append_chunk(0, dK[j], dV[j])
+            cache.compress()
+            cache.attend(0, dQ[j], dO)
+
+    def timed(n, host):
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(n)]
+        barrier(world)
+        torch.cuda.synchronize()
+        for i in range(n):
+            flush.zero_()                        # L2 flushed between timed steps (outside events)
+            evs[i][0].record(stream)
+            step(i, host)
+            evs[i][1].record(stream)
+        torch.cuda.synchronize()
+        barrier(world)
+        return sum(a.elapsed_time(b) for a, b in evs)
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize()
+    st = cache.sync_status()
+    if st != 0:
+        raise SystemExit("device status %d during warm-up" % st)
+    keys = [cache.key_count(0, h) for h in range(w.n_heads)]
+    alg = _algorithmic(w, keys)
+
+    cache.profile_enable(True)
+    cache.profile_reset()
+    n0 = cache.launch_count()
+    with Clocks(local_rank) as clk:
+        total_ms = timed(args.steps, host=False)
+    launches = cache.launch_count() - n0
+    prof = {k: cache.profile_read(k) for k in ("append", "score", "select", "compact", "attend")}
+    cache.profile_enable(False)
+    st = cache.sync_status()
+    if st != 0:
+        raise SystemExit("device status %d during the timed region" % st)
+    total_ms = reduce_max(total_ms, world)
+
+    for i in range(min(args.warmup, 3)):
+        step(i, host=True)
+    torch.cuda.synchronize()
+    e2e_ms = reduce_max(timed(args.steps, host=True), world)
+    if cache.sync_status() != 0:
+        raise SystemExit("device status error during the end-to-end region")
+
+    peaks = _peaks()
+    ms_step = total_ms / args.steps
+    value = world * alg["attn_flops"] * args.steps / (total_ms * 1e-3) / 1e12
+    e2e_value = world * alg["attn_flops"] * args.steps / (e2e_ms * 1e-3) / 1e12
+
+    def per_launch(kind):
+        ms, n = prof[kind]
+        return ms / n if n else float("nan")
+
+    attn_ms = per_launch("attend")
+    attn_tflops = alg["attn_flops"] / (attn_ms * 1e-3) / 1e12
+    compact_ms, score_ms = per_launch("compact"), per_launch("score")
+    compact_gbs = alg["compact_bytes"] / (compact_ms * 1e-3) / 1e9
+    score_gbs = alg["score_bytes"] / (score_ms * 1e-3) / 1e9
+    append_ms = prof["append"][0] / max(1, prof["append"][1])
+    append_total = prof["append"][0] / args.steps
+    compress_ms = (prof["score"][0] + prof["select"][0] + prof["compact"][0]) / args.steps
+    attn_fps = w.frames_per_chunk / (DIT_LAYERS * (DENOISE_STEPS * attn_ms + append_total + compress_ms) * 1e-3)
+    traffic = _traffic(args.workload)
+    nbytes = dQ[0].numel() * 2
+    out = {
+        "metric": METRIC,
+        "value": round(value, 3),
+        "unit": "TFLOP/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(ms_step, 4),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic (seeded AR(1) bf16 K/V, iid Q; no model weights)",
+        "config": {
+            "workload": w.name + " streamed through an %d-frame window" % w.window_frames,
+            "heads": w.n_heads, "static_heads": int(sum(_workload_static(w))),
+            "head_dim": w.head_dim, "tokens_per_frame": w.tokens_per_frame,
+            "queries": w.n_queries, "sink_frames": w.n_sink_frames,
+            "history_frames": w.n_history_frames - w.n_sink_frames,
+            "segments": w.n_segments, "keep_budget": w.keep_budget_permille / 1000,
+            "keys_per_head": keys, "rescore": "whole window every step",
+            "l2": "flushed between timed steps (512 MiB write outside the step events)",
+            "parallelism": "replicas" if world > 1 else "single GPU",
+        },
+        "gpu_launches": int(launches),
+        "e2e": {"value": round(e2e_value, 3), "unit": "TFLOP/s", "ms_per_step": round(e2e_ms / args.steps, 4),
+                "h2d_bytes_per_step": 3 * nbytes, "d2h_bytes_per_step": nbytes},
+        "roofline": {
+            "bound": "tensor", "kernel": "attention (tcgen05)", "achieved": round(attn_tflops, 2),
+            "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
+            "frac": round(attn_tflops / peaks["bf16_tflops"], 4),
+            "peak_source": peaks["source"] + " bf16 dense burst (cuBLAS)",
+            "traffic": traffic.get("attend"),
+        },
+        "roofline_hbm": {
+            "compact": {"achieved": round(compact_gbs, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                        "frac": round(compact_gbs / peaks["hbm_gbs"], 4), "bytes": alg["compact_bytes"],
+                        "us": round(compact_ms * 1e3, 2), "traffic": traffic.get("compact")},
+            "score": {"achieved": round(score_gbs, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                      "frac": round(score_gbs / peaks["hbm_gbs"], 4), "bytes": alg["score_bytes"],
+                      "us": round(score_ms * 1e3, 2), "traffic": traffic.get("score")},
+            "peak_source": peaks["source"] + " HBM copy bandwidth",
+        },
+        "kernels_us_per_step": {k: round(prof[k][0] / args.steps * 1e3, 2) for k in prof},
+        "attn_fps_extrapolated": round(attn_fps, 2),
+        "attn_fps_note": "C frames / (30 layers x (4 attends + append + compress)) from one layer",
+        "attn_gflop_per_step": round(alg["attn_flops"] / 1e9, 2),
+        "clocks": clk.summary(),
+    }
+    if rank == 0 and not args.no_cpu_baseline:
+        out["cpu_baseline"] = cpu_baseline(w, budget_s=args.cpu_seconds)
+    cache.close()
+    return out
+
+
+def _traffic(workload):
+    """DRAM bytes per launch from the committed ncu summary of this workload, if present."""
+    p = os.path.join(ROOT, "profiles", "traffic_%s.json" % workload)
+    if os.path.exists(p):
+        try:
+            return json.load(open(p))
+        except ValueError:
+            return {}
+    return {}
+
+
+def cpu_baseline(w, budget_s=15.0, steps=1):
+    """The oracle, as it stands, on the host cores: one full compress (contract scores of
+    every dynamic head, selection) plus attention of a query-row sample; the full step is
+    extrapolated by scaling the attention time to all query rows."""
+    import numpy as np
+
+    import oracle as O
+    import workloads as W
+    hm = W.head_map(w)
+    fs = W.FrameStream(w, 0)
+    hk, hv = fs.frames(w.n_history_frames)
+    ck, cv = fs.frames(w.frames_per_chunk)
+    q = W.queries(w, 0, 0, 0)
+    orc = O.ForcingKVOracle.from_workload(w.with_(window_frames=0), hm)
+    orc.append_frames(0, hk, hv)
+    orc.set_current(0, ck, cv)
+    kept = {}
+    t0 = time.perf_counter()
+    for h in range(w.n_heads):
+        kept[h] = orc.kept(0, h)
+    t_compress = time.perf_counter() - t0
+    # calibrate the row sample to the time budget
+    rows = np.arange(0, w.n_queries, max(1, w.n_queries // 16))[:16]
+    t0 = time.perf_counter()
+    orc.attend(0, q, rows=rows, kept=kept)
+    t_small = time.perf_counter() - t0
+    per_row = t_small / len(rows)
+    n_rows = int(max(16, min(w.n_queries, (budget_s - t_compress) / max(per_row, 1e-9))))
+    rows = np.linspace(0, w.n_queries - 1, n_rows).astype(np.int64)
+    t0 = time.perf_counter()
+    orc.attend(0, q, rows=rows, kept=kept)
+    t_attn = time.perf_counter() - t0
+    step_s = t_compress + t_attn * w.n_queries / len(rows)
+    keys = [orc.view_length(0, h) for h in range(w.n_heads)]
+    flops = sum(4.0 * w.n_queries * nk * w.head_dim for nk in keys)
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    return {"value": round(flops / step_s / 1e12, 6), "unit": "TFLOP/s", "cores": cores,
+            "kind": "oracle",
+            "sample": "numpy fp64 oracle: contract scores + BottomK of all %d dynamic heads "
+                      "(%.2f s) and attention of %d of %d query rows of all heads (%.2f s), "
+                      "step time extrapolated to all rows = %.1f s; BLAS threads = host cores"
+                      % (sum(1 for x in hm[0] if not x), t_compress, len(rows), w.n_queries,
+                         t_attn, step_s),
+            "step_s": round(step_s, 3)}
+
+
+def run_reference(args, rank, world):
+    """The oracle arm: each step a bounded sample of the same workload on the host cores."""
+    w = _workload(args.workload)
+    budget = max(2.0, min(10.0, 150.0 / max(1, args.steps + args.warmup)))
+    for _ in range(args.warmup):
+        cpu_baseline(w, budget_s=budget)
+    vals, secs = [], 0.0
+    for _ in range(args.steps):
+        r = cpu_baseline(w, budget_s=budget)
+        vals.append(r["value"])
+        secs += r["step_s"]
+    value = statistics.mean(vals)
+    r["value"] = round(value, 6)
+    return {
+        "metric": METRIC, "value": round(value, 6), "unit": "TFLOP/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(secs / args.steps * 1e3, 1),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic (seeded AR(1) bf16 K/V, iid Q; no model weights)",
+        "config": {"workload": w.name + " streamed through an %d-frame window" % w.window_frames},
+        "impl": "reference", "cpu_baseline": r,
+        "e2e": {"value": round(value, 6), "unit": "TFLOP/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", choices=["fk", "reference"], default="fk")
+    ap.add_argument("--workload", default="480p_layer")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args(argv)
+    if args.warmup < 3:
+        ap.error("--warmup must be at least 3")
+    rank, world, local_rank = _dist()
+    if args.impl == "reference":
+        if rank == 0:
+            print(json.dumps(run_reference(args, rank, world)))
+        return 0
+    out = run_fk(args, rank, world, local_rank)
+    if rank == 0:
+        print(json.dumps(out))
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())
