@@ -1,16 +1,18 @@
 // Chunk attention over the per-head packed views (Sec. 4.2 Eq. 2, Sec. 4.3 Eq. 4):
 // O = softmax(Q K^T / sqrt(D)) V per head, with a different key count per head.
 //
-// One CTA computes 128 query rows of one head against all of the head's keys, in
-// tiles of 128 keys, on the 5th-generation tensor cores:
-//   warp 4 (one lane)  TMA: Q once (3D map over [Nq][H][D]), K and V tiles (2D maps over
-//                      the view arenas) into a two-stage ring, 128-byte swizzle;
-//   warp 5 (one lane)  tcgen05.mma: S = Q K^T into one of two TMEM buffers, then
-//                      O += P V into a TMEM accumulator; completion via tcgen05.commit;
-//   warps 0-3          softmax: thread r owns query row r = TMEM lane r; reads S with
-//                      tcgen05.ld, online softmax in the log2 domain with a lazily
-//                      rescaled running max, writes P (bf16) to shared memory for the
-//                      second MMA, and finally normalises O and stores it.
+// One CTA computes two 128-row query tiles of one head against all of the head's keys,
+// in tiles of 128 keys, on the 5th-generation tensor cores:
+//   warp 8 (one lane)  TMA: both Q tiles once (3D map over [Nq][H][D]), K and V tiles (2D
+//                      maps over the view arenas) into two-stage rings, 128-byte swizzle;
+//   warp 9 (one lane)  tcgen05.mma: S_t = Q_t K^T into TMEM (t = 0, 1), then
+//                      O_t += P_t V with P_t read from TMEM; completion via tcgen05.commit;
+//   warps 0-3 / 4-7    softmax of query tile 0 / 1 (ping-pong: one warpgroup's softmax
+//                      overlaps the other tile's MMAs): thread r owns row r = TMEM lane r,
+//                      reads S with tcgen05.ld, online softmax in the log2 domain with a
+//                      lazily rescaled running max, writes P as bf16 pairs over S's first
+//                      64 columns with tcgen05.st, and finally normalises O and stores it.
+// TMEM columns: S0 0-127, S1 128-255, O0 256.., O1 256+D.. (512 allocated).
 // Every mbarrier wait is bounded (%globaltimer); on expiry the CTA records
 // FK_ERR_TIMEOUT in the status word, drains its own TMA loads and MMAs and frees TMEM.
 #include "fk_internal.h"
@@ -21,26 +23,28 @@ namespace {
 constexpr uint64_t kWaitLimitNs = 2000000000ull;   // 2 s per wait
 constexpr float kRescaleThreshold = 8.0f;          // log2 units: rescale O when max grows > 2^8
 
+constexpr int kWarpTma = 8;                        // warps 0-3 / 4-7: softmax of query tile 0 / 1
+constexpr int kWarpMma = 9;
+constexpr int kAttnThreads = 320;
+
 struct AttnBarriers {
   uint64_t q_full;
   uint64_t k_full[2], k_empty[2];
   uint64_t v_full[2], v_empty[2];
-  uint64_t s_full[2], s_free[2];
-  uint64_t p_full, pv_done, fin;
+  uint64_t s_full[2], p_full[2];
+  uint64_t o_done, fin;
   uint32_t tmem_base;
   volatile int abort;
 };
 
 template <int D>
 struct Layout {
-  static constexpr int kQ = kAttnBM * D * 2;
-  static constexpr int kKV = kAttnBN * D * 2;
-  static constexpr int kP = kAttnBM * kAttnBN * 2;
-  static constexpr int kOffQ = 0;
-  static constexpr int kOffK = kOffQ + kQ;
-  static constexpr int kOffV = kOffK + 2 * kKV;
-  static constexpr int kOffP = kOffV + 2 * kKV;
-  static constexpr int kOffBar = kOffP + kP;
+  static constexpr int kQ = kAttnBM * D * 2;      // one 128-row query tile
+  static constexpr int kKV = kAttnBN * D * 2;     // one 128-key K or V tile
+  static constexpr int kOffQ = 0;                 // two query tiles
+  static constexpr int kOffK = kOffQ + 2 * kQ;    // two K stages
+  static constexpr int kOffV = kOffK + 2 * kKV;   // two V stages
+  static constexpr int kOffBar = kOffV + 2 * kKV;
   static constexpr int kUsed = kOffBar + 256;
   // at least ~116 KB so that one CTA occupies an SM (its 512 TMEM columns are then free)
   static constexpr int kSmem = (kUsed + 1024) > 118 * 1024 ? (kUsed + 1024) : 118 * 1024;
@@ -142,6 +146,14 @@ __device__ __forceinline__ void umma(uint32_t d_tmem, uint64_t a, uint64_t b, ui
       " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n"
       :: "r"(d_tmem), "l"(a), "l"(b), "r"(idesc), "r"(accumulate) : "memory");
 }
+// D[tmem] (+)= A[tmem] * B[smem]: A (M x 16, bf16 pairs packed along 8 columns) in tensor memory
+__device__ __forceinline__ void umma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b, uint32_t idesc,
+                                        uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}\n"
+      :: "r"(d_tmem), "r"(a_tmem), "l"(b), "r"(idesc), "r"(accumulate) : "memory");
+}
 __device__ __forceinline__ void umma_commit(uint64_t* b) {
   asm volatile(
       "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];"
@@ -158,6 +170,25 @@ __device__ __forceinline__ void umma_commit(uint64_t* b) {
         "=r"(v[19]), "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]), "=r"(v[24]),        \
         "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]),        \
         "=r"(v[31])                                                                         \
+      : "r"(taddr))
+
+#define FK_TMEM_LD64(taddr, v)                                                              \
+  asm volatile(                                                                             \
+      "tcgen05.ld.sync.aligned.32x32b.x64.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,"  \
+      "%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32,%33," \
+      "%34,%35,%36,%37,%38,%39,%40,%41,%42,%43,%44,%45,%46,%47,%48,%49,%50,%51,%52,%53,%54," \
+      "%55,%56,%57,%58,%59,%60,%61,%62,%63}, [%64];"                                        \
+      : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]),  \
+        "=r"(v[7]), "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]),           \
+        "=r"(v[13]), "=r"(v[14]), "=r"(v[15]), "=r"(v[16]), "=r"(v[17]), "=r"(v[18]),        \
+        "=r"(v[19]), "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]), "=r"(v[24]),        \
+        "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]),        \
+        "=r"(v[31]), "=r"(v[32]), "=r"(v[33]), "=r"(v[34]), "=r"(v[35]), "=r"(v[36]),        \
+        "=r"(v[37]), "=r"(v[38]), "=r"(v[39]), "=r"(v[40]), "=r"(v[41]), "=r"(v[42]),        \
+        "=r"(v[43]), "=r"(v[44]), "=r"(v[45]), "=r"(v[46]), "=r"(v[47]), "=r"(v[48]),        \
+        "=r"(v[49]), "=r"(v[50]), "=r"(v[51]), "=r"(v[52]), "=r"(v[53]), "=r"(v[54]),        \
+        "=r"(v[55]), "=r"(v[56]), "=r"(v[57]), "=r"(v[58]), "=r"(v[59]), "=r"(v[60]),        \
+        "=r"(v[61]), "=r"(v[62]), "=r"(v[63])                                               \
       : "r"(taddr))
 
 #define FK_TMEM_ST32(taddr, v)                                                              \
@@ -183,31 +214,70 @@ __device__ __forceinline__ float fast_exp2(float x) {
   return y;
 }
 
+// packed fp32 pair arithmetic (sm_100+): two lanes of work per instruction
+__device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) {
+  float2 d;
+  asm("{\n .reg .b64 ra, rb, rc, rd;\n mov.b64 ra, {%2, %3};\n mov.b64 rb, {%4, %5};\n"
+      " mov.b64 rc, {%6, %7};\n fma.rn.f32x2 rd, ra, rb, rc;\n mov.b64 {%0, %1}, rd;\n}"
+      : "=f"(d.x), "=f"(d.y) : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
+  return d;
+}
+__device__ __forceinline__ float2 fadd2(float2 a, float2 b) {
+  float2 d;
+  asm("{\n .reg .b64 ra, rb, rd;\n mov.b64 ra, {%2, %3};\n mov.b64 rb, {%4, %5};\n"
+      " add.rn.f32x2 rd, ra, rb;\n mov.b64 {%0, %1}, rd;\n}"
+      : "=f"(d.x), "=f"(d.y) : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+  return d;
+}
+
+// 2^x on the FMA pipe for a pair: range reduction x = n + f, n = round(x) (by adding and
+// subtracting 1.5 * 2^23), f in [-1/2, 1/2]; 2^f by a degree-3 polynomial fitted for
+// minimum relative error (7.5e-5; exp2_poly_fit.py); 2^n added to the exponent field.
+// x is clamped at -126 (results below 2^-126 are flushed to that magnitude; they are
+// far below the bf16 resolution of P relative to the row maximum 1).
+#ifndef FK_POLY_EVERY
+#define FK_POLY_EVERY 0
+#endif
+constexpr int kPolyEvery = FK_POLY_EVERY;          // one pair in kPolyEvery uses the polynomial
+__device__ __forceinline__ float2 exp2_poly2(float2 x) {
+  x.x = fmaxf(x.x, -126.0f);
+  x.y = fmaxf(x.y, -126.0f);
+  const float2 magic = make_float2(12582912.0f, 12582912.0f);
+  const float2 t = fadd2(x, magic);
+  const float2 n = fadd2(t, make_float2(-12582912.0f, -12582912.0f));
+  const float2 f = fadd2(x, make_float2(-n.x, -n.y));
+  float2 p = ffma2(make_float2(5.517166493e-02f, 5.517166493e-02f), f,
+                   make_float2(2.426111219e-01f, 2.426111219e-01f));
+  p = ffma2(p, f, make_float2(6.932609862e-01f, 6.932609862e-01f));
+  p = ffma2(p, f, make_float2(9.999280736e-01f, 9.999280736e-01f));
+  return make_float2(__int_as_float(__float_as_int(p.x) + (__float_as_int(t.x) << 23)),
+                     __int_as_float(__float_as_int(p.y) + (__float_as_int(t.y) << 23)));
+}
+
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   const __nv_bfloat162 p = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<const uint32_t*>(&p);
 }
 
 template <int D>
-__global__ void __launch_bounds__(192, 1)
+__global__ void __launch_bounds__(kAttnThreads, 1)
 attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
             const __grid_constant__ CUtensorMap tmV, const AttnArgs a) {
   using Lay = Layout<D>;
   constexpr int kHalves = D / 64;                 // 64-column (128-byte) swizzle atoms
   constexpr uint32_t kTmemCols = 512;
-  constexpr uint32_t kColO = 2 * kAttnBN;         // S0 = cols 0..127, S1 = 128..255, O = 256..
+  constexpr uint32_t kColO = 2 * kAttnBN;         // S0 = cols 0..127, S1 = 128..255, O0, O1 after
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
   uint8_t* sQ = smem + Lay::kOffQ;
   uint8_t* sK = smem + Lay::kOffK;
   uint8_t* sV = smem + Lay::kOffV;
-  uint8_t* sP = smem + Lay::kOffP;
   AttnBarriers* bar = reinterpret_cast<AttnBarriers*>(smem + Lay::kOffBar);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int hi = blockIdx.x / a.n_qtiles;
-  const int q0 = (blockIdx.x - hi * a.n_qtiles) * kAttnBM;
+  const int q0 = (blockIdx.x - hi * a.n_qtiles) * (2 * kAttnBM);
   const int head = a.head_of[hi];
   const int nk = a.n_keys[head];
   const int row0 = a.row_base[head];
@@ -221,15 +291,14 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
       mbar_init(&bar->v_full[i], 1);
       mbar_init(&bar->v_empty[i], 1);
       mbar_init(&bar->s_full[i], 1);
-      mbar_init(&bar->s_free[i], 4);
+      mbar_init(&bar->p_full[i], 4);
     }
-    mbar_init(&bar->p_full, 4);
-    mbar_init(&bar->pv_done, 1);
+    mbar_init(&bar->o_done, 1);
     mbar_init(&bar->fin, 1);
     bar->abort = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
-  if (warp == 5) {
+  if (warp == kWarpMma) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;"
                  :: "r"(su32(&bar->tmem_base)), "r"(kTmemCols) : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
@@ -239,14 +308,16 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
   tc_fence_after();
   const uint32_t tmem = bar->tmem_base;
 
-  if (warp == 4) {
+  if (warp == kWarpTma) {
     // ------------------------------------------------------------------ TMA producer
     if (lane == 0) {
       int lastK[2] = {-1, -1}, lastV[2] = {-1, -1};
       bool ok = true;
-      mbar_expect_tx(&bar->q_full, Lay::kQ);
-      for (int h = 0; h < kHalves; ++h)
-        tma_load_3d(sQ + h * 16384, &tmQ, &bar->q_full, h * 64, head, q0);
+      mbar_expect_tx(&bar->q_full, 2 * Lay::kQ);
+      for (int t = 0; t < 2; ++t)
+        for (int h = 0; h < kHalves; ++h)
+          tma_load_3d(sQ + t * Lay::kQ + h * 16384, &tmQ, &bar->q_full, h * 64, head,
+                      q0 + t * kAttnBM);
       for (int j = 0; j < nt && ok; ++j) {
         const int st = j & 1, u = j >> 1;
         if (j >= 2 && !wait_phase(&bar->k_empty[st], (u - 1) & 1, bar, a.status)) { ok = false; break; }
@@ -271,142 +342,186 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
       }
     }
     __syncwarp();
-  } else if (warp == 5) {
+  } else if (warp == kWarpMma) {
     // ------------------------------------------------------------------ MMA issuer
+    // Order per key tile j:  PV0(j), S0(j+1), PV1(j), S1(j+1).  Tensor-core operations of
+    // one thread complete in issue order, so when S_t(j+1) is reported complete, PV_t(j)
+    // is complete too: the softmax of tile j+1 may rescale O_t without a further wait, and
+    // S_t(j+1) overwriting P_t(j) (same columns) happens after PV_t(j) has read it.
     if (lane == 0) {
       constexpr uint32_t kIdQK = idesc_bf16(kAttnBM, kAttnBN, 0);
       constexpr uint32_t kIdPV = idesc_bf16(kAttnBM, D, 1);
-      const uint32_t aQ = su32(sQ), aK = su32(sK), aV = su32(sV), aP = su32(sP);
-      auto pv = [&](int i) -> bool {
-        const int st = i & 1;
-        if (!wait_phase(&bar->p_full, i & 1, bar, a.status)) return false;
-        if (!wait_phase(&bar->v_full[st], (i >> 1) & 1, bar, a.status)) return false;
-        tc_fence_after();
-#pragma unroll
-        for (int kk = 0; kk < kAttnBN / 16; ++kk) {
-          const uint64_t da = sdesc(aP + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024);
-          const uint64_t db = sdesc(aV + st * Lay::kKV + kk * 2048, 16384, 1024);
-          umma(tmem + kColO, da, db, kIdPV, (i > 0 || kk > 0) ? 1u : 0u);
-        }
-        umma_commit(&bar->v_empty[st]);
-        umma_commit(&bar->pv_done);
-        return true;
-      };
-      bool ok = wait_phase(&bar->q_full, 0, bar, a.status);
-      for (int j = 0; j < nt && ok; ++j) {
-        const int st = j & 1, u = j >> 1;
-        if (!wait_phase(&bar->k_full[st], u & 1, bar, a.status)) { ok = false; break; }
-        if (j >= 2 && !wait_phase(&bar->s_free[j & 1], (u - 1) & 1, bar, a.status)) { ok = false; break; }
-        tc_fence_after();
-        const uint32_t tS = tmem + (uint32_t)((j & 1) * kAttnBN);
+      const uint32_t aQ = su32(sQ), aK = su32(sK), aV = su32(sV);
+      auto qk = [&](int j, int t) {
+        const int st = j & 1;
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
-          const uint64_t da = sdesc(aQ + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024);
+          const uint64_t da = sdesc(aQ + t * Lay::kQ + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024);
           const uint64_t db = sdesc(aK + st * Lay::kKV + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024);
-          umma(tS, da, db, kIdQK, kk > 0 ? 1u : 0u);
+          umma(tmem + (uint32_t)(t * kAttnBN), da, db, kIdQK, kk > 0 ? 1u : 0u);
         }
-        umma_commit(&bar->s_full[j & 1]);
-        umma_commit(&bar->k_empty[st]);
-        if (j >= 1 && !pv(j - 1)) { ok = false; break; }
+        umma_commit(&bar->s_full[t]);
+      };
+      auto pv = [&](int j, int t) {
+        const int st = j & 1;
+#pragma unroll
+        for (int kk = 0; kk < kAttnBN / 16; ++kk) {
+          const uint64_t db = sdesc(aV + st * Lay::kKV + kk * 2048, 16384, 1024);
+          umma_ts(tmem + kColO + (uint32_t)(t * D), tmem + (uint32_t)(t * kAttnBN + kk * 8), db,
+                  kIdPV, (j > 0 || kk > 0) ? 1u : 0u);
+        }
+      };
+      bool ok = wait_phase(&bar->q_full, 0, bar, a.status) &&
+                wait_phase(&bar->k_full[0], 0, bar, a.status);
+      if (ok) {
+        tc_fence_after();
+        qk(0, 0);
+        qk(0, 1);
+        umma_commit(&bar->k_empty[0]);
       }
-      if (ok) pv(nt - 1);
+      for (int j = 0; j < nt && ok; ++j) {
+        const int st = j & 1;
+        const bool more = j + 1 < nt;
+        if (!wait_phase(&bar->p_full[0], j & 1, bar, a.status) ||
+            !wait_phase(&bar->v_full[st], (j >> 1) & 1, bar, a.status)) { ok = false; break; }
+        tc_fence_after();
+        pv(j, 0);
+        if (more) {
+          if (!wait_phase(&bar->k_full[(j + 1) & 1], ((j + 1) >> 1) & 1, bar, a.status)) { ok = false; break; }
+          tc_fence_after();
+          qk(j + 1, 0);
+        }
+        if (!wait_phase(&bar->p_full[1], j & 1, bar, a.status)) { ok = false; break; }
+        tc_fence_after();
+        pv(j, 1);
+        umma_commit(&bar->v_empty[st]);
+        if (more) {
+          qk(j + 1, 1);
+          umma_commit(&bar->k_empty[(j + 1) & 1]);
+        }
+      }
+      if (ok) umma_commit(&bar->o_done);
       umma_commit(&bar->fin);                       // completes once every MMA above is done
       wait_phase(&bar->fin, 0, bar, a.status, false);
     }
     __syncwarp();
   } else {
-    // ------------------------------------------------------------------ softmax warps 0-3
-    const int row = warp * 32 + lane;
-    const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+    // ------------------------------------------------------------------ softmax warpgroups
+    const int t = warp >> 2;                        // query tile of this warpgroup
+    const int wq = warp & 3;
+    const int row = wq * 32 + lane;
+    const uint32_t lane_base = (uint32_t)(wq * 32) << 16;
+    const uint32_t tS = tmem + lane_base + (uint32_t)(t * kAttnBN);
+    const uint32_t tO = tmem + lane_base + kColO + (uint32_t)(t * D);
     float m = -INFINITY, l = 0.0f;
     bool ok = true;
     for (int j = 0; j < nt; ++j) {
-      if (!warp_wait(&bar->s_full[j & 1], (j >> 1) & 1, bar, a.status)) { ok = false; break; }
+      if (!warp_wait(&bar->s_full[t], j & 1, bar, a.status)) { ok = false; break; }
       tc_fence_after();
-      float s[kAttnBN];
-      {
-        uint32_t* sv = reinterpret_cast<uint32_t*>(s);
-        const uint32_t tS = tmem + lane_base + (uint32_t)((j & 1) * kAttnBN);
-        FK_TMEM_LD32(tS + 0, (sv + 0));
-        FK_TMEM_LD32(tS + 32, (sv + 32));
-        FK_TMEM_LD32(tS + 64, (sv + 64));
-        FK_TMEM_LD32(tS + 96, (sv + 96));
+      const int valid = nk - j * kAttnBN;           // keys of this tile (< 128 only in the last)
+      const bool full = valid >= kAttnBN;           // uniform over the CTA
+      // pass 1: row maximum, 64 columns at a time, eight independent chains
+      float mxa[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) mxa[i] = -INFINITY;
+#pragma unroll
+      for (int half = 0; half < 2; ++half) {
+        uint32_t sv[64];
+        FK_TMEM_LD64(tS + half * 64, sv);
         tmem_wait_ld();
-      }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&bar->s_free[j & 1]);
-
-      const int valid = nk - j * kAttnBN;
-      if (valid < kAttnBN) {
+        if (full) {
 #pragma unroll
-        for (int c = 0; c < kAttnBN; ++c)
-          if (c >= valid) s[c] = -INFINITY;
-      }
-      float mx = s[0];
+          for (int c = 0; c < 64; ++c) mxa[c & 7] = fmaxf(mxa[c & 7], __uint_as_float(sv[c]));
+        } else {
 #pragma unroll
-      for (int c = 1; c < kAttnBN; ++c) mx = fmaxf(mx, s[c]);
-      const float m_new = fmaxf(m, mx * a.scale_log2);
-      bool pv_waited = false;
-      const bool need = m_new > m + kRescaleThreshold;
-      if (__any_sync(0xffffffffu, need)) {
-        const float alpha = fast_exp2(m - m_new);    // 0 when m = -inf
-        if (j > 0) {
-          if (!warp_wait(&bar->pv_done, (j - 1) & 1, bar, a.status)) { ok = false; break; }
-          pv_waited = true;
-          tc_fence_after();
-#pragma unroll
-          for (int c = 0; c < D / 32; ++c) {
-            uint32_t o[32];
-            const uint32_t tO = tmem + lane_base + kColO + c * 32;
-            FK_TMEM_LD32(tO, o);
-            tmem_wait_ld();
-#pragma unroll
-            for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
-            FK_TMEM_ST32(tO, o);
-          }
-          tmem_wait_st();
+          for (int c = 0; c < 64; ++c)
+            if (half * 64 + c < valid) mxa[c & 7] = fmaxf(mxa[c & 7], __uint_as_float(sv[c]));
         }
+      }
+      const float mx = fmaxf(fmaxf(fmaxf(mxa[0], mxa[1]), fmaxf(mxa[2], mxa[3])),
+                             fmaxf(fmaxf(mxa[4], mxa[5]), fmaxf(mxa[6], mxa[7])));
+      const float m_new = fmaxf(m, mx * a.scale_log2);
+      const bool need = m_new > m + kRescaleThreshold;
+      float alpha = 1.0f;
+      const bool rescale = __any_sync(0xffffffffu, need);   // warp-uniform
+      if (rescale) {
+        alpha = fast_exp2(m - m_new);                // 0 when m = -inf
         l *= alpha;
         m = m_new;
       }
-      float rs = 0.0f;
+      // pass 2: P = exp2(S*c - m) as bf16 pairs, written over the S columns already read
+      // (P columns 32h..32h+31 come from S columns 64h..64h+63): the A operand of PV
+      const float2 sc2 = make_float2(a.scale_log2, a.scale_log2);
+      const float2 nm2 = make_float2(-m, -m);
+      float2 acc[4];
 #pragma unroll
-      for (int c = 0; c < kAttnBN; ++c) {
-        s[c] = fast_exp2(fmaf(s[c], a.scale_log2, -m));
-        rs += s[c];
+      for (int i = 0; i < 4; ++i) acc[i] = make_float2(0.0f, 0.0f);
+#pragma unroll
+      for (int half = 0; half < 2; ++half) {
+        uint32_t sv[64];
+        FK_TMEM_LD64(tS + half * 64, sv);
+        tmem_wait_ld();
+        uint32_t pk[32];
+        if (full) {
+#pragma unroll
+          for (int q = 0; q < 32; ++q) {
+            const float2 x = ffma2(make_float2(__uint_as_float(sv[2 * q]), __uint_as_float(sv[2 * q + 1])),
+                                   sc2, nm2);
+            float2 e;
+            if (kPolyEvery > 0 && q % (kPolyEvery > 0 ? kPolyEvery : 1) == kPolyEvery - 1) {
+              e = exp2_poly2(x);                     // FMA pipe
+            } else {
+              e.x = fast_exp2(x.x);                  // MUFU
+              e.y = fast_exp2(x.y);
+            }
+            acc[q & 3] = fadd2(acc[q & 3], e);
+            pk[q] = pack_bf16(e.x, e.y);
+          }
+        } else {
+#pragma unroll
+          for (int q = 0; q < 32; ++q) {
+            const int c = half * 64 + 2 * q;
+            const float x0 = c < valid ? __uint_as_float(sv[2 * q]) : -INFINITY;
+            const float x1 = c + 1 < valid ? __uint_as_float(sv[2 * q + 1]) : -INFINITY;
+            float2 e;
+            e.x = fast_exp2(fmaf(x0, a.scale_log2, -m));
+            e.y = fast_exp2(fmaf(x1, a.scale_log2, -m));
+            acc[q & 3] = fadd2(acc[q & 3], e);
+            pk[q] = pack_bf16(e.x, e.y);
+          }
+        }
+        FK_TMEM_ST32(tS + half * 32, pk);
       }
+      const float2 acc01 = fadd2(acc[0], acc[1]), acc23 = fadd2(acc[2], acc[3]);
+      const float2 acc4 = fadd2(acc01, acc23);
+      const float rs = acc4.x + acc4.y;
       l += rs;
-      if (j > 0 && !pv_waited) {
-        if (!warp_wait(&bar->pv_done, (j - 1) & 1, bar, a.status)) { ok = false; break; }
-      }
-      // P row -> shared memory, K-major with the 128-byte swizzle (chunk ^= row % 8)
-      uint8_t* prow = sP + row * 128;
+      if (rescale && j > 0) {                        // PV_t(j-1) is complete (see MMA order)
 #pragma unroll
-      for (int cc = 0; cc < kAttnBN / 8; ++cc) {
-        uint4 v;
-        v.x = pack_bf16(s[cc * 8 + 0], s[cc * 8 + 1]);
-        v.y = pack_bf16(s[cc * 8 + 2], s[cc * 8 + 3]);
-        v.z = pack_bf16(s[cc * 8 + 4], s[cc * 8 + 5]);
-        v.w = pack_bf16(s[cc * 8 + 6], s[cc * 8 + 7]);
-        const int atom = cc >> 3, ch = (cc & 7) ^ (row & 7);
-        *reinterpret_cast<uint4*>(prow + atom * 16384 + ch * 16) = v;
+        for (int c = 0; c < D / 32; ++c) {
+          uint32_t o[32];
+          FK_TMEM_LD32(tO + c * 32, o);
+          tmem_wait_ld();
+#pragma unroll
+          for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
+          FK_TMEM_ST32(tO + c * 32, o);
+        }
       }
-      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      tmem_wait_st();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&bar->p_full);
+      if (lane == 0) mbar_arrive(&bar->p_full[t]);
     }
     // ---------------------------------------------------------------- epilogue
-    if (ok && warp_wait(&bar->pv_done, (nt - 1) & 1, bar, a.status)) {
+    if (ok && warp_wait(&bar->o_done, 0, bar, a.status)) {
       tc_fence_after();
       const float inv = 1.0f / l;
-      const int q = q0 + row;
+      const int q = q0 + t * kAttnBM + row;
       bf16* orow = a.O + ((int64_t)q * a.H + head) * D;
 #pragma unroll
       for (int c = 0; c < D / 32; ++c) {
         uint32_t o[32];
-        FK_TMEM_LD32(tmem + lane_base + kColO + c * 32, o);
+        FK_TMEM_LD32(tO + c * 32, o);
         tmem_wait_ld();
         if (q < a.Nq) {
 #pragma unroll
@@ -425,7 +540,7 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
 
   tc_fence_before();
   __syncthreads();
-  if (warp == 5) {
+  if (warp == kWarpMma) {
     tc_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" :: "r"(tmem),
                  "r"(kTmemCols) : "memory");
@@ -446,9 +561,9 @@ void launch_attention(int head_dim, const CUtensorMap& tmQ, const CUtensorMap& t
                       const CUtensorMap& tmV, const AttnArgs& a, cudaStream_t s) {
   const unsigned grid = (unsigned)(a.n_qtiles * a.H);
   if (head_dim == 128)
-    attn_kernel<128><<<grid, 192, Layout<128>::kSmem, s>>>(tmQ, tmK, tmV, a);
+    attn_kernel<128><<<grid, kAttnThreads, Layout<128>::kSmem, s>>>(tmQ, tmK, tmV, a);
   else
-    attn_kernel<64><<<grid, 192, Layout<64>::kSmem, s>>>(tmQ, tmK, tmV, a);
+    attn_kernel<64><<<grid, kAttnThreads, Layout<64>::kSmem, s>>>(tmQ, tmK, tmV, a);
 }
 
 }  // namespace fk

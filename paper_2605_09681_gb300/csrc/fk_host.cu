@@ -806,7 +806,7 @@ fk_status fk_attend(fk_handle* h, int layer, const void* Q, void* O, void* strea
   a.O = o;
   a.Nq = h->CF;
   a.H = h->H;
-  a.n_qtiles = (h->CF + kAttnBM - 1) / kAttnBM;
+  a.n_qtiles = (h->CF + 2 * kAttnBM - 1) / (2 * kAttnBM);   // CTA = two 128-row query tiles
   a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)h->D));
   a.status = h->status;
   std::vector<int> order(h->H);
