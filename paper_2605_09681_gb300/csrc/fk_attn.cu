@@ -420,15 +420,25 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
       tc_fence_after();
       const int valid = nk - j * kAttnBN;           // keys of this tile (< 128 only in the last)
       const bool full = valid >= kAttnBN;           // uniform over the CTA
-      // pass 1: row maximum, 64 columns at a time, eight independent chains
-      float mxa[8];
+      const float2 sc2 = make_float2(a.scale_log2, a.scale_log2);
+      float2 acc[4];
 #pragma unroll
-      for (int i = 0; i < 8; ++i) mxa[i] = -INFINITY;
+      for (int i = 0; i < 4; ++i) acc[i] = make_float2(0.0f, 0.0f);
+      float alpha_tile = 1.0f;
+      bool rescaled = false;
+      // One pass per 64-column half: the half's maximum (eight independent chains), a lazy
+      // update of the running max m (only when it grows by more than 2^8), then
+      // P = exp2(S*c - m) as bf16 pairs written over the S columns already read (P columns
+      // 32h..32h+31 come from S columns 64h..64h+63): the A operand of PV.  If the second
+      // half raises m, the first half's stored P is rescaled in place.
 #pragma unroll
       for (int half = 0; half < 2; ++half) {
         uint32_t sv[64];
         FK_TMEM_LD64(tS + half * 64, sv);
         tmem_wait_ld();
+        float mxa[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) mxa[i] = -INFINITY;
         if (full) {
 #pragma unroll
           for (int c = 0; c < 64; ++c) mxa[c & 7] = fmaxf(mxa[c & 7], __uint_as_float(sv[c]));
@@ -437,30 +447,31 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
           for (int c = 0; c < 64; ++c)
             if (half * 64 + c < valid) mxa[c & 7] = fmaxf(mxa[c & 7], __uint_as_float(sv[c]));
         }
-      }
-      const float mx = fmaxf(fmaxf(fmaxf(mxa[0], mxa[1]), fmaxf(mxa[2], mxa[3])),
-                             fmaxf(fmaxf(mxa[4], mxa[5]), fmaxf(mxa[6], mxa[7])));
-      const float m_new = fmaxf(m, mx * a.scale_log2);
-      const bool need = m_new > m + kRescaleThreshold;
-      float alpha = 1.0f;
-      const bool rescale = __any_sync(0xffffffffu, need);   // warp-uniform
-      if (rescale) {
-        alpha = fast_exp2(m - m_new);                // 0 when m = -inf
-        l *= alpha;
-        m = m_new;
-      }
-      // pass 2: P = exp2(S*c - m) as bf16 pairs, written over the S columns already read
-      // (P columns 32h..32h+31 come from S columns 64h..64h+63): the A operand of PV
-      const float2 sc2 = make_float2(a.scale_log2, a.scale_log2);
-      const float2 nm2 = make_float2(-m, -m);
-      float2 acc[4];
+        const float mx = fmaxf(fmaxf(fmaxf(mxa[0], mxa[1]), fmaxf(mxa[2], mxa[3])),
+                               fmaxf(fmaxf(mxa[4], mxa[5]), fmaxf(mxa[6], mxa[7])));
+        const float m_new = fmaxf(m, mx * a.scale_log2);
+        if (__any_sync(0xffffffffu, m_new > m + kRescaleThreshold)) {   // warp-uniform
+          const float alpha = fast_exp2(m - m_new);  // 0 when m = -inf
+          l *= alpha;
 #pragma unroll
-      for (int i = 0; i < 4; ++i) acc[i] = make_float2(0.0f, 0.0f);
+          for (int i = 0; i < 4; ++i) acc[i] = make_float2(acc[i].x * alpha, acc[i].y * alpha);
+          if (half == 1) {                           // rare: first half of P was stored with the old m
+            uint32_t p0[32];
+            tmem_wait_st();
+            FK_TMEM_LD32(tS, p0);
+            tmem_wait_ld();
 #pragma unroll
-      for (int half = 0; half < 2; ++half) {
-        uint32_t sv[64];
-        FK_TMEM_LD64(tS + half * 64, sv);
-        tmem_wait_ld();
+            for (int e = 0; e < 32; ++e) {
+              const __nv_bfloat162 b = *reinterpret_cast<const __nv_bfloat162*>(&p0[e]);
+              p0[e] = pack_bf16(__low2float(b) * alpha, __high2float(b) * alpha);
+            }
+            FK_TMEM_ST32(tS, p0);
+          }
+          alpha_tile *= alpha;
+          rescaled = true;
+          m = m_new;
+        }
+        const float2 nm2 = make_float2(-m, -m);
         uint32_t pk[32];
         if (full) {
 #pragma unroll
@@ -494,16 +505,15 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
       }
       const float2 acc01 = fadd2(acc[0], acc[1]), acc23 = fadd2(acc[2], acc[3]);
       const float2 acc4 = fadd2(acc01, acc23);
-      const float rs = acc4.x + acc4.y;
-      l += rs;
-      if (rescale && j > 0) {                        // PV_t(j-1) is complete (see MMA order)
+      l += acc4.x + acc4.y;
+      if (rescaled && j > 0) {                       // PV_t(j-1) is complete (see MMA order)
 #pragma unroll
         for (int c = 0; c < D / 32; ++c) {
           uint32_t o[32];
           FK_TMEM_LD32(tO + c * 32, o);
           tmem_wait_ld();
 #pragma unroll
-          for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
+          for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha_tile);
           FK_TMEM_ST32(tO + c * 32, o);
         }
       }

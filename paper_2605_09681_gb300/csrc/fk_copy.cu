@@ -1,8 +1,9 @@
-// Data-movement kernels of the Forcing-KV cache: the current chunk's scatter from the
-// caller's token-major [tokens][H][D] layout into per-head views, frame copies into the
-// history pages (append), and the select-and-compact gather of kept segments into the
+// Data-movement kernels of the Forcing-KV cache: the current-chunk update (the previous
+// current chunk joins the history pages and the new chunk is scattered from the caller's
+// token-major [tokens][H][D] layout into the per-head views, in one pass), the prefill
+// scatter of history frames, and the select-and-compact gather of kept segments into the
 // packed per-head views of dynamic heads (Sec. 4.3, Eq. 4: [sink, kept segments, anchor]).
-// All three are HBM-bound: every byte is read once and written once with 16-byte accesses.
+// All of them are HBM-bound: every byte is read once and written once in 16-byte accesses.
 #include "fk_internal.h"
 
 namespace fk {
@@ -15,58 +16,97 @@ __device__ __forceinline__ uint4 ld_stream(const void* p) {
   return v;
 }
 
+// plain (coherent) load: the current kernel reads view rows it may itself have written
+// in an earlier launch, never in the same launch
+__device__ __forceinline__ uint4 ld_plain(const void* p) {
+  return *reinterpret_cast<const uint4*>(p);
+}
+
 __device__ __forceinline__ void st_v4(void* p, uint4 v) {
   asm volatile("st.global.v4.u32 [%0], {%1,%2,%3,%4};" :: "l"(p), "r"(v.x), "r"(v.y), "r"(v.z),
                "r"(v.w) : "memory");
-}
-
-// token-major [rows][H][D] -> dst[h] + row*D.  Consecutive threads read consecutive
-// 16-byte granules of the source; each head's destination rows are contiguous.
-__global__ void __launch_bounds__(256) scatter_kernel(const ScatterArgs a) {
-  const int gpr = a.head_dim / 8;                       // granules per head row
-  const int64_t per_row = (int64_t)a.heads * gpr;
-  const int64_t total = (int64_t)a.rows * per_row;
-  for (int64_t g = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; g < total;
-       g += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t row = g / per_row;
-    const int rem = (int)(g - row * per_row);
-    const int h = rem / gpr;
-    const int c = rem - h * gpr;
-    const int64_t dst_off = row * a.head_dim + c * 8;
-    if (a.dstK[h]) st_v4(a.dstK[h] + dst_off, ld_stream(a.srcK + g * 8));
-    if (a.dstV[h]) st_v4(a.dstV[h] + dst_off, ld_stream(a.srcV + g * 8));
-  }
-}
-
-// a list of contiguous copies; blockIdx.y selects the job
-__global__ void __launch_bounds__(256) copy_jobs_kernel(const CopyJobs j) {
-  const CopyJob& job = j.job[blockIdx.y];
-  const int64_t n = job.bytes / 16;
-  const uint4* src = static_cast<const uint4*>(job.src);
-  uint4* dst = static_cast<uint4*>(job.dst);
-  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-  int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-  for (; i + 3 * stride < n; i += 4 * stride) {
-    uint4 v0 = ld_stream(src + i), v1 = ld_stream(src + i + stride);
-    uint4 v2 = ld_stream(src + i + 2 * stride), v3 = ld_stream(src + i + 3 * stride);
-    st_v4(dst + i, v0); st_v4(dst + i + stride, v1);
-    st_v4(dst + i + 2 * stride, v2); st_v4(dst + i + 3 * stride, v3);
-  }
-  for (; i < n; i += stride) st_v4(dst + i, ld_stream(src + i));
 }
 
 __device__ __forceinline__ int ring_slot(int f, int S, int cap) {
   return f < S ? f : S + (f - S) % cap;
 }
 
-// One CTA copies one unit (F/n tokens of keys and values) of one dynamic head's view.
-// Units in view order: sink frames (n units each), kept segments (ascending t*n+j),
-// anchor frame (n units).  Unit u lands at view row CF + u*seg_len.
+// One thread per 16-byte granule of the current chunk, indexed in the caller's token-major
+// order (row, head, granule) so that the reads of the new chunk are fully coalesced.
+__global__ void __launch_bounds__(256) current_kernel(const CurrentArgs a) {
+  const int gpr = a.head_dim / 8;
+  const uint32_t per_row = (uint32_t)(a.heads * gpr);
+  const uint32_t total = (uint32_t)a.rows * per_row;   // < 2^31 (checked at configuration)
+  const int nh_new = a.nh_old + a.rows / a.F;
+  const int lo_new = a.W > 0 ? max(a.S, nh_new - a.W) : a.S;
+  for (uint32_t g = blockIdx.x * blockDim.x + threadIdx.x; g < total; g += gridDim.x * blockDim.x) {
+    const int row = (int)(g / per_row);
+    const int rem = (int)(g - row * per_row);
+    const int h = rem / gpr;
+    const int c = rem - h * gpr;
+    const int64_t vo = (int64_t)row * a.head_dim + c * 8;
+    bool to_page = false, to_slot = false;
+    int64_t po = 0, so = 0;
+    if (a.retire) {
+      const int f = a.nh_old + row / a.F;
+      const int p = row - (row / a.F) * a.F;
+      const bool sink = f < a.S;
+      to_page = a.pageK[h] != nullptr && (sink || f >= lo_new);   // frames replaced within
+      to_slot = a.is_static[h] && (sink || f == nh_new - 1);      // the retire are skipped
+      po = ((int64_t)ring_slot(f, a.S, a.cap_nonsink) * a.F + p) * a.head_dim + c * 8;
+      so = ((int64_t)a.rows + (int64_t)(sink ? f : a.S) * a.F + p) * a.head_dim + c * 8;
+    }
+    // every load first (old granule, new granule), then the stores
+    uint4 ko = make_uint4(0, 0, 0, 0), vo4 = ko, kn = ko, vn = ko;
+    if (to_page || to_slot) {
+      ko = ld_plain(a.viewK[h] + vo);
+      vo4 = ld_plain(a.viewV[h] + vo);
+    }
+    if (a.srcK) {
+      kn = ld_stream(a.srcK + (size_t)g * 8);
+      vn = ld_stream(a.srcV + (size_t)g * 8);
+    }
+    if (to_page) {
+      st_v4(a.pageK[h] + po, ko);
+      st_v4(a.pageV[h] + po, vo4);
+    }
+    if (to_slot) {
+      st_v4(a.viewK[h] + so, ko);
+      st_v4(a.viewV[h] + so, vo4);
+    }
+    if (a.srcK) {
+      st_v4(a.viewK[h] + vo, kn);
+      st_v4(a.viewV[h] + vo, vn);
+    }
+  }
+}
+
+// token-major [rows][H][D] -> dst[h] + row*D.  Consecutive threads read consecutive
+// 16-byte granules of the source; each head's destination rows are contiguous.
+__global__ void __launch_bounds__(256) scatter_kernel(const ScatterArgs a) {
+  const int gpr = a.head_dim / 8;
+  const uint32_t per_row = (uint32_t)(a.heads * gpr);
+  const uint32_t total = (uint32_t)a.rows * per_row;   // < 2^31 (checked at configuration)
+  for (uint32_t g = blockIdx.x * blockDim.x + threadIdx.x; g < total; g += gridDim.x * blockDim.x) {
+    const uint32_t row = g / per_row;
+    const int rem = (int)(g - row * per_row);
+    const int h = rem / gpr;
+    const int c = rem - h * gpr;
+    const int64_t dst_off = (int64_t)row * a.head_dim + c * 8;
+    if (a.dstK[h]) st_v4(a.dstK[h] + dst_off, ld_stream(a.srcK + (size_t)g * 8));
+    if (a.dstV[h]) st_v4(a.dstV[h] + dst_off, ld_stream(a.srcV + (size_t)g * 8));
+  }
+}
+
+// One CTA copies one piece (<= 16 KB of keys and 16 KB of values) of one unit of one
+// dynamic head's view.  Units in view order: sink frames (n units each), kept segments
+// (ascending t*n+j), anchor frame (n units); unit u lands at view row CF + u*seg_len.
 __global__ void __launch_bounds__(256) compact_kernel(const CompactArgs a) {
   const CompactItem it = a.items[blockIdx.y];
   const int l = it.layer;
   if (!a.active[l]) return;
-  const int u = blockIdx.x;
+  const int u = blockIdx.x / a.splits;
+  const int piece = blockIdx.x - u * a.splits;
   const int n_sink_units = a.n_sink_present[l] * a.n_seg;
   const int n_keep = a.n_keep[l];
   const int units = n_sink_units + n_keep + (a.anchor[l] >= 0 ? a.n_seg : 0);
@@ -87,46 +127,54 @@ __global__ void __launch_bounds__(256) compact_kernel(const CompactArgs a) {
   const int64_t src_off = ((int64_t)slot * a.F + (int64_t)seg * a.seg_len) * a.D;
   const int64_t dst_off = ((int64_t)a.CF + (int64_t)u * a.seg_len) * a.D;
   const int64_t n = (int64_t)a.seg_len * a.D / 8;      // 16-byte granules per tensor
+  const int64_t g0 = (int64_t)piece * (kCompactPiece / 16);
   const uint4* sK = reinterpret_cast<const uint4*>(it.pagesK + src_off);
   const uint4* sV = reinterpret_cast<const uint4*>(it.pagesV + src_off);
   uint4* dK = reinterpret_cast<uint4*>(it.viewK + dst_off);
   uint4* dV = reinterpret_cast<uint4*>(it.viewV + dst_off);
-  int64_t i = threadIdx.x;
-  for (; i + 256 < n; i += 512) {
-    uint4 k0 = ld_stream(sK + i), k1 = ld_stream(sK + i + 256);
-    uint4 v0 = ld_stream(sV + i), v1 = ld_stream(sV + i + 256);
-    st_v4(dK + i, k0); st_v4(dK + i + 256, k1);
-    st_v4(dV + i, v0); st_v4(dV + i + 256, v1);
+  constexpr int kPer = kCompactPiece / 16 / 256;         // granules per thread and tensor
+  uint4 k[kPer], v[kPer];
+#pragma unroll
+  for (int r = 0; r < kPer; ++r) {
+    const int64_t i = g0 + threadIdx.x + r * 256;
+    if (i < n) {
+      k[r] = ld_stream(sK + i);
+      v[r] = ld_stream(sV + i);
+    }
   }
-  for (; i < n; i += 256) {
-    st_v4(dK + i, ld_stream(sK + i));
-    st_v4(dV + i, ld_stream(sV + i));
+#pragma unroll
+  for (int r = 0; r < kPer; ++r) {
+    const int64_t i = g0 + threadIdx.x + r * 256;
+    if (i < n) {
+      st_v4(dK + i, k[r]);
+      st_v4(dV + i, v[r]);
+    }
   }
+}
+
+unsigned grid_for(int64_t granules) {
+  int64_t blocks = (granules + 255) / 256;
+  if (blocks > 152 * 16) blocks = 152 * 16;
+  return (unsigned)(blocks < 1 ? 1 : blocks);
 }
 
 }  // namespace
 
+void launch_current(const CurrentArgs& a, cudaStream_t s) {
+  const int64_t total = (int64_t)a.rows * a.heads * (a.head_dim / 8);
+  if (total == 0) return;
+  current_kernel<<<grid_for(total), 256, 0, s>>>(a);
+}
+
 void launch_scatter(const ScatterArgs& a, cudaStream_t s) {
   const int64_t total = (int64_t)a.rows * a.heads * (a.head_dim / 8);
   if (total == 0) return;
-  int64_t blocks = (total + 255) / 256;
-  if (blocks > 152 * 16) blocks = 152 * 16;
-  scatter_kernel<<<(unsigned)blocks, 256, 0, s>>>(a);
-}
-
-void launch_copy_jobs(const CopyJobs& j, cudaStream_t s) {
-  if (j.n == 0) return;
-  int64_t maxb = 0;
-  for (int i = 0; i < j.n; ++i) maxb = j.job[i].bytes > maxb ? j.job[i].bytes : maxb;
-  int64_t bx = (maxb / 16 + 1023) / 1024;
-  if (bx < 1) bx = 1;
-  if (bx > 64) bx = 64;
-  copy_jobs_kernel<<<dim3((unsigned)bx, (unsigned)j.n), 256, 0, s>>>(j);
+  scatter_kernel<<<grid_for(total), 256, 0, s>>>(a);
 }
 
 void launch_compact(const CompactArgs& a, cudaStream_t s) {
   if (a.n_items == 0 || a.max_units == 0) return;
-  compact_kernel<<<dim3((unsigned)a.max_units, (unsigned)a.n_items), 256, 0, s>>>(a);
+  compact_kernel<<<dim3((unsigned)(a.max_units * a.splits), (unsigned)a.n_items), 256, 0, s>>>(a);
 }
 
 }  // namespace fk

@@ -12,7 +12,8 @@
 //                (dynamic heads; every head of layer 0 under layer-0 pooled scoring);
 //                frame f lives in slot f (f < S) or S + (f - S) mod cap_nonsink.
 //   scores       fp32 [target][ring_slots][n]; kept lists int32 [target][kmax];
-//                scoring partials int64 (scratch); status word; host-input staging.
+//                int64 scoring sums and CTA counters (scratch); status word;
+//                host-input staging.
 #include <algorithm>
 #include <cmath>
 #include <cstdio>
@@ -92,7 +93,8 @@ struct fk_handle {
   int64_t view_rows_total = 0;
   float* scores = nullptr;
   int* kept = nullptr;
-  long long* partials = nullptr;
+  unsigned long long* sums = nullptr;
+  int* counters = nullptr;
   int* status = nullptr;
   bf16* stage_q = nullptr;
   bf16* stage_o = nullptr;
@@ -107,6 +109,7 @@ struct fk_handle {
   std::vector<int> target_layer;
   std::vector<CompactItem> compact_items;
   int max_run = 0;
+  int score_ctas = 0;
   CUtensorMap tmK{}, tmV{};
   const void* q_cached = nullptr;
   CUtensorMap tmQ{};
@@ -272,88 +275,49 @@ fk_status encode_q(CUtensorMap* m, const void* q, int Nq, int H, int D) {
   return r == CUDA_SUCCESS ? FK_OK : FK_ERR_CUDA;
 }
 
-// Move frames of `layer` into history.  K/V sources are per-head row-major views
-// (src_per_head = true: headK[h] + i*F*D) or token-major [nf*F][H][D] device buffers.
-fk_status push_history(fk_handle* h, int layer, const bf16* const* headK, const bf16* const* headV,
-                       const bf16* tokK, const bf16* tokV, int nf, cudaStream_t s) {
+// Prefill: append nf frames from token-major [nf*F][H][D] device buffers to the history.
+fk_status push_history(fk_handle* h, int layer, const bf16* tokK, const bf16* tokV, int nf,
+                       cudaStream_t s) {
   LayerState& ls = h->layers[layer];
   const int nh0 = ls.nh, nh1 = ls.nh + nf;
   const int lo1 = h->W > 0 ? std::max(h->S, nh1 - h->W) : h->S;   // window after the push
   const int64_t frame_elems = (int64_t)h->F * h->D;
-  CopyJobs jobs;
-  jobs.n = 0;
-  auto flush = [&]() -> fk_status {
-    fk_status st = launch(h, s, FK_KERNEL_APPEND, [&] { launch_copy_jobs(jobs, s); });
-    jobs.n = 0;
-    return st;
-  };
   for (int i = 0; i < nf; ++i) {
     const int f = nh0 + i;
     const bool sink = f < h->S;
     const bool in_window = sink || f >= lo1;        // frames overwritten within this push are skipped
     const bool is_anchor = !sink && f == nh1 - 1;
     if (!in_window) continue;
-    if (tokK) {
-      ScatterArgs pa{}, va{};
-      pa.srcK = tokK + (int64_t)i * h->F * h->H * h->D;
-      pa.srcV = tokV + (int64_t)i * h->F * h->H * h->D;
-      pa.rows = h->F;
-      pa.heads = h->H;
-      pa.head_dim = h->D;
-      va = pa;
-      bool any_p = false, any_v = false;
-      for (int hd = 0; hd < h->H; ++hd) {
-        const HeadBuf& hb = h->heads[layer * h->H + hd];
-        if (hb.retains) {
-          pa.dstK[hd] = hb.pageK + ring_slot(h, f) * frame_elems;
-          pa.dstV[hd] = hb.pageV + ring_slot(h, f) * frame_elems;
-          any_p = true;
-        }
-        if (hb.is_static && (sink || is_anchor)) {
-          const int64_t row = h->CF + (int64_t)(sink ? f : h->S) * h->F;
-          va.dstK[hd] = hb.viewK + row * h->D;
-          va.dstV[hd] = hb.viewV + row * h->D;
-          any_v = true;
-        }
+    ScatterArgs pa{}, va{};
+    pa.srcK = tokK + (int64_t)i * h->F * h->H * h->D;
+    pa.srcV = tokV + (int64_t)i * h->F * h->H * h->D;
+    pa.rows = h->F;
+    pa.heads = h->H;
+    pa.head_dim = h->D;
+    va = pa;
+    bool any_p = false, any_v = false;
+    for (int hd = 0; hd < h->H; ++hd) {
+      const HeadBuf& hb = h->heads[layer * h->H + hd];
+      if (hb.retains) {
+        pa.dstK[hd] = hb.pageK + ring_slot(h, f) * frame_elems;
+        pa.dstV[hd] = hb.pageV + ring_slot(h, f) * frame_elems;
+        any_p = true;
       }
-      if (any_p) {
-        fk_status st = launch(h, s, FK_KERNEL_APPEND, [&] { launch_scatter(pa, s); });
-        if (st != FK_OK) return st;
-      }
-      if (any_v) {
-        fk_status st = launch(h, s, FK_KERNEL_APPEND, [&] { launch_scatter(va, s); });
-        if (st != FK_OK) return st;
-      }
-    } else {
-      for (int hd = 0; hd < h->H; ++hd) {
-        const HeadBuf& hb = h->heads[layer * h->H + hd];
-        const bf16* sk = headK[hd] + i * frame_elems;
-        const bf16* sv = headV[hd] + i * frame_elems;
-        auto add = [&](bf16* dk, bf16* dv) -> fk_status {
-          if (jobs.n + 2 > kMaxCopyJobs) {
-            fk_status st = flush();
-            if (st != FK_OK) return st;
-          }
-          jobs.job[jobs.n++] = {sk, dk, frame_elems * 2};
-          jobs.job[jobs.n++] = {sv, dv, frame_elems * 2};
-          return FK_OK;
-        };
-        if (hb.retains) {
-          fk_status st = add(hb.pageK + ring_slot(h, f) * frame_elems,
-                             hb.pageV + ring_slot(h, f) * frame_elems);
-          if (st != FK_OK) return st;
-        }
-        if (hb.is_static && (sink || is_anchor)) {
-          const int64_t row = h->CF + (int64_t)(sink ? f : h->S) * h->F;
-          fk_status st = add(hb.viewK + row * h->D, hb.viewV + row * h->D);
-          if (st != FK_OK) return st;
-        }
+      if (hb.is_static && (sink || is_anchor)) {
+        const int64_t row = h->CF + (int64_t)(sink ? f : h->S) * h->F;
+        va.dstK[hd] = hb.viewK + row * h->D;
+        va.dstV[hd] = hb.viewV + row * h->D;
+        any_v = true;
       }
     }
-  }
-  if (jobs.n) {
-    fk_status st = flush();
-    if (st != FK_OK) return st;
+    if (any_p) {
+      fk_status st = launch(h, s, FK_KERNEL_APPEND, [&] { launch_scatter(pa, s); });
+      if (st != FK_OK) return st;
+    }
+    if (any_v) {
+      fk_status st = launch(h, s, FK_KERNEL_APPEND, [&] { launch_scatter(va, s); });
+      if (st != FK_OK) return st;
+    }
   }
   ls.nh = nh1;
   ls.dirty = true;
@@ -361,42 +325,49 @@ fk_status push_history(fk_handle* h, int layer, const bf16* const* headK, const 
   return FK_OK;
 }
 
-// The current chunk (view fronts) joins the history.
-fk_status retire_current(fk_handle* h, int layer, cudaStream_t s) {
+// One pass of the current-chunk kernel: optionally retire the current chunk (view fronts)
+// into the history, optionally write a new current chunk from K/V (host or device).
+fk_status update_current(fk_handle* h, int layer, bool retire, const void* K, const void* V,
+                         cudaStream_t s) {
   LayerState& ls = h->layers[layer];
-  if (!ls.has_current) return FK_OK;
-  if (h->W == 0 && ls.nh + h->C > h->max_hist) return FK_ERR_FULL;
-  std::vector<const bf16*> hk(h->H), hv(h->H);
-  for (int hd = 0; hd < h->H; ++hd) {
-    hk[hd] = h->heads[layer * h->H + hd].viewK;
-    hv[hd] = h->heads[layer * h->H + hd].viewV;
+  retire = retire && ls.has_current;
+  if (retire && h->W == 0 && ls.nh + h->C > h->max_hist) return FK_ERR_FULL;
+  const bf16 *k = nullptr, *v = nullptr;
+  if (K) {
+    const size_t bytes = (size_t)h->CF * h->H * h->D * 2;
+    fk_status st = stage_input(h, K, h->stage_k, bytes, s, &k);
+    if (st != FK_OK) return st;
+    st = stage_input(h, V, h->stage_v, bytes, s, &v);
+    if (st != FK_OK) return st;
   }
-  fk_status st = push_history(h, layer, hk.data(), hv.data(), nullptr, nullptr, h->C, s);
-  if (st != FK_OK) return st;
-  ls.has_current = false;
-  return FK_OK;
-}
-
-fk_status write_current(fk_handle* h, int layer, const void* K, const void* V, cudaStream_t s) {
-  const size_t bytes = (size_t)h->CF * h->H * h->D * 2;
-  const bf16 *k, *v;
-  fk_status st = stage_input(h, K, h->stage_k, bytes, s, &k);
-  if (st != FK_OK) return st;
-  st = stage_input(h, V, h->stage_v, bytes, s, &v);
-  if (st != FK_OK) return st;
-  ScatterArgs a{};
+  if (!retire && !k) return FK_OK;
+  CurrentArgs a{};
   a.srcK = k;
   a.srcV = v;
   a.rows = h->CF;
   a.heads = h->H;
   a.head_dim = h->D;
+  a.F = h->F;
+  a.S = h->S;
+  a.W = h->W;
+  a.cap_nonsink = h->cap_nonsink;
+  a.retire = retire ? 1 : 0;
+  a.nh_old = ls.nh;
   for (int hd = 0; hd < h->H; ++hd) {
-    a.dstK[hd] = h->heads[layer * h->H + hd].viewK;
-    a.dstV[hd] = h->heads[layer * h->H + hd].viewV;
+    const HeadBuf& hb = h->heads[layer * h->H + hd];
+    a.viewK[hd] = hb.viewK;
+    a.viewV[hd] = hb.viewV;
+    a.pageK[hd] = hb.retains ? hb.pageK : nullptr;
+    a.pageV[hd] = hb.retains ? hb.pageV : nullptr;
+    a.is_static[hd] = hb.is_static ? 1 : 0;
   }
-  st = launch(h, s, FK_KERNEL_APPEND, [&] { launch_scatter(a, s); });
+  fk_status st = launch(h, s, FK_KERNEL_APPEND, [&] { launch_current(a, s); });
   if (st != FK_OK) return st;
-  h->layers[layer].has_current = true;
+  if (retire) {
+    ls.nh += h->C;
+    ls.dirty = true;
+  }
+  ls.has_current = k != nullptr || (ls.has_current && !retire);
   update_lengths(h, layer);
   return FK_OK;
 }
@@ -438,6 +409,8 @@ fk_status fk_validate_config(const fk_config* c) {
   if (c->window_frames == 0 && c->max_history_frames < 1) return FK_ERR_CONFIG;
   const int64_t cf = (int64_t)c->frames_per_chunk * c->tokens_per_frame;
   if (cf > (1 << 24) || (int64_t)c->tokens_per_frame * c->head_dim > (1 << 28)) return FK_ERR_CONFIG;
+  // 16-byte granules of one chunk (all heads) are indexed with 32-bit integers
+  if (cf * c->n_heads * (c->head_dim / 8) >= ((int64_t)1 << 31)) return FK_ERR_CONFIG;
   const int64_t cap = c->window_frames > 0 ? c->window_frames
                                            : std::max(0, c->max_history_frames - c->n_sink_frames);
   if (cap > 4096 || c->n_sink_frames > 4096) return FK_ERR_CONFIG;
@@ -475,7 +448,7 @@ fk_status fk_create(const fk_config* cfg, fk_handle** out) {
   h->ring_slots = h->S + h->cap_nonsink;
   h->k_frame = (h->b * h->n) / 1000;
   h->kmax = std::max(1, keep_total(h, h->cap_nonsink - 1));
-  h->chunks = (h->seg + kScoreTokens - 1) / kScoreTokens;
+  h->chunks = (h->seg + kScoreTokensPerCta - 1) / kScoreTokensPerCta;
   h->max_run = h->cap_nonsink;
   h->heads.resize((size_t)h->L * h->H);
   h->layers.resize(h->L);
@@ -490,6 +463,7 @@ fk_status fk_create(const fk_config* cfg, fk_handle** out) {
   }
   if (!get_encode()) return fail(FK_ERR_CUDA);
   if (attention_prepare(h->D) != cudaSuccess) return fail(FK_ERR_CUDA);
+  if (score_prepare(h->D, h->cap_nonsink, h->n, &h->score_ctas) != cudaSuccess) return fail(FK_ERR_CUDA);
 
   // heads: roles, view rows, targets
   int n_dynamic = 0;
@@ -556,9 +530,11 @@ fk_status fk_create(const fk_config* cfg, fk_handle** out) {
   if ((st = dev_alloc(h, nt * h->kmax * sizeof(int), &p)) != FK_OK) return fail(st);
   h->kept = static_cast<int*>(p);
   const size_t n_items = std::max<size_t>(1, h->score_items.size());
-  if ((st = dev_alloc(h, n_items * h->max_run * h->n * h->chunks * 2 * sizeof(long long), &p)) != FK_OK)
+  if ((st = dev_alloc(h, nt * h->max_run * h->n * 2 * sizeof(unsigned long long), &p)) != FK_OK)
     return fail(st);
-  h->partials = static_cast<long long*>(p);
+  h->sums = static_cast<unsigned long long*>(p);
+  if ((st = dev_alloc(h, (nt + 2) * sizeof(int), &p)) != FK_OK) return fail(st);
+  h->counters = static_cast<int*>(p);     // [nt] per-target CTA counters, then the work counters
   if ((st = dev_alloc(h, 256, &p)) != FK_OK) return fail(st);
   h->status = static_cast<int*>(p);
   const size_t chunk_bytes = (size_t)h->CF * h->H * h->D * 2;
@@ -644,7 +620,7 @@ fk_status fk_append_frames(fk_handle* h, int layer, const void* K, const void* V
   LayerState& ls = h->layers[layer];
   const int extra = ls.has_current ? h->C : 0;
   if (h->W == 0 && ls.nh + extra + n_frames > h->max_hist) return FK_ERR_FULL;
-  if ((st = retire_current(h, layer, s)) != FK_OK) return st;
+  if ((st = update_current(h, layer, true, nullptr, nullptr, s)) != FK_OK) return st;
   const bool dev_in = n_frames > 0 && is_device_ptr(K) && is_device_ptr(V);
   const size_t frame_bytes = (size_t)h->F * h->H * h->D * 2;
   for (int f0 = 0; f0 < n_frames;) {
@@ -657,7 +633,7 @@ fk_status fk_append_frames(fk_handle* h, int layer, const void* K, const void* V
       k = h->stage_k;
       v = h->stage_v;
     }
-    if ((st = push_history(h, layer, nullptr, nullptr, k, v, nf, s)) != FK_OK) return st;
+    if ((st = push_history(h, layer, k, v, nf, s)) != FK_OK) return st;
     f0 += nf;
   }
   ls.dirty = true;
@@ -670,8 +646,7 @@ fk_status fk_append_chunk(fk_handle* h, int layer, const void* K, const void* V,
   if (!K || !V || !aligned16(K) || !aligned16(V)) return FK_ERR_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   FK_CUDA(cudaSetDevice(h->dev));
-  if ((st = retire_current(h, layer, s)) != FK_OK) return st;
-  if ((st = write_current(h, layer, K, V, s)) != FK_OK) return st;
+  if ((st = update_current(h, layer, true, K, V, s)) != FK_OK) return st;
   h->layers[layer].dirty = true;
   return FK_OK;
 }
@@ -681,7 +656,7 @@ fk_status fk_set_current(fk_handle* h, int layer, const void* K, const void* V, 
   if (st != FK_OK) return st;
   if (!K || !V || !aligned16(K) || !aligned16(V)) return FK_ERR_ARG;
   FK_CUDA(cudaSetDevice(h->dev));
-  return write_current(h, layer, K, V, static_cast<cudaStream_t>(stream));
+  return update_current(h, layer, false, K, V, static_cast<cudaStream_t>(stream));
 }
 
 fk_status fk_compress(fk_handle* h, void* stream) {
@@ -697,9 +672,8 @@ fk_status fk_compress(fk_handle* h, void* stream) {
       if (h->layers[l].nh != h->layers[0].nh) return FK_ERR_STATE;
   }
   ScoreArgs sa{};
-  SelectArgs se{};
   CompactArgs ca{};
-  bool any_run = false, any_select = false, any_compact = false;
+  bool any_run = false, any_compact = false;
   for (int l = 0; l < h->L; ++l) {
     LayerState& ls = h->layers[l];
     const Roles r = roles_of(h, ls.nh);
@@ -707,19 +681,18 @@ fk_status fk_compress(fk_handle* h, void* stream) {
     // scoring run of the layer whose keys score (every layer per head; layer 0 pooled)
     const bool scores_here = pooled_src ? l == 0 : true;
     if (ls.dirty && scores_here) {
-      int t_first = h->incremental ? std::max(r.t_lo, ls.scored_upto) : r.t_lo;
+      const int t_first = h->incremental ? std::max(r.t_lo, ls.scored_upto) : r.t_lo;
       const int last_t = r.t_lo + r.n_scoreable - 1;
       if (r.n_scoreable > 0 && t_first <= last_t) {
         sa.run[l] = {t_first, last_t + 2 - t_first};
+        sa.max_active_run = std::max(sa.max_active_run, sa.run[l].n_run);
         any_run = true;
       }
       ls.scored_upto = r.anchor >= 0 ? r.anchor : ls.scored_upto;
     }
-    se.run[l] = sa.run[l];
-    se.t_lo[l] = r.t_lo;
-    se.n_scoreable[l] = r.n_scoreable;
-    se.n_keep[l] = keep;
-    if (ls.dirty && r.n_scoreable > 0 && scores_here) any_select = true;
+    sa.t_lo[l] = r.t_lo;
+    sa.n_scoreable[l] = r.n_scoreable;
+    sa.n_keep[l] = keep;
     ca.n_sink_present[l] = r.n_sink;
     ca.n_keep[l] = keep;
     ca.anchor[l] = r.anchor;
@@ -731,6 +704,7 @@ fk_status fk_compress(fk_handle* h, void* stream) {
   fk_status st;
   if (any_run) {
     sa.items = h->d_score_items;
+    sa.targets = h->d_targets;
     sa.n_items = (int)h->score_items.size();
     sa.F = h->F;
     sa.D = h->D;
@@ -739,27 +713,20 @@ fk_status fk_compress(fk_handle* h, void* stream) {
     sa.chunks = h->chunks;
     sa.S = h->S;
     sa.cap_nonsink = h->cap_nonsink;
+    sa.ring_slots = h->ring_slots;
     sa.max_run = h->max_run;
-    sa.partials = h->partials;
+    sa.scope = h->scope;
+    sa.k_frame = h->k_frame;
+    sa.kmax = h->kmax;
+    sa.sums = h->sums;
+    sa.counters = h->counters;
+    sa.work = h->counters + (h->targets.empty() ? 1 : h->targets.size());
+    sa.max_ctas = h->score_ctas;
+    sa.n_sub_max = sa.max_active_run > 1 ? (sa.max_active_run - 2) / kScorePairsPerCta + 1 : 1;
+    sa.scores = h->scores;
+    sa.kept = h->kept;
     sa.status = h->status;
     if ((st = launch(h, s, FK_KERNEL_SCORE, [&] { launch_score(sa, s); })) != FK_OK) return st;
-  }
-  if (any_select && !h->targets.empty()) {
-    se.targets = h->d_targets;
-    se.n_targets = (int)h->targets.size();
-    se.n_seg = h->n;
-    se.chunks = h->chunks;
-    se.max_run = h->max_run;
-    se.S = h->S;
-    se.cap_nonsink = h->cap_nonsink;
-    se.ring_slots = h->ring_slots;
-    se.scope = h->scope;
-    se.k_frame = h->k_frame;
-    se.kmax = h->kmax;
-    se.partials = h->partials;
-    se.scores = h->scores;
-    se.kept = h->kept;
-    if ((st = launch(h, s, FK_KERNEL_SELECT, [&] { launch_select(se, s); })) != FK_OK) return st;
   }
   if (any_compact && ca.max_units > 0) {
     ca.items = h->d_compact_items;
@@ -772,6 +739,7 @@ fk_status fk_compress(fk_handle* h, void* stream) {
     ca.S = h->S;
     ca.cap_nonsink = h->cap_nonsink;
     ca.kmax = h->kmax;
+    ca.splits = (int)((int64_t(h->seg) * h->D * 2 + kCompactPiece - 1) / kCompactPiece);
     ca.kept = h->kept;
     if ((st = launch(h, s, FK_KERNEL_COMPACT, [&] { launch_compact(ca, s); })) != FK_OK) return st;
   }

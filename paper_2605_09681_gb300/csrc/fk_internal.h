@@ -20,13 +20,36 @@ constexpr int kMaxLayers = 256;
 constexpr int kAttnBM = 128;          // query rows per attention CTA
 constexpr int kAttnBN = 128;          // keys per attention tile
 constexpr int kViewAlignRows = 128;   // packed views are padded to whole key tiles
-constexpr int kScoreTokens = 32;      // tokens of one segment handled by one scoring CTA
+// scoring CTA: 4 warps; a token is owned by 4 lanes, so a CTA covers 32 tokens of a segment
+constexpr int kScoreThreads = 128;
+constexpr int kScoreTokensPerCta = (kScoreThreads / 32) * 8;
+constexpr int kScorePairsPerCta = 9;   // frame pairs per scoring CTA (sub-run of a run)
 
 // device status word bits (set by kernels, read by fk_sync_status)
 constexpr int kStatusRange = 1;
 constexpr int kStatusTimeout = 2;
 
 // ------------------------------------------------------------------ copy kernels
+// Current chunk update in one pass: each 16-byte granule of the previous current chunk (in
+// the view fronts) is first copied to its history location, then overwritten by the new
+// chunk's granule from the caller's token-major [C*F][H][D] buffer.
+struct CurrentArgs {
+  const bf16* srcK;             // new chunk, token-major; nullptr = retire only
+  const bf16* srcV;
+  int rows;                     // C*F
+  int heads;
+  int head_dim;
+  int F, S, W, cap_nonsink;
+  int retire;                   // 1: the previous current chunk joins the history
+  int nh_old;                   // history frames before the retire
+  bf16* viewK[kMaxHeads];       // view fronts (current chunk rows)
+  bf16* viewV[kMaxHeads];
+  bf16* pageK[kMaxHeads];       // page rings (nullptr: head keeps no history pages)
+  bf16* pageV[kMaxHeads];
+  unsigned char is_static[kMaxHeads];   // static: sink / anchor slots live in the view
+};
+void launch_current(const CurrentArgs& a, cudaStream_t s);
+
 struct ScatterArgs {            // token-major [rows][H][D] -> per-head row-major [rows][D]
   const bf16* srcK;
   const bf16* srcV;
@@ -36,20 +59,7 @@ struct ScatterArgs {            // token-major [rows][H][D] -> per-head row-majo
   bf16* dstK[kMaxHeads];        // nullptr = skip this head
   bf16* dstV[kMaxHeads];
 };
-
-struct CopyJob {                // contiguous byte copy, 16-byte granules
-  const void* src;
-  void* dst;
-  int64_t bytes;
-};
-constexpr int kMaxCopyJobs = 512;
-struct CopyJobs {
-  int n;
-  CopyJob job[kMaxCopyJobs];
-};
-
 void launch_scatter(const ScatterArgs& a, cudaStream_t s);
-void launch_copy_jobs(const CopyJobs& j, cudaStream_t s);
 
 // ------------------------------------------------------------------ scoring / selection
 struct ScoreItem {              // one (layer, head) whose keys are scored
@@ -58,46 +68,50 @@ struct ScoreItem {              // one (layer, head) whose keys are scored
   int target;
 };
 
+struct SelectTarget {           // one kept set: its layer and the score items feeding it
+  int layer;
+  int first_item;
+  int n_items;
+};
+
 struct LayerRun {               // per layer: frames t_first..t_first+n_run-1 are read
   int t_first;
   int n_run;                    // 0 = nothing to score in this layer
 };
 
+// Scoring of new frame pairs, then (in the last CTA of each target) the finish of the
+// scores and BottomK selection of that target.
 struct ScoreArgs {
   const ScoreItem* items;       // device table
+  const SelectTarget* targets;  // device table
   int n_items;
   int F, D, n_seg, seg_len, chunks;
-  int S, cap_nonsink;
-  int max_run;
-  long long* partials;          // [item][max_run][n_seg][chunks][2] : {N, Dnext}
-  int* status;
-  LayerRun run[kMaxLayers];
-};
-void launch_score(const ScoreArgs& a, cudaStream_t s);
-
-struct SelectTarget {           // per target (selection unit)
-  int layer;                    // layer whose frames the target covers
-  int first_item;               // score items feeding the target: [first_item, first_item+n_items)
-  int n_items;
-};
-
-struct SelectArgs {
-  const SelectTarget* targets;  // device table
-  int n_targets;
-  int n_seg, chunks, max_run;
   int S, cap_nonsink, ring_slots;
+  int max_run;                  // frames one target's sums can hold
+  int max_active_run;           // longest run of this launch
+  int n_sub_max;                // sub-runs of the longest run
+  int max_ctas;                 // persistent grid size
+  int* work;                    // [2]: next work unit, CTAs finished (zero between launches)
   int scope;                    // FK_SCOPE_*
   int k_frame;                  // kept per frame (per-frame scope)
   int kmax;                     // capacity of one kept list
-  const long long* partials;
+  unsigned long long* sums;     // scratch [target][max_run][n_seg][2] : {N(t), D(t-1,t)}, zero between launches
+  int* counters;                // [target], zero between launches
   float* scores;                // [target][ring_slots][n_seg]
   int* kept;                    // [target][kmax]
-  LayerRun run[kMaxLayers];     // frames scored now (as in ScoreArgs)
+  int* status;
+  LayerRun run[kMaxLayers];
   int t_lo[kMaxLayers];         // first scoreable frame of the window
   int n_scoreable[kMaxLayers];  // |T| (scoreable frames)
   int n_keep[kMaxLayers];       // kept segments of the layer's targets
 };
-void launch_select(const SelectArgs& a, cudaStream_t s);
+void launch_score(const ScoreArgs& a, cudaStream_t s);
+// dynamic shared memory limit and the persistent grid size (CTAs resident at once)
+cudaError_t score_prepare(int head_dim, int max_run, int n_seg, int* max_ctas);
+// shared memory of a scoring CTA: int32 accumulators (4 per frame) or the window's scores
+constexpr int score_smem_ints(int max_run, int n_seg) {
+  return 4 * max_run > max_run * n_seg ? 4 * max_run : max_run * n_seg;
+}
 
 struct CompactItem {            // one dynamic (layer, head)
   const bf16* pagesK;
@@ -113,6 +127,7 @@ struct CompactArgs {
   int n_items;
   int F, D, n_seg, seg_len, CF;
   int S, cap_nonsink, kmax;
+  int splits;                   // pieces per unit (each at most kCompactPiece bytes per tensor)
   const int* kept;
   int n_sink_present[kMaxLayers];
   int n_keep[kMaxLayers];
@@ -120,6 +135,7 @@ struct CompactArgs {
   unsigned char active[kMaxLayers];
   int max_units;
 };
+constexpr int kCompactPiece = 16384;
 void launch_compact(const CompactArgs& a, cudaStream_t s);
 
 // ------------------------------------------------------------------ attention

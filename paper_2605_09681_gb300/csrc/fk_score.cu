@@ -1,13 +1,17 @@
-// Segment-wise similarity scoring and BottomK selection (Sec. 4.3, Eq. 3).
+// Segment-wise similarity scoring and BottomK selection (Sec. 4.3, Eq. 3) in one launch.
 //
-// score_kernel streams the key pages of a run of consecutive history frames once,
-// 16 bytes per lane, and produces per CTA the int64 sums N_t = sum_p n_p(t) and
-// D_t = sum_p d_p(t-1, t) over its tokens of one segment (the score contract: per
-// token fp32 dot in a fixed fma/butterfly order, scaled by 2^24 and truncated to
-// int64, so that the cross-token and cross-CTA sums are exact and order-free).
-// select_kernel finishes s = D / sqrt(N_t N_{t+1}) in IEEE double, stores the fp32
-// score per frame slot, ranks the scoreable candidates by (score, segment id) and
-// stream-compacts the kept segment ids with warp ballots and prefix sums.
+// Each CTA owns a few tokens of one segment of one scored (layer, head) and streams that
+// token range through the run of consecutive history frames, 16 bytes per lane, with a
+// four-frame register prefetch ring; every key byte is read once.  Per token it forms the
+// score-contract quantities (fp32 channel dot in a fixed fma/butterfly order, scaled by 2^24
+// and truncated to int64, carried as two exact int32 halves): the squared norm n_p(t) and
+// the dot d_p(t-1, t).  Warp sums go into shared-memory int32 accumulators (at most 32
+// tokens per CTA, so no overflow) and each CTA adds them as int64 into the target's global
+// int64 sums (exact integer adds, so the order is free).  The last CTA of a selection
+// target (counted with a global atomic)
+// finishes s = D / sqrt(N_t N_{t+1}) in IEEE double, stores the fp32 scores per frame slot,
+// ranks the scoreable candidates by (score, segment id) and stream-compacts the kept
+// segment ids with warp ballots and prefix sums.
 #include "fk_internal.h"
 
 namespace fk {
@@ -20,119 +24,27 @@ __device__ __forceinline__ uint4 ld_keys(const void* p) {
   return v;
 }
 
-__device__ __forceinline__ float bf_lo(uint32_t w) { return __uint_as_float(w << 16); }
-__device__ __forceinline__ float bf_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
-
-// fp32 fma chain over the 8 channels of one 16-byte granule, channel order = memory order
-__device__ __forceinline__ float dot8(const uint4 a, const uint4 b) {
-  float acc = 0.0f;
-  acc = __fmaf_rn(bf_lo(a.x), bf_lo(b.x), acc);
-  acc = __fmaf_rn(bf_hi(a.x), bf_hi(b.x), acc);
-  acc = __fmaf_rn(bf_lo(a.y), bf_lo(b.y), acc);
-  acc = __fmaf_rn(bf_hi(a.y), bf_hi(b.y), acc);
-  acc = __fmaf_rn(bf_lo(a.z), bf_lo(b.z), acc);
-  acc = __fmaf_rn(bf_hi(a.z), bf_hi(b.z), acc);
-  acc = __fmaf_rn(bf_lo(a.w), bf_lo(b.w), acc);
-  acc = __fmaf_rn(bf_hi(a.w), bf_hi(b.w), acc);
-  return acc;
+// Two channels (one 32-bit word: low half first) of the norm and dot fma chains, with the
+// bf16 values used directly as fma operands (fp32 product and accumulation, one rounding):
+// n += c*c and d += p*c for the low channel, then for the high channel.
+__device__ __forceinline__ void fma_word(uint32_t cw, uint32_t pw, float& n, float& d) {
+  asm("{\n .reg .b16 cl, ch, pl, ph;\n mov.b32 {cl, ch}, %2;\n mov.b32 {pl, ph}, %3;\n"
+      " fma.rn.f32.bf16 %0, cl, cl, %0;\n fma.rn.f32.bf16 %1, pl, cl, %1;\n"
+      " fma.rn.f32.bf16 %0, ch, ch, %0;\n fma.rn.f32.bf16 %1, ph, ch, %1;\n}"
+      : "+f"(n), "+f"(d) : "r"(cw), "r"(pw));
 }
 
-// butterfly over the LPT lanes that own one token: p[g] += p[g ^ s], s = LPT/2 .. 1
-template <int LPT>
-__device__ __forceinline__ float token_reduce(float v) {
-#pragma unroll
-  for (int s = LPT / 2; s >= 1; s >>= 1) v = __fadd_rn(v, __shfl_xor_sync(0xffffffffu, v, s));
-  return v;
-}
-
-__device__ __forceinline__ unsigned long long fixed24(float v) {
-  return (unsigned long long)__float2ll_rz(__fmul_rn(v, 16777216.0f));
-}
-
-__device__ __forceinline__ unsigned long long warp_sum_u64(unsigned long long v) {
-#pragma unroll
-  for (int s = 16; s >= 1; s >>= 1) v += __shfl_xor_sync(0xffffffffu, v, s);
-  return v;
+// trunc(v * 2^24) = hi * 2^24 + lo exactly, as two int32: hi = trunc(v) (|hi| <= 2^23 under
+// the precondition), v - hi is exact in fp32 (the low-order bits of v), lo = trunc((v - hi) *
+// 2^24) with |lo| < 2^24; hi and lo carry the sign of v, so both truncations go toward zero.
+// 32-bit conversions only (a float-to-int64 conversion would run on the FP64 pipe).
+__device__ __forceinline__ void fixed24_split(float v, int& hi, int& lo) {
+  hi = __float2int_rz(v);
+  lo = __float2int_rz(__fmul_rn(__fsub_rn(v, __int2float_rn(hi)), 16777216.0f));
 }
 
 __device__ __forceinline__ int ring_slot(int f, int S, int cap) {
   return f < S ? f : S + (f - S) % cap;
-}
-
-// D = head_dim; LPT = lanes per token (one 16-byte granule each)
-template <int D>
-__global__ void __launch_bounds__(256) score_kernel(const ScoreArgs a) {
-  constexpr int LPT = D / 8;
-  constexpr int TPW = 32 / LPT;                // tokens per warp per pass
-  constexpr int TPP = 8 * TPW;                 // tokens per CTA per pass
-  constexpr int PASSES = kScoreTokens / TPP;   // passes per frame
-  static_assert(PASSES >= 1 && kScoreTokens % TPP == 0, "token tiling");
-  __shared__ unsigned long long red[8][2];
-
-  const ScoreItem it = a.items[blockIdx.y];
-  const LayerRun run = a.run[it.layer];
-  if (run.n_run == 0) return;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int j = blockIdx.x / a.chunks;
-  const int c = blockIdx.x - j * a.chunks;
-  const int seg_lo = j * a.seg_len;
-  const int tok0 = seg_lo + c * kScoreTokens;
-  const int tok_end = min(tok0 + kScoreTokens, seg_lo + a.seg_len);
-  const int g = lane % LPT;
-  const int sub = lane / LPT;
-
-  int tok[PASSES];
-  bool ok[PASSES];
-#pragma unroll
-  for (int p = 0; p < PASSES; ++p) {
-    tok[p] = tok0 + p * TPP + warp * TPW + sub;
-    ok[p] = tok[p] < tok_end;
-  }
-
-  uint4 prev[PASSES], cur[PASSES];
-  const uint4 zero = make_uint4(0, 0, 0, 0);
-  auto load_frame = [&](int k, uint4 (&dst)[PASSES]) {
-    const int slot = ring_slot(run.t_first + k, a.S, a.cap_nonsink);
-    const bf16* base = it.pagesK + (int64_t)slot * a.F * D;
-#pragma unroll
-    for (int p = 0; p < PASSES; ++p)
-      dst[p] = ok[p] ? ld_keys(base + (int64_t)tok[p] * D + g * 8) : zero;
-  };
-
-  load_frame(0, cur);
-  for (int k = 0; k < run.n_run; ++k) {
-    uint4 nxt[PASSES];
-    if (k + 1 < run.n_run) load_frame(k + 1, nxt);   // one frame of prefetch
-    unsigned long long accN = 0, accD = 0;
-    bool bad = false;
-#pragma unroll
-    for (int p = 0; p < PASSES; ++p) {
-      const float np = token_reduce<LPT>(dot8(cur[p], cur[p]));
-      float dp = 0.0f;
-      if (k > 0) dp = token_reduce<LPT>(dot8(prev[p], cur[p]));
-      if (g == 0 && ok[p]) {
-        bad |= !(np <= 8388608.0f);
-        accN += fixed24(np);
-        accD += fixed24(dp);
-      }
-    }
-    if (bad) atomicOr(a.status, kStatusRange);
-    accN = warp_sum_u64(accN);
-    accD = warp_sum_u64(accD);
-    if (lane == 0) { red[warp][0] = accN; red[warp][1] = accD; }
-    __syncthreads();
-    if (threadIdx.x == 0) {
-      unsigned long long sN = 0, sD = 0;
-#pragma unroll
-      for (int w = 0; w < 8; ++w) { sN += red[w][0]; sD += red[w][1]; }
-      const int64_t idx =
-          (((int64_t)blockIdx.y * a.max_run + k) * a.n_seg + j) * a.chunks + c;
-      reinterpret_cast<longlong2*>(a.partials)[idx] = make_longlong2((long long)sN, (long long)sD);
-    }
-    __syncthreads();
-#pragma unroll
-    for (int p = 0; p < PASSES; ++p) { prev[p] = cur[p]; if (k + 1 < run.n_run) cur[p] = nxt[p]; }
-  }
 }
 
 __device__ __forceinline__ float finish_score(long long dsum, long long n1, long long n2) {
@@ -141,46 +53,46 @@ __device__ __forceinline__ float finish_score(long long dsum, long long n1, long
   return __double2float_rn(__ddiv_rn(__ll2double_rn(dsum), den));
 }
 
-// one CTA per selection target
-__global__ void __launch_bounds__(256) select_kernel(const SelectArgs a) {
-  __shared__ int warp_tot[8];
+// Finish the scored pairs of target `tgi` and select its kept segments (one CTA).
+__device__ void finish_and_select(const ScoreArgs& a, int tgi, int* stage) {
+  __shared__ int warp_tot[32];
   __shared__ int base_off;
-  const SelectTarget tg = a.targets[blockIdx.x];
+  const SelectTarget tg = a.targets[tgi];
   const int l = tg.layer;
   const LayerRun run = a.run[l];
   const int n = a.n_seg;
-  float* sc = a.scores + (int64_t)blockIdx.x * a.ring_slots * n;
+  float* sc = a.scores + (int64_t)tgi * a.ring_slots * n;
 
-  // 1. finish the pairs (t, t+1) scored by this launch
+  // 1. finish the pairs (t, t+1) scored by this launch from the target's int64 sums
+  //    (read past L1: other CTAs added them), then clear the sums for the next launch
+  unsigned long long* sums = a.sums + (int64_t)tgi * a.max_run * n * 2;
   if (run.n_run >= 2) {
     const int pairs = (run.n_run - 1) * n;
     for (int idx = threadIdx.x; idx < pairs; idx += blockDim.x) {
       const int k = idx / n, j = idx - k * n;
-      long long N1 = 0, N2 = 0, Dd = 0;
-      for (int i = 0; i < tg.n_items; ++i) {
-        const longlong2* P = reinterpret_cast<const longlong2*>(a.partials) +
-                             ((int64_t)(tg.first_item + i) * a.max_run) * n * a.chunks;
-        for (int c = 0; c < a.chunks; ++c) {
-          const longlong2 x = P[((int64_t)k * n + j) * a.chunks + c];
-          const longlong2 y = P[((int64_t)(k + 1) * n + j) * a.chunks + c];
-          N1 += x.x;
-          N2 += y.x;
-          Dd += y.y;
-        }
-      }
+      const unsigned long long N1 = __ldcg(sums + ((int64_t)k * n + j) * 2);
+      const unsigned long long N2 = __ldcg(sums + ((int64_t)(k + 1) * n + j) * 2);
+      const unsigned long long Dd = __ldcg(sums + ((int64_t)(k + 1) * n + j) * 2 + 1);
       const int slot = ring_slot(run.t_first + k, a.S, a.cap_nonsink);
-      sc[slot * n + j] = finish_score(Dd, N1, N2);
+      sc[slot * n + j] = finish_score((long long)Dd, (long long)N1, (long long)N2);
     }
   }
   __syncthreads();
+  for (int i = threadIdx.x; i < run.n_run * n * 2; i += blockDim.x) sums[i] = 0ull;
 
-  // 2. BottomK over the scoreable frames, compacted in ascending segment-id order
+  // 2. BottomK over the scoreable frames, compacted in ascending segment-id order; the
+  //    window's scores are staged in shared memory in candidate order (t - t_lo)*n + j
   const int nT = a.n_scoreable[l];
   const int M = nT * n;
   const int K = a.n_keep[l];
   const int t_lo = a.t_lo[l];
-  int* out = a.kept + (int64_t)blockIdx.x * a.kmax;
+  int* out = a.kept + (int64_t)tgi * a.kmax;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  float* ssc = reinterpret_cast<float*>(stage);
+  for (int idx = threadIdx.x; idx < M; idx += blockDim.x) {
+    const int t = t_lo + idx / n, jj = idx - (idx / n) * n;
+    ssc[idx] = __ldcg(sc + ring_slot(t, a.S, a.cap_nonsink) * n + jj);
+  }
   if (threadIdx.x == 0) base_off = 0;
   __syncthreads();
   for (int b0 = 0; b0 < M; b0 += blockDim.x) {
@@ -190,20 +102,19 @@ __global__ void __launch_bounds__(256) select_kernel(const SelectArgs a) {
     if (idx < M) {
       t = t_lo + idx / n;
       j = idx - (idx / n) * n;
-      const float s = sc[ring_slot(t, a.S, a.cap_nonsink) * n + j];
+      const float* row = ssc + (idx - j);
+      const float s = row[j];
       int rank = 0;
       if (a.scope == FK_SCOPE_PER_FRAME) {
-        const float* row = sc + ring_slot(t, a.S, a.cap_nonsink) * n;
         for (int jj = 0; jj < n; ++jj) {
           const float o = row[jj];
           rank += (o < s) || (o == s && jj < j);
         }
         keep = rank < a.k_frame;
       } else {
-        for (int q = 0; q < M; ++q) {
-          const int tq = t_lo + q / n, jq = q - (q / n) * n;
-          const float o = sc[ring_slot(tq, a.S, a.cap_nonsink) * n + jq];
-          rank += (o < s) || (o == s && q < idx);
+        for (int qq = 0; qq < M; ++qq) {
+          const float o = ssc[qq];
+          rank += (o < s) || (o == s && qq < idx);
         }
         keep = rank < K;
       }
@@ -218,25 +129,213 @@ __global__ void __launch_bounds__(256) select_kernel(const SelectArgs a) {
     __syncthreads();
     if (threadIdx.x == 0) {
       int tot = 0;
-      for (int w = 0; w < 8; ++w) tot += warp_tot[w];
+      for (int w = 0; w < (int)(blockDim.x >> 5); ++w) tot += warp_tot[w];
       base_off += tot;
     }
     __syncthreads();
   }
 }
 
+// D = head_dim.  Four lanes own one token: lane q of the token holds channel groups
+// 4i + q, i < GPL (GPL = D/32 groups of 8 channels, one 16-byte granule each), so each
+// load instruction reads 64 contiguous bytes per token; a warp covers 8 tokens and a
+// 128-thread CTA 32 tokens of one segment.
+// One work unit: item y, segment j, token chunk c, sub-run z (block-uniform arguments).
+template <int D>
+__device__ __forceinline__ void score_unit(const ScoreArgs& a, int y, int j, int c, int z,
+                                           int* acc32, int& is_last) {
+  constexpr int LPT = 4;                       // lanes per token
+  constexpr int GPL = D / 32;                  // granules (channel groups) per lane
+  constexpr int TPW = 32 / LPT;                // tokens per warp
+  constexpr int TB = (kScoreThreads / 32) * TPW;
+  constexpr int PF = 4;                        // ring of packed frames per lane
+  const ScoreItem it = a.items[y];
+  const LayerRun run = a.run[it.layer];
+  // sub-run blockIdx.z: frames k_lo .. k_hi of the run (pairs (k-1, k) for k_lo < k <= k_hi);
+  // a sub-run's first frame is the previous sub-run's last one, whose norm that one counts
+  const int n_sub = run.n_run > 1 ? (run.n_run - 2) / kScorePairsPerCta + 1 : 1;
+  if (run.n_run == 0 || z >= n_sub) return;
+  const int k_lo = z * kScorePairsPerCta;
+  const int k_hi = min(k_lo + kScorePairsPerCta, run.n_run - 1);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int seg_lo = j * a.seg_len;
+  const int tok0 = seg_lo + c * TB;
+  const int tok_end = min(tok0 + TB, seg_lo + a.seg_len);
+  const int q = lane % LPT;                    // lane within the token
+  const int tok = tok0 + warp * TPW + lane / LPT;
+  const bool ok = tok < tok_end;
+
+  for (int i = threadIdx.x; i < 4 * run.n_run; i += blockDim.x) acc32[i] = 0;
+  __syncthreads();
+
+  const bf16* base = it.pagesK + (int64_t)tok * D + q * 8;
+  const int64_t frame_elems = (int64_t)a.F * D;
+  // ring slot of the next frame to load; scored frames are never sinks, so the slot
+  // advances by one and wraps from the last slot to the first non-sink slot
+  const int slot_end = a.S + a.cap_nonsink;
+  int next_slot = ring_slot(run.t_first + k_lo, a.S, a.cap_nonsink);
+  auto load = [&](int k, uint4 (&dst)[GPL]) {
+#pragma unroll
+    for (int i = 0; i < GPL; ++i) dst[i] = make_uint4(0, 0, 0, 0);
+    if (k <= k_hi) {
+      if (ok) {
+        const bf16* p = base + (int64_t)next_slot * frame_elems;
+#pragma unroll
+        for (int i = 0; i < GPL; ++i) dst[i] = ld_keys(p + i * 32);
+      }
+      next_slot = next_slot + 1 == slot_end ? a.S : next_slot + 1;
+    }
+  };
+  // ring of PF packed frames: frame k lives in buf[(k - k_lo) % PF]; the previous frame is
+  // the previous slot, and a slot is refilled (PF - 1 frames ahead) once it has served as
+  // "previous"
+  uint4 buf[PF][GPL];
+#pragma unroll
+  for (int u = 0; u < PF - 1; ++u) load(k_lo + u, buf[u]);
+#pragma unroll
+  for (int i = 0; i < GPL; ++i) buf[PF - 1][i] = make_uint4(0, 0, 0, 0);   // "previous" of k_lo
+  bool bad = false;
+  for (int k0 = k_lo; k0 <= k_hi; k0 += PF) {
+#pragma unroll
+    for (int u = 0; u < PF; ++u) {
+      const int k = k0 + u;
+      if (k > k_hi) break;
+      const uint4 (&cur)[GPL] = buf[u];
+      const uint4 (&prv)[GPL] = buf[(u + PF - 1) % PF];
+      // one fma chain per channel group (channel order), for n_p and d_p
+      float n[GPL], d[GPL];
+#pragma unroll
+      for (int i = 0; i < GPL; ++i) {
+        n[i] = 0.0f;
+        d[i] = 0.0f;
+        fma_word(cur[i].x, prv[i].x, n[i], d[i]);
+        fma_word(cur[i].y, prv[i].y, n[i], d[i]);
+        fma_word(cur[i].z, prv[i].z, n[i], d[i]);
+        fma_word(cur[i].w, prv[i].w, n[i], d[i]);
+      }
+      load(k + PF - 1, buf[(u + PF - 1) % PF]);   // the previous frame's slot is free now
+      // butterfly p[g] += p[g ^ s], s = D/16 .. 1 over groups g = 4i + q: strides s >= 4 pair
+      // i with i ^ (s/4) inside the lane, strides 2 and 1 pair lane q with q ^ s
+#pragma unroll
+      for (int sft = GPL / 2; sft >= 1; sft >>= 1) {
+#pragma unroll
+        for (int i = 0; i < GPL; ++i) {
+          if ((i & sft) == 0) {
+            const float nn = __fadd_rn(n[i], n[i ^ sft]);
+            const float dd = __fadd_rn(d[i], d[i ^ sft]);
+            n[i] = nn; n[i ^ sft] = nn;
+            d[i] = dd; d[i ^ sft] = dd;
+          }
+        }
+      }
+#pragma unroll
+      for (int sft = 2; sft >= 1; sft >>= 1) {
+        n[0] = __fadd_rn(n[0], __shfl_xor_sync(0xffffffffu, n[0], sft));
+        d[0] = __fadd_rn(d[0], __shfl_xor_sync(0xffffffffu, d[0], sft));
+      }
+      const float np = n[0];
+      const float dp = d[0];                     // 0 for the first frame of the run
+      // lane q = 0 of a token converts n_p, lane q = 1 converts d_p (then summed over the
+      // warp's tokens); the other lanes contribute zero
+      // the norm of a sub-run's last frame belongs to the next sub-run (except at the end)
+      const bool count_n = k < k_hi || k_hi == run.n_run - 1;
+      int hi = 0, lo = 0;
+      if (ok && q < 2) {
+        const float v = q == 0 ? (count_n ? np : 0.0f) : (k > k_lo ? dp : 0.0f);
+        if (q == 0) bad |= !(np <= 8388608.0f);
+        fixed24_split(v, hi, lo);
+      }
+#pragma unroll
+      for (int sft = LPT; sft < 32; sft <<= 1) {
+        hi += __shfl_xor_sync(0xffffffffu, hi, sft);
+        lo += __shfl_xor_sync(0xffffffffu, lo, sft);
+      }
+      if (lane < 2) {                            // lane 0: N(t) parts, lane 1: D(t-1, t) parts
+        atomicAdd(&acc32[4 * k + 2 * lane], hi);
+        atomicAdd(&acc32[4 * k + 2 * lane + 1], lo);
+      }
+    }
+  }
+  if (bad) atomicOr(a.status, kStatusRange);
+  __syncthreads();
+  unsigned long long* sums = a.sums + (int64_t)it.target * a.max_run * a.n_seg * 2;
+  for (int qq = 2 * k_lo + threadIdx.x; qq < 2 * (k_hi + 1); qq += blockDim.x) {
+    const int k = qq >> 1, which = qq & 1;
+    const long long v = (long long)acc32[4 * k + 2 * which] * 16777216ll + (long long)acc32[4 * k + 2 * which + 1];
+    atomicAdd(sums + ((int64_t)k * a.n_seg + j) * 2 + which, (unsigned long long)v);
+  }
+
+  // the last CTA of this item's selection target finishes it
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    const SelectTarget tg = a.targets[it.target];
+    const int expected = a.n_seg * a.chunks * tg.n_items * n_sub;
+    is_last = atomicAdd(&a.counters[it.target], 1) == expected - 1;
+  }
+  __syncthreads();
+  if (!is_last) return;
+  __threadfence();
+  finish_and_select(a, it.target, acc32);
+  if (threadIdx.x == 0) a.counters[it.target] = 0;
+  __syncthreads();                               // acc32 is reused by the next unit
+}
+
+// Persistent grid (one wave): CTAs take work units from a global counter until none is left;
+// the last CTA to leave resets the counter for the next launch.
+template <int D>
+__global__ void __launch_bounds__(kScoreThreads, 4) score_kernel(const ScoreArgs a) {
+  extern __shared__ int acc32[];               // [n_run][4] : {N hi, N lo, D hi, D lo}
+  __shared__ int s_unit, is_last;
+  const int per_sub = a.n_seg * a.chunks;
+  const int per_item = per_sub * a.n_sub_max;
+  const int total = a.n_items * per_item;
+  for (;;) {
+    if (threadIdx.x == 0) s_unit = atomicAdd(a.work, 1);
+    __syncthreads();
+    const int unit = s_unit;
+    __syncthreads();
+    if (unit >= total) break;
+    const int y = unit / per_item;
+    const int r = unit - y * per_item;
+    const int z = r / per_sub;
+    const int r2 = r - z * per_sub;
+    const int j = r2 / a.chunks;
+    score_unit<D>(a, y, j, r2 - j * a.chunks, z, acc32, is_last);
+  }
+  if (threadIdx.x == 0) {
+    __threadfence();
+    if (atomicAdd(a.work + 1, 1) == (int)gridDim.x - 1) {
+      a.work[0] = 0;
+      a.work[1] = 0;
+    }
+  }
+}
+
 }  // namespace
+
+cudaError_t score_prepare(int head_dim, int max_run, int n_seg, int* max_ctas) {
+  const int smem = score_smem_ints(max_run, n_seg) * (int)sizeof(int);
+  const void* fn = head_dim == 128 ? (const void*)score_kernel<128> : (const void*)score_kernel<64>;
+  cudaError_t e = cudaSuccess;
+  if (smem > 48 * 1024) e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e != cudaSuccess) return e;
+  int dev = 0, sms = 0, per_sm = 0;
+  if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+  if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+  if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, kScoreThreads, smem)) != cudaSuccess)
+    return e;
+  *max_ctas = sms * (per_sm > 0 ? per_sm : 1);
+  return cudaSuccess;
+}
 
 void launch_score(const ScoreArgs& a, cudaStream_t s) {
   if (a.n_items == 0) return;
-  dim3 grid((unsigned)(a.n_seg * a.chunks), (unsigned)a.n_items);
-  if (a.D == 128) score_kernel<128><<<grid, 256, 0, s>>>(a);
-  else score_kernel<64><<<grid, 256, 0, s>>>(a);
-}
-
-void launch_select(const SelectArgs& a, cudaStream_t s) {
-  if (a.n_targets == 0) return;
-  select_kernel<<<(unsigned)a.n_targets, 256, 0, s>>>(a);
+  const int64_t units = (int64_t)a.n_items * a.n_seg * a.chunks * a.n_sub_max;
+  const unsigned grid = (unsigned)(units < a.max_ctas ? units : a.max_ctas);
+  const size_t smem = (size_t)score_smem_ints(a.max_run, a.n_seg) * sizeof(int);
+  if (a.D == 128) score_kernel<128><<<grid, kScoreThreads, smem, s>>>(a);
+  else score_kernel<64><<<grid, kScoreThreads, smem, s>>>(a);
 }
 
 }  // namespace fk
