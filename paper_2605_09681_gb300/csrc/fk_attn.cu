@@ -80,9 +80,10 @@ __device__ __forceinline__ bool mbar_test(uint64_t* b, uint32_t parity) {
 }
 
 // Bounded wait for the phase of parity `parity`.  Returns false when the CTA is
-// aborting or the limit expired (which starts the abort).
-__device__ __noinline__ bool wait_phase(uint64_t* b, uint32_t parity, AttnBarriers* bar,
-                                        int* status, bool honour_abort = true) {
+// aborting or the limit expired (which starts the abort).  Inlined: a call would save and
+// restore the caller's live registers on every wait, even when the phase is complete.
+__device__ __forceinline__ bool wait_phase(uint64_t* b, uint32_t parity, AttnBarriers* bar,
+                                           int* status, bool honour_abort = true) {
   if (mbar_test(b, parity)) return true;
   const uint64_t t0 = now_ns();
   while (true) {
