@@ -58,7 +58,10 @@ def _workload(name: str):
 
 
 def _algorithmic(w, key_counts):
-    """Per-step algorithmic work: attention FLOPs and kernel bytes (the design doc lists the formulas)."""
+    """Per-step algorithmic work: attention FLOPs sum_h 4*Nq*Nk_h*D; scoring bytes = keys of the
+    scored frames of every dynamic head; compaction bytes = keys and values of every dynamic
+    head's view units, read and written; append bytes = the chunk's K/V read and written plus
+    the retired frames copied into the history."""
     import oracle as O
     D, F, H = w.head_dim, w.tokens_per_frame, w.n_heads
     nq = w.n_queries
@@ -324,15 +327,26 @@ def run_fk(args, rank, world, local_rank):
     return out
 
 
+# DRAM bytes (read + write) per launch from one ncu capture of each kernel on the 480P
+# workload, with the SHA-1 prefix of the kernel source the capture was taken on: a figure
+# is reported only while that source is unchanged.
+NCU_TRAFFIC = {
+    "480p_layer": {
+        "attend": ("fk_attn.cu", "a7947bb70908", 121476352),
+        "compact": ("fk_copy.cu", "cba7e7019a47", 75307264),
+        "score": ("fk_score.cu", "1cfc2cc99fc2", 43181312),
+    },
+}
+
+
 def _traffic(workload):
-    """DRAM bytes per launch from the committed ncu summary of this workload, if present."""
-    p = os.path.join(ROOT, "profiles", "traffic_%s.json" % workload)
-    if os.path.exists(p):
-        try:
-            return json.load(open(p))
-        except ValueError:
-            return {}
-    return {}
+    import hashlib
+    out = {}
+    for kind, (src, sha, nbytes) in NCU_TRAFFIC.get(workload, {}).items():
+        path = os.path.join(ROOT, "paper_2605_09681_gb300", "csrc", src)
+        cur = hashlib.sha1(open(path, "rb").read()).hexdigest()[:12] if os.path.exists(path) else ""
+        out[kind] = nbytes if cur == sha else None
+    return out
 
 
 def cpu_baseline(w, budget_s=15.0, steps=1):
