@@ -62,20 +62,22 @@ def _algorithmic(w, key_counts):
     scored frames of every dynamic head; compaction bytes = keys and values of every dynamic
     head's view units, read and written; append bytes = the chunk's K/V read and written plus
     the retired frames copied into the history."""
-    import oracle as O
     D, F, H = w.head_dim, w.tokens_per_frame, w.n_heads
     nq = w.n_queries
     flops = sum(4.0 * nq * nk * D for nk in key_counts)
-    roles = O.frame_roles(w.n_history_frames, w.n_sink_frames, w.window_frames)
-    n_dyn = sum(1 for nk, st in zip(key_counts, _workload_static(w)) if not st)
-    run_frames = len(roles.scoreable) + 1 if roles.scoreable else 0
-    score_bytes = n_dyn * run_frames * F * D * 2
-    n_keep = len(roles.scoreable) * O.keep_count(w.keep_budget_permille, w.n_segments)
-    units_tokens = len(roles.sink) * F + n_keep * (F // w.n_segments) + (F if roles.anchor is not None else 0)
-    compact_bytes = n_dyn * 2 * 2 * units_tokens * D * 2
+    nh, S, Wn = w.n_history_frames, w.n_sink_frames, w.window_frames
+    n_sink = min(S, nh)
+    lo = max(S, nh - Wn) if Wn > 0 else S
+    has_anchor = nh - 1 >= lo
+    n_scoreable = (nh - 1 - lo) if has_anchor else 0
+    static = _workload_static(w)
+    n_dyn = sum(1 for st in static if not st)
+    score_bytes = n_dyn * (n_scoreable + 1 if n_scoreable else 0) * F * D * 2
+    n_keep = n_scoreable * (w.keep_budget_permille * w.n_segments // 1000)
+    unit_tokens = n_sink * F + n_keep * (F // w.n_segments) + (F if has_anchor else 0)
+    compact_bytes = n_dyn * 2 * 2 * unit_tokens * D * 2
     append_bytes = 2 * 2 * nq * H * D * 2 + sum(
-        2 * 2 * w.frames_per_chunk * F * D * 2 if not st else 2 * 2 * F * D * 2
-        for st in _workload_static(w))
+        2 * 2 * (F if st else w.frames_per_chunk * F) * D * 2 for st in static)
     return dict(attn_flops=flops, score_bytes=score_bytes, compact_bytes=compact_bytes,
                 append_bytes=append_bytes)
 
