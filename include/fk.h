@@ -181,6 +181,27 @@ FK_API fk_status fk_profile_reset(fk_handle* h);
 /* Kernels launched by this handle since creation (all kinds). */
 FK_API int64_t fk_launch_count(const fk_handle* h);
 
+/* Segment scores of consecutive frames of one head without allocating any memory.
+ * The paper has no counterpart: this is a service entry point of this library.  It is for
+ * callers that must not call cudaMalloc: code running inside a framework whose allocator owns
+ * all device memory, or a real-time generation loop whose memory budget is fixed up front and
+ * that cannot risk an allocation failing or stalling mid-stream.
+ * K: device memory [n_frames][tokens_per_frame][head_dim] bf16 (one head's frames, oldest
+ * first, 16-byte aligned).  scores: device memory [n_frames - 1][n_segments] fp32; on
+ * completion scores[t][j] = s_t^(j), the cosine of segment j of frames t and t+1 (Eq. 3) under
+ * the same score contract as fk_compress, bit-identical to fk_get_scores for the same frames.
+ * Requires every token's contract squared key norm <= 2^23 (else the scores are unspecified).
+ * Limits: head_dim 64 or 128, 2 <= n_frames <= 256, 1 <= n_segments <= 32, n_frames *
+ * n_segments <= 4096, tokens_per_frame a multiple of n_segments; larger sizes return
+ * FK_ERR_CONFIG, host pointers FK_ERR_ARG.  The scratch is one fixed 65,728-byte array per
+ * device that loads the library (held until the process exits), shared by every call: calls
+ * whose work overlaps on the GPU (e.g. on two streams) race and must be ordered by the caller.
+ * The first call on a device resolves that array's address and must come before any stream
+ * capture.  Asynchronous on `stream`; uses the current device. */
+FK_API fk_status fk_segment_scores_noalloc(const void* K, int n_frames, int tokens_per_frame,
+                                           int head_dim, int n_segments, float* scores,
+                                           void* stream);
+
 /* Static text for a status code. */
 FK_API const char* fk_status_str(fk_status s);
 

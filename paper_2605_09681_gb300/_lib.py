@@ -22,6 +22,7 @@ EXPORTS = [
     "fk_set_current", "fk_compress", "fk_attend", "fk_cache_bytes", "fk_reserved_bytes",
     "fk_key_count", "fk_get_kept", "fk_get_scores", "fk_sync_status", "fk_profile_enable",
     "fk_profile_read", "fk_profile_reset", "fk_launch_count", "fk_status_str", "fk_abi_version",
+    "fk_segment_scores_noalloc",
 ]
 
 
@@ -80,6 +81,7 @@ def load(path: str | None = None) -> ctypes.CDLL:
         "fk_launch_count": (ctypes.c_int64, [vp]),
         "fk_status_str": (cp, [i32]),
         "fk_abi_version": (i32, []),
+        "fk_segment_scores_noalloc": (st, [vp, i32, i32, i32, i32, vp, vp]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)

@@ -12,6 +12,8 @@
 // finishes s = D / sqrt(N_t N_{t+1}) in IEEE double, stores the fp32 scores per frame slot,
 // ranks the scoreable candidates by (score, segment id) and stream-compacts the kept
 // segment ids with warp ballots and prefix sums.
+#include <mutex>
+
 #include "fk_internal.h"
 
 namespace fk {
@@ -338,4 +340,130 @@ void launch_score(const ScoreArgs& a, cudaStream_t s) {
   else score_kernel<64><<<grid, kScoreThreads, smem, s>>>(a);
 }
 
+// ---------------------------------------------------------------------------------------
+// Allocation-free scoring (fk_segment_scores_noalloc in fk.h).  The scoring kernel's scratch
+// (int64 sums, CTA and work counters, its one-item tables) lives in a file-scope device array
+// of fixed size instead of memory from cudaMalloc, so the call allocates nothing.  The array
+// exists once per device that loads the library; every call uses it.
+namespace {
+
+constexpr int kNoAllocMaxFrames = 256;
+constexpr int kNoAllocMaxSegments = 32;
+constexpr int kNoAllocMaxCells = 4096;                 // n_frames * n_segments
+constexpr size_t kNoAllocSumsBytes = (size_t)kNoAllocMaxCells * 2 * sizeof(unsigned long long);
+constexpr size_t kNoAllocCtrOff = kNoAllocSumsBytes;   // target counter, work[2], status
+constexpr size_t kNoAllocItemOff = kNoAllocCtrOff + 64;
+constexpr size_t kNoAllocTargetOff = kNoAllocItemOff + 64;
+constexpr size_t kNoAllocBytes = kNoAllocTargetOff + 64;   // 65,728 bytes
+static_assert(kNoAllocBytes == 65728, "documented size");
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocBytes];
+
+struct NoAllocDevice {
+  bool ready = false;
+  unsigned char* scratch = nullptr;   // device address of g_noalloc_scratch on this device
+  int ctas64 = 0, ctas128 = 0;        // persistent grid sizes
+};
+constexpr int kNoAllocMaxDevices = 64;
+NoAllocDevice g_noalloc[kNoAllocMaxDevices];
+std::mutex g_noalloc_mu;
+
+bool device_pointer(const void* p) {
+  cudaPointerAttributes at{};
+  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged;
+}
+
+}  // namespace
 }  // namespace fk
+
+extern "C" fk_status fk_segment_scores_noalloc(const void* K, int n_frames, int tokens_per_frame,
+                                                int head_dim, int n_segments, float* scores,
+                                                void* stream) {
+  using namespace fk;
+  if (!K || !scores) return FK_ERR_ARG;
+  if ((reinterpret_cast<uintptr_t>(K) & 15u) || (reinterpret_cast<uintptr_t>(scores) & 3u))
+    return FK_ERR_ARG;
+  if (head_dim != 64 && head_dim != 128) return FK_ERR_CONFIG;
+  if (n_segments < 1 || n_segments > kNoAllocMaxSegments) return FK_ERR_CONFIG;
+  if (tokens_per_frame < 1 || tokens_per_frame % n_segments) return FK_ERR_CONFIG;
+  if ((int64_t)tokens_per_frame * head_dim > (1 << 28)) return FK_ERR_CONFIG;
+  if (n_frames < 2 || n_frames > kNoAllocMaxFrames || n_frames * n_segments > kNoAllocMaxCells)
+    return FK_ERR_CONFIG;
+  if (!device_pointer(K) || !device_pointer(scores)) return FK_ERR_ARG;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kNoAllocMaxDevices) {
+    cudaGetLastError();
+    return FK_ERR_CUDA;
+  }
+  NoAllocDevice& nd = g_noalloc[dev];
+  {
+    std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    if (!nd.ready) {   // first call on this device: resolve the array's address, size the grid
+      void* p = nullptr;
+      if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) {
+        cudaGetLastError();
+        return FK_ERR_CUDA;
+      }
+      if (score_prepare(64, kNoAllocMaxFrames, kNoAllocMaxSegments, &nd.ctas64) != cudaSuccess ||
+          score_prepare(128, kNoAllocMaxFrames, kNoAllocMaxSegments, &nd.ctas128) != cudaSuccess) {
+        cudaGetLastError();
+        return FK_ERR_CUDA;
+      }
+      nd.scratch = static_cast<unsigned char*>(p);
+      nd.ready = true;
+    }
+  }
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  unsigned char* sc = nd.scratch;
+  // the sums and counters must start at zero; the previous call leaves them cleared, but
+  // clear them here anyway
+  const size_t sums_bytes = (size_t)n_frames * n_segments * 2 * sizeof(unsigned long long);
+  if (cudaMemsetAsync(sc, 0, sums_bytes, s) != cudaSuccess ||
+      cudaMemsetAsync(sc + kNoAllocCtrOff, 0, 64, s) != cudaSuccess) {
+    cudaGetLastError();
+    return FK_ERR_CUDA;
+  }
+  const ScoreItem item{static_cast<const bf16*>(K), 0, 0};
+  const SelectTarget target{0, 0, 1};
+  if (cudaMemcpyAsync(sc + kNoAllocItemOff, &item, sizeof(item), cudaMemcpyHostToDevice, s) != cudaSuccess ||
+      cudaMemcpyAsync(sc + kNoAllocTargetOff, &target, sizeof(target), cudaMemcpyHostToDevice, s) !=
+          cudaSuccess) {
+    cudaGetLastError();
+    return FK_ERR_CUDA;
+  }
+  ScoreArgs a{};
+  a.items = reinterpret_cast<const ScoreItem*>(sc + kNoAllocItemOff);
+  a.targets = reinterpret_cast<const SelectTarget*>(sc + kNoAllocTargetOff);
+  a.n_items = 1;
+  a.F = tokens_per_frame;
+  a.D = head_dim;
+  a.n_seg = n_segments;
+  a.seg_len = tokens_per_frame / n_segments;
+  a.chunks = (a.seg_len + kScoreTokensPerCta - 1) / kScoreTokensPerCta;
+  a.S = 0;                         // frames 0..n_frames-1 in slots 0..n_frames-1
+  a.cap_nonsink = n_frames;
+  a.ring_slots = n_frames;         // scores[t][j] for t = 0..n_frames-2
+  a.max_run = n_frames;
+  a.max_active_run = n_frames;
+  a.n_sub_max = (n_frames - 2) / kScorePairsPerCta + 1;
+  a.max_ctas = head_dim == 128 ? nd.ctas128 : nd.ctas64;
+  a.scope = FK_SCOPE_PER_FRAME;
+  a.k_frame = 0;
+  a.kmax = 1;
+  a.sums = reinterpret_cast<unsigned long long*>(sc);
+  a.counters = reinterpret_cast<int*>(sc + kNoAllocCtrOff);
+  a.work = reinterpret_cast<int*>(sc + kNoAllocCtrOff) + 1;
+  a.status = reinterpret_cast<int*>(sc + kNoAllocCtrOff) + 3;
+  a.scores = scores;
+  a.kept = reinterpret_cast<int*>(sc + kNoAllocTargetOff + 32);   // unused: no selection
+  a.run[0] = {0, n_frames};
+  a.t_lo[0] = 0;
+  a.n_scoreable[0] = 0;
+  a.n_keep[0] = 0;
+  launch_score(a, s);
+  return cudaGetLastError() == cudaSuccess ? FK_OK : FK_ERR_CUDA;
+}
