@@ -336,7 +336,7 @@ NCU_TRAFFIC = {
     "480p_layer": {
         "attend": ("fk_attn.cu", "a7947bb70908", 121476352),
         "compact": ("fk_copy.cu", "cba7e7019a47", 75307264),
-        "score": ("fk_score.cu", "1cfc2cc99fc2", 43181312),
+        "score": ("fk_score.cu", "630b903cffb0", 43159552),
     },
 }
 

@@ -12,7 +12,7 @@
 //                (dynamic heads; every head of layer 0 under layer-0 pooled scoring);
 //                frame f lives in slot f (f < S) or S + (f - S) mod cap_nonsink.
 //   scores       fp32 [target][ring_slots][n]; kept lists int32 [target][kmax];
-//                int64 scoring sums and CTA counters (scratch); status word;
+//                int64 scoring sums (scratch); status word;
 //                host-input staging.
 #include <algorithm>
 #include <cmath>
@@ -94,7 +94,6 @@ struct fk_handle {
   float* scores = nullptr;
   int* kept = nullptr;
   unsigned long long* sums = nullptr;
-  int* counters = nullptr;
   int* status = nullptr;
   bf16* stage_q = nullptr;
   bf16* stage_o = nullptr;
@@ -105,6 +104,7 @@ struct fk_handle {
   SelectTarget* d_targets = nullptr;
   CompactItem* d_compact_items = nullptr;
   std::vector<ScoreItem> score_items;
+  std::vector<std::pair<int, int>> layer_items;   // [L]: first score item, item count
   std::vector<SelectTarget> targets;
   std::vector<int> target_layer;
   std::vector<CompactItem> compact_items;
@@ -498,6 +498,12 @@ fk_status fk_create(const fk_config* cfg, fk_handle** out) {
         h->score_items.push_back({nullptr, l, hb.target});
       }
   }
+  h->layer_items.assign(h->L, {0, 0});   // score items are grouped by ascending layer
+  for (size_t y = 0; y < h->score_items.size(); ++y) {
+    auto& li = h->layer_items[h->score_items[y].layer];
+    if (li.second == 0) li.first = (int)y;
+    ++li.second;
+  }
 
   // allocations
   void* p = nullptr;
@@ -533,8 +539,6 @@ fk_status fk_create(const fk_config* cfg, fk_handle** out) {
   if ((st = dev_alloc(h, nt * h->max_run * h->n * 2 * sizeof(unsigned long long), &p)) != FK_OK)
     return fail(st);
   h->sums = static_cast<unsigned long long*>(p);
-  if ((st = dev_alloc(h, (nt + 2) * sizeof(int), &p)) != FK_OK) return fail(st);
-  h->counters = static_cast<int*>(p);     // [nt] per-target CTA counters, then the work counters
   if ((st = dev_alloc(h, 256, &p)) != FK_OK) return fail(st);
   h->status = static_cast<int*>(p);
   const size_t chunk_bytes = (size_t)h->CF * h->H * h->D * 2;
@@ -685,7 +689,6 @@ fk_status fk_compress(fk_handle* h, void* stream) {
       const int last_t = r.t_lo + r.n_scoreable - 1;
       if (r.n_scoreable > 0 && t_first <= last_t) {
         sa.run[l] = {t_first, last_t + 2 - t_first};
-        sa.max_active_run = std::max(sa.max_active_run, sa.run[l].n_run);
         any_run = true;
       }
       ls.scored_upto = r.anchor >= 0 ? r.anchor : ls.scored_upto;
@@ -719,14 +722,25 @@ fk_status fk_compress(fk_handle* h, void* stream) {
     sa.k_frame = h->k_frame;
     sa.kmax = h->kmax;
     sa.sums = h->sums;
-    sa.counters = h->counters;
-    sa.work = h->counters + (h->targets.empty() ? 1 : h->targets.size());
     sa.max_ctas = h->score_ctas;
-    sa.n_sub_max = sa.max_active_run > 1 ? (sa.max_active_run - 2) / kScorePairsPerCta + 1 : 1;
+    // active layers in ascending order with the start of their frame-chunks in the
+    // flattened (layer, item, segment, chunk, frame) range; items are grouped by layer
+    long long units = 0;
+    for (int l = 0; l < h->L; ++l) {
+      if (sa.run[l].n_run == 0 || h->layer_items[l].second == 0) continue;
+      sa.act_layer[sa.n_active] = l;
+      sa.act_first_item[sa.n_active] = h->layer_items[l].first;
+      sa.act_start[sa.n_active] = units;
+      units += (long long)h->layer_items[l].second * h->n * h->chunks * sa.run[l].n_run;
+      ++sa.n_active;
+    }
+    sa.total_units = units;
     sa.scores = h->scores;
     sa.kept = h->kept;
     sa.status = h->status;
     if ((st = launch(h, s, FK_KERNEL_SCORE, [&] { launch_score(sa, s); })) != FK_OK) return st;
+    const int nt = (int)h->targets.size();
+    if ((st = launch(h, s, FK_KERNEL_SELECT, [&] { launch_select(sa, nt, s); })) != FK_OK) return st;
   }
   if (any_compact && ca.max_units > 0) {
     ca.items = h->d_compact_items;

@@ -21,9 +21,9 @@ constexpr int kAttnBM = 128;          // query rows per attention CTA
 constexpr int kAttnBN = 128;          // keys per attention tile
 constexpr int kViewAlignRows = 128;   // packed views are padded to whole key tiles
 // scoring CTA: 4 warps; a token is owned by 4 lanes, so a CTA covers 32 tokens of a segment
+// (one frame-chunk)
 constexpr int kScoreThreads = 128;
 constexpr int kScoreTokensPerCta = (kScoreThreads / 32) * 8;
-constexpr int kScorePairsPerCta = 9;   // frame pairs per scoring CTA (sub-run of a run)
 
 // device status word bits (set by kernels, read by fk_sync_status)
 constexpr int kStatusRange = 1;
@@ -79,8 +79,8 @@ struct LayerRun {               // per layer: frames t_first..t_first+n_run-1 ar
   int n_run;                    // 0 = nothing to score in this layer
 };
 
-// Scoring of new frame pairs, then (in the last CTA of each target) the finish of the
-// scores and BottomK selection of that target.
+// Scoring of new frame pairs (score kernel), then the finish of the scores and BottomK
+// selection of every target with a run (select kernel, one CTA per target).
 struct ScoreArgs {
   const ScoreItem* items;       // device table
   const SelectTarget* targets;  // device table
@@ -88,15 +88,16 @@ struct ScoreArgs {
   int F, D, n_seg, seg_len, chunks;
   int S, cap_nonsink, ring_slots;
   int max_run;                  // frames one target's sums can hold
-  int max_active_run;           // longest run of this launch
-  int n_sub_max;                // sub-runs of the longest run
   int max_ctas;                 // persistent grid size
-  int* work;                    // [2]: next work unit, CTAs finished (zero between launches)
+  long long total_units;        // frame-chunks of this launch (item, segment, chunk, frame)
+  int n_active;                 // layers with a run, ascending
+  int act_layer[kMaxLayers];
+  int act_first_item[kMaxLayers];   // first score item of the layer
+  long long act_start[kMaxLayers];  // first frame-chunk of the layer in the flattened range
   int scope;                    // FK_SCOPE_*
   int k_frame;                  // kept per frame (per-frame scope)
   int kmax;                     // capacity of one kept list
   unsigned long long* sums;     // scratch [target][max_run][n_seg][2] : {N(t), D(t-1,t)}, zero between launches
-  int* counters;                // [target], zero between launches
   float* scores;                // [target][ring_slots][n_seg]
   int* kept;                    // [target][kmax]
   int* status;
@@ -106,12 +107,12 @@ struct ScoreArgs {
   int n_keep[kMaxLayers];       // kept segments of the layer's targets
 };
 void launch_score(const ScoreArgs& a, cudaStream_t s);
-// dynamic shared memory limit and the persistent grid size (CTAs resident at once)
+void launch_select(const ScoreArgs& a, int n_targets, cudaStream_t s);
+// dynamic shared memory limits and the persistent grid size (CTAs resident at once)
 cudaError_t score_prepare(int head_dim, int max_run, int n_seg, int* max_ctas);
-// shared memory of a scoring CTA: int32 accumulators (4 per frame) or the window's scores
-constexpr int score_smem_ints(int max_run, int n_seg) {
-  return 4 * max_run > max_run * n_seg ? 4 * max_run : max_run * n_seg;
-}
+// frame-chunks in flight per scoring CTA (one bulk copy each)
+constexpr int kScoreStages = 6;
+constexpr int kSelectThreads = 256;
 
 struct CompactItem {            // one dynamic (layer, head)
   const bf16* pagesK;

@@ -1,16 +1,19 @@
 // Segment-wise similarity scoring and BottomK selection (Sec. 4.3, Eq. 3) in one launch.
 //
-// Each CTA owns a few tokens of one segment of one scored (layer, head) and streams that
-// token range through the run of consecutive history frames, 16 bytes per lane, with a
-// four-frame register prefetch ring; every key byte is read once.  Per token it forms the
-// score-contract quantities (fp32 channel dot in a fixed fma/butterfly order, scaled by 2^24
-// and truncated to int64, carried as two exact int32 halves): the squared norm n_p(t) and
-// the dot d_p(t-1, t).  Warp sums go into shared-memory int32 accumulators (at most 32
-// tokens per CTA, so no overflow) and each CTA adds them as int64 into the target's global
-// int64 sums (exact integer adds, so the order is free).  The last CTA of a selection
-// target (counted with a global atomic)
-// finishes s = D / sqrt(N_t N_{t+1}) in IEEE double, stores the fp32 scores per frame slot,
-// ranks the scoreable candidates by (score, segment id) and stream-compacts the kept
+// Work unit: one frame-chunk, i.e. 32 tokens of one segment of one scored (layer, head) in
+// one frame of the run.  The units of all scored heads, ordered (layer, item, segment,
+// token chunk, frame), are split into equal contiguous ranges, one per CTA of a persistent
+// grid, so every CTA streams the same number of key bytes (no partial last wave).  A range
+// walks consecutive frames of a token chunk through a cp.async shared-memory ring, loading
+// one extra frame at its start as the partner of its first pair; every other key byte is
+// read once.  Per token it forms the score-contract quantities (fp32 channel dot in a fixed
+// fma/butterfly order, scaled by 2^24 and truncated to int64, carried as two exact int32
+// halves): the squared norm n_p(t) and the dot d_p(t-1, t).  Warp sums go into shared-memory
+// int32 accumulators (at most 32 tokens per run, so no overflow) and each run adds them as
+// int64 into the target's global int64 sums (exact integer adds, so the order is free).  The
+// CTA whose run completes a selection target's last frame-chunks (counted with a global
+// atomic) finishes s = D / sqrt(N_t N_{t+1}) in IEEE double, stores the fp32 scores per frame
+// slot, ranks the scoreable candidates by (score, segment id) and stream-compacts the kept
 // segment ids with warp ballots and prefix sums.
 #include <mutex>
 
@@ -23,6 +26,26 @@ __device__ __forceinline__ uint4 ld_keys(const void* p) {
   uint4 v;
   asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
                : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "l"(p));
+  return v;
+}
+
+__device__ __forceinline__ uint32_t su32_shared(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void cp_async16(uint32_t smem, const void* gmem) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" :: "r"(smem), "l"(gmem) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" :: "n"(N) : "memory");
+}
+__device__ __forceinline__ uint4 lds128(uint32_t smem) {
+  uint4 v;
+  asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "r"(smem) : "memory");
   return v;
 }
 
@@ -55,46 +78,94 @@ __device__ __forceinline__ float finish_score(long long dsum, long long n1, long
   return __double2float_rn(__ddiv_rn(__ll2double_rn(dsum), den));
 }
 
-// Finish the scored pairs of target `tgi` and select its kept segments (one CTA).
-__device__ void finish_and_select(const ScoreArgs& a, int tgi, int* stage) {
-  __shared__ int warp_tot[32];
+constexpr uint64_t kWaitLimitNs = 2000000000ull;   // 2 s per wait
+
+__device__ __forceinline__ uint64_t now_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" :: "r"(bar), "r"(count));
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" :: "r"(bar), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ bool mbar_test(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok) : "r"(bar), "r"(parity) : "memory");
+  return ok != 0;
+}
+// bounded wait for the phase of parity `parity`; false when the limit expired
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
+  if (mbar_test(bar, parity)) return true;
+  const uint64_t t0 = now_ns();
+  while (!mbar_test(bar, parity))
+    if (now_ns() - t0 > kWaitLimitNs) return false;
+  return true;
+}
+// one contiguous global -> shared copy on the TMA engine, completing on `bar`
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+               :: "r"(dst), "l"(src), "r"(bytes), "r"(bar) : "memory");
+}
+// programmatic dependent launch: let the next kernel of the stream start its prologue /
+// wait until the previous kernel of the stream has completed and its writes are visible
+// (both are no-ops for a launch without the programmatic attribute)
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+// Selection kernel: one CTA per selection target.  Finishes the pairs (t, t+1) scored by
+// this launch from the target's int64 sums, clears the sums for the next launch, then
+// BottomK over the scoreable frames compacted in ascending segment-id order; the window's
+// scores are staged in shared memory in candidate order (t - t_lo)*n + j.
+__global__ void __launch_bounds__(kSelectThreads) select_kernel(const ScoreArgs a) {
+  extern __shared__ float ssc[];
+  __shared__ int warp_tot[kSelectThreads / 32];
   __shared__ int base_off;
+  const int tgi = blockIdx.x;
   const SelectTarget tg = a.targets[tgi];
   const int l = tg.layer;
   const LayerRun run = a.run[l];
+  pdl_trigger();
+  if (run.n_run < 2) return;
+  pdl_wait();
   const int n = a.n_seg;
-  float* sc = a.scores + (int64_t)tgi * a.ring_slots * n;
-
-  // 1. finish the pairs (t, t+1) scored by this launch from the target's int64 sums
-  //    (read past L1: other CTAs added them), then clear the sums for the next launch
-  unsigned long long* sums = a.sums + (int64_t)tgi * a.max_run * n * 2;
-  if (run.n_run >= 2) {
-    const int pairs = (run.n_run - 1) * n;
-    for (int idx = threadIdx.x; idx < pairs; idx += blockDim.x) {
-      const int k = idx / n, j = idx - k * n;
-      const unsigned long long N1 = __ldcg(sums + ((int64_t)k * n + j) * 2);
-      const unsigned long long N2 = __ldcg(sums + ((int64_t)(k + 1) * n + j) * 2);
-      const unsigned long long Dd = __ldcg(sums + ((int64_t)(k + 1) * n + j) * 2 + 1);
-      const int slot = ring_slot(run.t_first + k, a.S, a.cap_nonsink);
-      sc[slot * n + j] = finish_score((long long)Dd, (long long)N1, (long long)N2);
-    }
-  }
-  __syncthreads();
-  for (int i = threadIdx.x; i < run.n_run * n * 2; i += blockDim.x) sums[i] = 0ull;
-
-  // 2. BottomK over the scoreable frames, compacted in ascending segment-id order; the
-  //    window's scores are staged in shared memory in candidate order (t - t_lo)*n + j
   const int nT = a.n_scoreable[l];
   const int M = nT * n;
-  const int K = a.n_keep[l];
   const int t_lo = a.t_lo[l];
-  int* out = a.kept + (int64_t)tgi * a.kmax;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  float* ssc = reinterpret_cast<float*>(stage);
+  float* sc = a.scores + (int64_t)tgi * a.ring_slots * n;
+  unsigned long long* sums = a.sums + (int64_t)tgi * a.max_run * n * 2;
+  // 1. finish: s = D / sqrt(N_t N_{t+1}) in IEEE double, stored per frame slot and staged
+  //    for the ranking when the frame is in the window
+  const int pairs = (run.n_run - 1) * n;
+  for (int idx = threadIdx.x; idx < pairs; idx += blockDim.x) {
+    const int k = idx / n, j = idx - k * n;
+    const unsigned long long N1 = sums[((int64_t)k * n + j) * 2];
+    const unsigned long long N2 = sums[((int64_t)(k + 1) * n + j) * 2];
+    const unsigned long long Dd = sums[((int64_t)(k + 1) * n + j) * 2 + 1];
+    const int t = run.t_first + k;
+    const float v = finish_score((long long)Dd, (long long)N1, (long long)N2);
+    sc[ring_slot(t, a.S, a.cap_nonsink) * n + j] = v;
+    if (t >= t_lo && t < t_lo + nT) ssc[(t - t_lo) * n + j] = v;
+  }
+  // window frames scored by an earlier launch (incremental scoring)
   for (int idx = threadIdx.x; idx < M; idx += blockDim.x) {
     const int t = t_lo + idx / n, jj = idx - (idx / n) * n;
-    ssc[idx] = __ldcg(sc + ring_slot(t, a.S, a.cap_nonsink) * n + jj);
+    if (t < run.t_first) ssc[idx] = sc[ring_slot(t, a.S, a.cap_nonsink) * n + jj];
   }
+  __syncthreads();   // every sum has been read
+  for (int i = threadIdx.x; i < run.n_run * n * 2; i += blockDim.x) sums[i] = 0ull;
+
+  // 2. BottomK: rank by (score, segment id) within the frame (per-frame scope) or over the
+  //    whole window (pooled scope), then stream-compact with warp ballots
+  const int K = a.n_keep[l];
+  int* out = a.kept + (int64_t)tgi * a.kmax;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) base_off = 0;
   __syncthreads();
   for (int b0 = 0; b0 < M; b0 += blockDim.x) {
@@ -105,18 +176,18 @@ __device__ void finish_and_select(const ScoreArgs& a, int tgi, int* stage) {
       t = t_lo + idx / n;
       j = idx - (idx / n) * n;
       const float* row = ssc + (idx - j);
-      const float s = row[j];
+      const float sv = row[j];
       int rank = 0;
       if (a.scope == FK_SCOPE_PER_FRAME) {
         for (int jj = 0; jj < n; ++jj) {
           const float o = row[jj];
-          rank += (o < s) || (o == s && jj < j);
+          rank += (o < sv) || (o == sv && jj < j);
         }
         keep = rank < a.k_frame;
       } else {
         for (int qq = 0; qq < M; ++qq) {
           const float o = ssc[qq];
-          rank += (o < s) || (o == s && qq < idx);
+          rank += (o < sv) || (o == sv && qq < idx);
         }
         keep = rank < K;
       }
@@ -138,189 +209,241 @@ __device__ void finish_and_select(const ScoreArgs& a, int tgi, int* stage) {
   }
 }
 
-// D = head_dim.  Four lanes own one token: lane q of the token holds channel groups
-// 4i + q, i < GPL (GPL = D/32 groups of 8 channels, one 16-byte granule each), so each
-// load instruction reads 64 contiguous bytes per token; a warp covers 8 tokens and a
-// 128-thread CTA 32 tokens of one segment.
-// One work unit: item y, segment j, token chunk c, sub-run z (block-uniform arguments).
+// Shared-memory layout of the scoring kernel (offsets in bytes from the dynamic base).
 template <int D>
-__device__ __forceinline__ void score_unit(const ScoreArgs& a, int y, int j, int c, int z,
-                                           int* acc32, int& is_last) {
-  constexpr int LPT = 4;                       // lanes per token
-  constexpr int GPL = D / 32;                  // granules (channel groups) per lane
-  constexpr int TPW = 32 / LPT;                // tokens per warp
-  constexpr int TB = (kScoreThreads / 32) * TPW;
-  constexpr int PF = 4;                        // ring of packed frames per lane
+struct ScoreSmem {
+  static constexpr int kStageBytes = kScoreTokensPerCta * D * 2;   // one frame-chunk
+  static constexpr int kBarOff = kScoreStages * kStageBytes;
+  static constexpr int kAccOff = kBarOff + kScoreStages * 8;
+};
+
+// D = head_dim.  Four lanes own one token (a warp 8 tokens, the CTA the 32 tokens of one
+// frame-chunk).  Lane q of a token holds channel groups g = 4*(i ^ o) + q in register slot
+// i < GPL = D/32 (groups of 8 channels, 16 bytes each), o = the token's parity: with the
+// odd tokens' slots swapped pairwise, the 8 lanes of each quarter-warp read 8 distinct
+// 16-byte bank groups from the unswizzled staged rows.  The slot permutation i -> i ^ o is
+// an automorphism of the butterfly below (it maps the pair {g, g ^ s} of every stage onto
+// itself), and fp32 addition is commutative, so every slot ends with the contract value.
+//
+// One run: item y, segment j, token chunk c, frames k_first..k_last of the item's run, all
+// owned by this CTA (it adds N(k) for each and D(k) = sum d_p(k-1, k) for k >= 1; the frame
+// before k_first is loaded only as the partner of k_first).  Block-uniform arguments.
+// Returns false when a wait expired (the status word records it).
+template <int D>
+__device__ __forceinline__ bool score_run(const ScoreArgs& a, int y, int j, int c, int k_first,
+                                          int k_last, uint8_t* smem, uint32_t& seq) {
+  using L = ScoreSmem<D>;
+  constexpr int GPL = D / 32;
   const ScoreItem it = a.items[y];
   const LayerRun run = a.run[it.layer];
-  // sub-run blockIdx.z: frames k_lo .. k_hi of the run (pairs (k-1, k) for k_lo < k <= k_hi);
-  // a sub-run's first frame is the previous sub-run's last one, whose norm that one counts
-  const int n_sub = run.n_run > 1 ? (run.n_run - 2) / kScorePairsPerCta + 1 : 1;
-  if (run.n_run == 0 || z >= n_sub) return;
-  const int k_lo = z * kScorePairsPerCta;
-  const int k_hi = min(k_lo + kScorePairsPerCta, run.n_run - 1);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int q = lane & 3;
+  const int tl = warp * 8 + (lane >> 2);        // token within the chunk
+  const int odd = tl & 1;
   const int seg_lo = j * a.seg_len;
-  const int tok0 = seg_lo + c * TB;
-  const int tok_end = min(tok0 + TB, seg_lo + a.seg_len);
-  const int q = lane % LPT;                    // lane within the token
-  const int tok = tok0 + warp * TPW + lane / LPT;
-  const bool ok = tok < tok_end;
+  const int tok0 = seg_lo + c * kScoreTokensPerCta;
+  const int ntok = min(kScoreTokensPerCta, seg_lo + a.seg_len - tok0);
+  const bool ok = tl < ntok;
+  const int n_own = k_last - k_first + 1;
+  const int k_load0 = k_first > 0 ? k_first - 1 : 0;
+  const int n_load = k_last - k_load0 + 1;
+  int* acc32 = reinterpret_cast<int*>(smem + L::kAccOff);   // [frame][4]: N hi, N lo, D hi, D lo
+  const uint32_t sbase = su32_shared(smem);
 
-  for (int i = threadIdx.x; i < 4 * run.n_run; i += blockDim.x) acc32[i] = 0;
-  __syncthreads();
-
-  const bf16* base = it.pagesK + (int64_t)tok * D + q * 8;
-  const int64_t frame_elems = (int64_t)a.F * D;
-  // ring slot of the next frame to load; scored frames are never sinks, so the slot
-  // advances by one and wraps from the last slot to the first non-sink slot
+  for (int i = threadIdx.x; i < 4 * n_own; i += blockDim.x) acc32[i] = 0;
+  // producer: thread 0 streams the frame-chunks (ntok consecutive rows of a page, one
+  // contiguous block) through the kScoreStages-stage ring; frame u of the run is sequence
+  // number seq + u of this CTA, in stage (seq + u) % NS, phase parity ((seq + u) / NS) & 1
+  const uint32_t bytes = (uint32_t)ntok * D * 2;
   const int slot_end = a.S + a.cap_nonsink;
-  int next_slot = ring_slot(run.t_first + k_lo, a.S, a.cap_nonsink);
-  auto load = [&](int k, uint4 (&dst)[GPL]) {
-#pragma unroll
-    for (int i = 0; i < GPL; ++i) dst[i] = make_uint4(0, 0, 0, 0);
-    if (k <= k_hi) {
-      if (ok) {
-        const bf16* p = base + (int64_t)next_slot * frame_elems;
-#pragma unroll
-        for (int i = 0; i < GPL; ++i) dst[i] = ld_keys(p + i * 32);
-      }
-      next_slot = next_slot + 1 == slot_end ? a.S : next_slot + 1;
-    }
+  int next_slot = ring_slot(run.t_first + k_load0, a.S, a.cap_nonsink);
+  const bf16* src0 = it.pagesK + (int64_t)tok0 * D;
+  const int64_t frame_elems = (int64_t)a.F * D;
+  auto issue = [&](int u) {
+    const uint32_t st = (seq + u) % kScoreStages;
+    const uint32_t bar = sbase + L::kBarOff + st * 8;
+    mbar_expect_tx(bar, bytes);
+    bulk_load(sbase + st * L::kStageBytes, src0 + (int64_t)next_slot * frame_elems, bytes, bar);
+    // scored frames are never sinks: the slot advances and wraps to the first non-sink slot
+    next_slot = next_slot + 1 == slot_end ? a.S : next_slot + 1;
   };
-  // ring of PF packed frames: frame k lives in buf[(k - k_lo) % PF]; the previous frame is
-  // the previous slot, and a slot is refilled (PF - 1 frames ahead) once it has served as
-  // "previous"
-  uint4 buf[PF][GPL];
+  if (threadIdx.x == 0)
+    for (int u = 0; u < min(kScoreStages, n_load); ++u) issue(u);
+
+  uint4 prv[GPL];
 #pragma unroll
-  for (int u = 0; u < PF - 1; ++u) load(k_lo + u, buf[u]);
+  for (int i = 0; i < GPL; ++i) prv[i] = make_uint4(0, 0, 0, 0);   // partner of frame 0: none
+  bool bad = false, timed_out = false;
+  for (int u = 0; u < n_load; ++u) {
+    const int k = k_load0 + u;
+    const uint32_t st = (seq + u) % kScoreStages;
+    if (!mbar_wait(sbase + L::kBarOff + st * 8, ((seq + u) / kScoreStages) & 1)) timed_out = true;
+    uint4 cur[GPL];
+    const uint32_t row = sbase + st * L::kStageBytes + tl * (D * 2) + q * 16;
 #pragma unroll
-  for (int i = 0; i < GPL; ++i) buf[PF - 1][i] = make_uint4(0, 0, 0, 0);   // "previous" of k_lo
-  bool bad = false;
-  for (int k0 = k_lo; k0 <= k_hi; k0 += PF) {
-#pragma unroll
-    for (int u = 0; u < PF; ++u) {
-      const int k = k0 + u;
-      if (k > k_hi) break;
-      const uint4 (&cur)[GPL] = buf[u];
-      const uint4 (&prv)[GPL] = buf[(u + PF - 1) % PF];
+    for (int i = 0; i < GPL; ++i) cur[i] = lds128(row + ((i ^ odd) * 64));
+    // every thread has its registers: the stage can be refilled
+    if (__syncthreads_or(timed_out)) {
+      if (threadIdx.x == 0) atomicOr(a.status, kStatusTimeout);
+      // drain: wait (bounded) for the copies still in flight before the CTA leaves
+      for (int v = u; v < min(u + kScoreStages, n_load); ++v)
+        mbar_wait(sbase + L::kBarOff + ((seq + v) % kScoreStages) * 8, ((seq + v) / kScoreStages) & 1);
+      return false;
+    }
+    if (threadIdx.x == 0 && u + kScoreStages < n_load) issue(u + kScoreStages);
+    if (k >= k_first) {
       // one fma chain per channel group (channel order), for n_p and d_p
-      float n[GPL], d[GPL];
+      float nn[GPL], dd[GPL];
 #pragma unroll
       for (int i = 0; i < GPL; ++i) {
-        n[i] = 0.0f;
-        d[i] = 0.0f;
-        fma_word(cur[i].x, prv[i].x, n[i], d[i]);
-        fma_word(cur[i].y, prv[i].y, n[i], d[i]);
-        fma_word(cur[i].z, prv[i].z, n[i], d[i]);
-        fma_word(cur[i].w, prv[i].w, n[i], d[i]);
+        nn[i] = 0.0f;
+        dd[i] = 0.0f;
+        fma_word(cur[i].x, prv[i].x, nn[i], dd[i]);
+        fma_word(cur[i].y, prv[i].y, nn[i], dd[i]);
+        fma_word(cur[i].z, prv[i].z, nn[i], dd[i]);
+        fma_word(cur[i].w, prv[i].w, nn[i], dd[i]);
       }
-      load(k + PF - 1, buf[(u + PF - 1) % PF]);   // the previous frame's slot is free now
-      // butterfly p[g] += p[g ^ s], s = D/16 .. 1 over groups g = 4i + q: strides s >= 4 pair
-      // i with i ^ (s/4) inside the lane, strides 2 and 1 pair lane q with q ^ s
+      // butterfly p[g] += p[g ^ s], s = D/16 .. 1: strides s >= 4 pair slot i with
+      // i ^ (s/4) inside the lane, strides 2 and 1 pair lane q with q ^ s
 #pragma unroll
       for (int sft = GPL / 2; sft >= 1; sft >>= 1) {
 #pragma unroll
         for (int i = 0; i < GPL; ++i) {
           if ((i & sft) == 0) {
-            const float nn = __fadd_rn(n[i], n[i ^ sft]);
-            const float dd = __fadd_rn(d[i], d[i ^ sft]);
-            n[i] = nn; n[i ^ sft] = nn;
-            d[i] = dd; d[i ^ sft] = dd;
+            const float n2 = __fadd_rn(nn[i], nn[i ^ sft]);
+            const float d2 = __fadd_rn(dd[i], dd[i ^ sft]);
+            nn[i] = n2; nn[i ^ sft] = n2;
+            dd[i] = d2; dd[i ^ sft] = d2;
           }
         }
       }
 #pragma unroll
       for (int sft = 2; sft >= 1; sft >>= 1) {
-        n[0] = __fadd_rn(n[0], __shfl_xor_sync(0xffffffffu, n[0], sft));
-        d[0] = __fadd_rn(d[0], __shfl_xor_sync(0xffffffffu, d[0], sft));
+        nn[0] = __fadd_rn(nn[0], __shfl_xor_sync(0xffffffffu, nn[0], sft));
+        dd[0] = __fadd_rn(dd[0], __shfl_xor_sync(0xffffffffu, dd[0], sft));
       }
-      const float np = n[0];
-      const float dp = d[0];                     // 0 for the first frame of the run
       // lane q = 0 of a token converts n_p, lane q = 1 converts d_p (then summed over the
       // warp's tokens); the other lanes contribute zero
-      // the norm of a sub-run's last frame belongs to the next sub-run (except at the end)
-      const bool count_n = k < k_hi || k_hi == run.n_run - 1;
       int hi = 0, lo = 0;
       if (ok && q < 2) {
-        const float v = q == 0 ? (count_n ? np : 0.0f) : (k > k_lo ? dp : 0.0f);
-        if (q == 0) bad |= !(np <= 8388608.0f);
+        const float v = q == 0 ? nn[0] : (k > 0 ? dd[0] : 0.0f);
+        if (q == 0) bad |= !(nn[0] <= 8388608.0f);
         fixed24_split(v, hi, lo);
       }
 #pragma unroll
-      for (int sft = LPT; sft < 32; sft <<= 1) {
+      for (int sft = 4; sft < 32; sft <<= 1) {
         hi += __shfl_xor_sync(0xffffffffu, hi, sft);
         lo += __shfl_xor_sync(0xffffffffu, lo, sft);
       }
-      if (lane < 2) {                            // lane 0: N(t) parts, lane 1: D(t-1, t) parts
-        atomicAdd(&acc32[4 * k + 2 * lane], hi);
-        atomicAdd(&acc32[4 * k + 2 * lane + 1], lo);
+      if (lane < 2) {                            // lane 0: N(k) parts, lane 1: D(k) parts
+        atomicAdd(&acc32[4 * (k - k_first) + 2 * lane], hi);
+        atomicAdd(&acc32[4 * (k - k_first) + 2 * lane + 1], lo);
       }
     }
+#pragma unroll
+    for (int i = 0; i < GPL; ++i) prv[i] = cur[i];
   }
+  seq += n_load;
   if (bad) atomicOr(a.status, kStatusRange);
   __syncthreads();
+  // exact int64 adds into the target's sums (fire-and-forget; the selection kernel reads
+  // them after this kernel has completed)
   unsigned long long* sums = a.sums + (int64_t)it.target * a.max_run * a.n_seg * 2;
-  for (int qq = 2 * k_lo + threadIdx.x; qq < 2 * (k_hi + 1); qq += blockDim.x) {
-    const int k = qq >> 1, which = qq & 1;
-    const long long v = (long long)acc32[4 * k + 2 * which] * 16777216ll + (long long)acc32[4 * k + 2 * which + 1];
-    atomicAdd(sums + ((int64_t)k * a.n_seg + j) * 2 + which, (unsigned long long)v);
+  for (int qq = threadIdx.x; qq < 2 * n_own; qq += blockDim.x) {
+    const int kk = qq >> 1, which = qq & 1;
+    const long long v =
+        (long long)acc32[4 * kk + 2 * which] * 16777216ll + (long long)acc32[4 * kk + 2 * which + 1];
+    atomicAdd(sums + ((int64_t)(k_first + kk) * a.n_seg + j) * 2 + which, (unsigned long long)v);
   }
-
-  // the last CTA of this item's selection target finishes it
-  __threadfence();
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    const SelectTarget tg = a.targets[it.target];
-    const int expected = a.n_seg * a.chunks * tg.n_items * n_sub;
-    is_last = atomicAdd(&a.counters[it.target], 1) == expected - 1;
-  }
-  __syncthreads();
-  if (!is_last) return;
-  __threadfence();
-  finish_and_select(a, it.target, acc32);
-  if (threadIdx.x == 0) a.counters[it.target] = 0;
-  __syncthreads();                               // acc32 is reused by the next unit
+  __syncthreads();                               // acc32 is reused by the next run
+  return true;
 }
 
-// Persistent grid (one wave): CTAs take work units from a global counter until none is left;
-// the last CTA to leave resets the counter for the next launch.
+// Persistent grid: the frame-chunks of all scored items (item, segment, token chunk, frame)
+// form one flattened range split into equal contiguous pieces, one per CTA; a piece walks
+// its runs in order.
 template <int D>
 __global__ void __launch_bounds__(kScoreThreads, 4) score_kernel(const ScoreArgs a) {
-  extern __shared__ int acc32[];               // [n_run][4] : {N hi, N lo, D hi, D lo}
-  __shared__ int s_unit, is_last;
-  const int per_sub = a.n_seg * a.chunks;
-  const int per_item = per_sub * a.n_sub_max;
-  const int total = a.n_items * per_item;
-  for (;;) {
-    if (threadIdx.x == 0) s_unit = atomicAdd(a.work, 1);
-    __syncthreads();
-    const int unit = s_unit;
-    __syncthreads();
-    if (unit >= total) break;
-    const int y = unit / per_item;
-    const int r = unit - y * per_item;
-    const int z = r / per_sub;
-    const int r2 = r - z * per_sub;
-    const int j = r2 / a.chunks;
-    score_unit<D>(a, y, j, r2 - j * a.chunks, z, acc32, is_last);
-  }
+  extern __shared__ __align__(128) uint8_t smem[];
+  using L = ScoreSmem<D>;
+  pdl_trigger();
   if (threadIdx.x == 0) {
-    __threadfence();
-    if (atomicAdd(a.work + 1, 1) == (int)gridDim.x - 1) {
-      a.work[0] = 0;
-      a.work[1] = 0;
-    }
+    for (int i = 0; i < kScoreStages; ++i) mbar_init(su32_shared(smem) + L::kBarOff + i * 8, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
+  __syncthreads();
+  pdl_wait();                                    // the keys were written by earlier kernels
+  const long long T = a.total_units;
+  long long g = T * blockIdx.x / gridDim.x;
+  const long long g_end = T * (blockIdx.x + 1) / gridDim.x;
+  const int per_item = a.n_seg * a.chunks;
+  uint32_t seq = 0;
+  while (g < g_end) {
+    int lo = 0, hi = a.n_active - 1;             // active layer holding unit g
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (a.act_start[mid] <= g) lo = mid;
+      else hi = mid - 1;
+    }
+    const LayerRun run = a.run[a.act_layer[lo]];
+    const long long idx = g - a.act_start[lo];
+    const long long chunk_id = idx / run.n_run;
+    const int k = (int)(idx - chunk_id * run.n_run);
+    const int item_local = (int)(chunk_id / per_item);
+    const int r = (int)(chunk_id - (long long)item_local * per_item);
+    const int j = r / a.chunks;
+    const long long left = g_end - g;
+    const int k_last = (int)(left < run.n_run - k ? k + left - 1 : run.n_run - 1);
+    if (!score_run<D>(a, a.act_first_item[lo] + item_local, j, r - j * a.chunks, k, k_last, smem, seq))
+      return;
+    g += k_last - k + 1;
+  }
+}
+
+template <int D>
+constexpr size_t score_smem_bytes_d(int max_run) {
+  return (size_t)ScoreSmem<D>::kAccOff + (size_t)4 * max_run * sizeof(int);
+}
+size_t score_smem_bytes(int head_dim, int max_run) {
+  return head_dim == 128 ? score_smem_bytes_d<128>(max_run) : score_smem_bytes_d<64>(max_run);
+}
+size_t select_smem_bytes(int max_run, int n_seg) { return (size_t)max_run * n_seg * sizeof(float); }
+
+// launch with the programmatic-dependent-launch attribute: the kernel's prologue may
+// overlap the previous kernel's tail; its pdl_wait() orders it after that kernel
+template <typename Kern>
+cudaError_t launch_pdl(Kern kern, unsigned grid, unsigned threads, size_t smem, cudaStream_t s,
+                       const ScoreArgs& a) {
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(threads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, a);
 }
 
 }  // namespace
 
 cudaError_t score_prepare(int head_dim, int max_run, int n_seg, int* max_ctas) {
-  const int smem = score_smem_ints(max_run, n_seg) * (int)sizeof(int);
+  const int smem = (int)score_smem_bytes(head_dim, max_run);
   const void* fn = head_dim == 128 ? (const void*)score_kernel<128> : (const void*)score_kernel<64>;
-  cudaError_t e = cudaSuccess;
-  if (smem > 48 * 1024) e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  // the limits are per function and shared by every handle: only ever raise them
+  cudaFuncAttributes fa{};
+  cudaError_t e = cudaFuncGetAttributes(&fa, fn);
+  if (e != cudaSuccess) return e;
+  if (smem > 48 * 1024 && smem > fa.maxDynamicSharedSizeBytes)
+    e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e != cudaSuccess) return e;
+  const int sel_smem = (int)select_smem_bytes(max_run, n_seg);
+  if ((e = cudaFuncGetAttributes(&fa, (const void*)select_kernel)) != cudaSuccess) return e;
+  if (sel_smem > 48 * 1024 && sel_smem > fa.maxDynamicSharedSizeBytes)
+    e = cudaFuncSetAttribute((const void*)select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             sel_smem);
   if (e != cudaSuccess) return e;
   int dev = 0, sms = 0, per_sm = 0;
   if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
@@ -333,16 +456,22 @@ cudaError_t score_prepare(int head_dim, int max_run, int n_seg, int* max_ctas) {
 
 void launch_score(const ScoreArgs& a, cudaStream_t s) {
   if (a.n_items == 0) return;
-  const int64_t units = (int64_t)a.n_items * a.n_seg * a.chunks * a.n_sub_max;
+  const long long units = a.total_units;
+  if (units <= 0) return;
   const unsigned grid = (unsigned)(units < a.max_ctas ? units : a.max_ctas);
-  const size_t smem = (size_t)score_smem_ints(a.max_run, a.n_seg) * sizeof(int);
-  if (a.D == 128) score_kernel<128><<<grid, kScoreThreads, smem, s>>>(a);
-  else score_kernel<64><<<grid, kScoreThreads, smem, s>>>(a);
+  const size_t smem = score_smem_bytes(a.D, a.max_run);
+  if (a.D == 128) launch_pdl(score_kernel<128>, grid, kScoreThreads, smem, s, a);
+  else launch_pdl(score_kernel<64>, grid, kScoreThreads, smem, s, a);
+}
+
+void launch_select(const ScoreArgs& a, int n_targets, cudaStream_t s) {
+  if (n_targets <= 0 || a.total_units <= 0) return;
+  launch_pdl(select_kernel, (unsigned)n_targets, kSelectThreads, select_smem_bytes(a.max_run, a.n_seg), s, a);
 }
 
 // ---------------------------------------------------------------------------------------
 // Allocation-free scoring (fk_segment_scores_noalloc in fk.h).  The scoring kernel's scratch
-// (int64 sums, CTA and work counters, its one-item tables) lives in a file-scope device array
+// (int64 sums, a status word, its one-item tables) lives in a file-scope device array
 // of fixed size instead of memory from cudaMalloc, so the call allocates nothing.  The array
 // exists once per device that loads the library; every call uses it.
 namespace {
@@ -351,7 +480,7 @@ constexpr int kNoAllocMaxFrames = 256;
 constexpr int kNoAllocMaxSegments = 32;
 constexpr int kNoAllocMaxCells = 4096;                 // n_frames * n_segments
 constexpr size_t kNoAllocSumsBytes = (size_t)kNoAllocMaxCells * 2 * sizeof(unsigned long long);
-constexpr size_t kNoAllocCtrOff = kNoAllocSumsBytes;   // target counter, work[2], status
+constexpr size_t kNoAllocCtrOff = kNoAllocSumsBytes;   // 64-byte word block; status at +12 bytes
 constexpr size_t kNoAllocItemOff = kNoAllocCtrOff + 64;
 constexpr size_t kNoAllocTargetOff = kNoAllocItemOff + 64;
 constexpr size_t kNoAllocBytes = kNoAllocTargetOff + 64;   // 65,728 bytes
@@ -419,8 +548,8 @@ extern "C" fk_status fk_segment_scores_noalloc(const void* K, int n_frames, int 
   }
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   unsigned char* sc = nd.scratch;
-  // the sums and counters must start at zero; the previous call leaves them cleared, but
-  // clear them here anyway
+  // the sums and the status word must start at zero; the previous call leaves the sums
+  // cleared, but clear them here anyway
   const size_t sums_bytes = (size_t)n_frames * n_segments * 2 * sizeof(unsigned long long);
   if (cudaMemsetAsync(sc, 0, sums_bytes, s) != cudaSuccess ||
       cudaMemsetAsync(sc + kNoAllocCtrOff, 0, 64, s) != cudaSuccess) {
@@ -448,15 +577,16 @@ extern "C" fk_status fk_segment_scores_noalloc(const void* K, int n_frames, int 
   a.cap_nonsink = n_frames;
   a.ring_slots = n_frames;         // scores[t][j] for t = 0..n_frames-2
   a.max_run = n_frames;
-  a.max_active_run = n_frames;
-  a.n_sub_max = (n_frames - 2) / kScorePairsPerCta + 1;
+  a.n_active = 1;
+  a.act_layer[0] = 0;
+  a.act_first_item[0] = 0;
+  a.act_start[0] = 0;
+  a.total_units = (long long)n_segments * a.chunks * n_frames;
   a.max_ctas = head_dim == 128 ? nd.ctas128 : nd.ctas64;
   a.scope = FK_SCOPE_PER_FRAME;
   a.k_frame = 0;
   a.kmax = 1;
   a.sums = reinterpret_cast<unsigned long long*>(sc);
-  a.counters = reinterpret_cast<int*>(sc + kNoAllocCtrOff);
-  a.work = reinterpret_cast<int*>(sc + kNoAllocCtrOff) + 1;
   a.status = reinterpret_cast<int*>(sc + kNoAllocCtrOff) + 3;
   a.scores = scores;
   a.kept = reinterpret_cast<int*>(sc + kNoAllocTargetOff + 32);   // unused: no selection
@@ -465,5 +595,6 @@ extern "C" fk_status fk_segment_scores_noalloc(const void* K, int n_frames, int 
   a.n_scoreable[0] = 0;
   a.n_keep[0] = 0;
   launch_score(a, s);
+  launch_select(a, 1, s);
   return cudaGetLastError() == cudaSuccess ? FK_OK : FK_ERR_CUDA;
 }
