@@ -323,10 +323,75 @@ def run_fk(args, rank, world, local_rank):
         "attn_gflop_per_step": round(alg["attn_flops"] / 1e9, 2),
         "clocks": clk.summary(),
     }
+    cache.close()
+    if not args.no_stack:
+        out["stack_480p"] = run_stack(local_rank)
     if rank == 0 and not args.no_cpu_baseline:
         out["cpu_baseline"] = cpu_baseline(w, budget_s=args.cpu_seconds)
-    cache.close()
     return out
+
+
+def run_stack(local_rank):
+    """The 480P 30-layer stack measured directly: 7 chunks of 3 frames, each appended to all
+    30 layers, compressed, and attended at 4 denoising steps per layer (set_current between
+    steps); frames/s = 21 frames / wall time of every library call, inputs resident on the
+    device.  The denoising steps reuse the chunk's clean K/V (the work does not depend on
+    the values), and the 4 query sets are reused across chunks and layers."""
+    import time
+
+    import numpy as np
+    import torch
+
+    import workloads as W
+    from paper_2605_09681_gb300 import ForcingKVCache
+
+    w = W.P480_STACK
+    dev = torch.device("cuda", local_rank)
+    hm = W.head_map(w)
+    fs = W.FrameStream(w, 0)
+    to_t = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16).to(dev)
+    kv = [tuple(to_t(x) for x in fs.frames(w.frames_per_chunk)) for _ in range(w.n_chunks)]
+    qs = [to_t(W.queries(w, 0, 0, d)) for d in range(w.denoise_steps)]
+    out_t = torch.empty_like(qs[0])
+
+    def run(cache):
+        calls = 0
+        for c in range(w.n_chunks):
+            for d in range(w.denoise_steps):
+                for l in range(w.n_layers):
+                    (cache.append_chunk if d == 0 else cache.set_current)(l, *kv[c])
+                    calls += 1
+                if d == 0:
+                    cache.compress()
+                    calls += 1
+                for l in range(w.n_layers):
+                    cache.attend(l, qs[d], out_t)
+                    calls += 1
+        return calls
+
+    with ForcingKVCache.from_workload(w, hm, device=local_rank) as cache:   # warm-up pass
+        run(cache)
+        torch.cuda.synchronize()
+    with ForcingKVCache.from_workload(w, hm, device=local_rank) as cache:
+        torch.cuda.synchronize()
+        n0 = cache.launch_count()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        t0 = time.perf_counter()
+        e0.record()
+        calls = run(cache)
+        e1.record()
+        torch.cuda.synchronize()
+        wall = time.perf_counter() - t0
+        launches = cache.launch_count() - n0
+        if cache.sync_status() != 0:
+            raise SystemExit("device status error in the stack run")
+        reserved = cache.reserved_bytes()
+    frames = w.n_chunks * w.frames_per_chunk
+    return {"frames": frames, "layers": w.n_layers, "heads": w.n_heads, "denoise_steps": w.denoise_steps,
+            "wall_s": round(wall, 4), "device_s": round(e0.elapsed_time(e1) * 1e-3, 4),
+            "fps": round(frames / wall, 2), "library_calls": calls, "gpu_launches": int(launches),
+            "reserved_gb": round(reserved / 1e9, 2),
+            "note": "layer-0 pooled scoring, incremental; every fk_* call of the 7 chunks inside the wall time"}
 
 
 # DRAM bytes (read + write) per launch from one ncu capture of each kernel on the 480P
@@ -431,6 +496,7 @@ def main(argv=None):
     ap.add_argument("--workload", default="480p_layer")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-stack", action="store_true", help="skip the directly measured 480P stack")
     args = ap.parse_args(argv)
     if args.warmup < 3:
         ap.error("--warmup must be at least 3")
