@@ -2,7 +2,9 @@
 // current chunk joins the history pages and the new chunk is scattered from the caller's
 // token-major [tokens][H][D] layout into the per-head views, in one pass), the prefill
 // scatter of history frames, and the select-and-compact gather of kept segments into the
-// packed per-head views of dynamic heads (Sec. 4.3, Eq. 4: [sink, kept segments, anchor]).
+// packed per-head views of dynamic heads (Sec. 4.3, Eq. 4: sink, kept segments and the
+// anchor frame; attention does not depend on the order of the keys, so a view holds them as
+// [sinks | anchor | kept-segment ring] and incremental compaction only appends).
 // All of them are HBM-bound: every byte is read once and written once in 16-byte accesses.
 #include "fk_internal.h"
 
@@ -31,9 +33,16 @@ __device__ __forceinline__ int ring_slot(int f, int S, int cap) {
   return f < S ? f : S + (f - S) % cap;
 }
 
+// programmatic dependent launch (no-ops for a launch without the programmatic attribute):
+// let the next kernel of the stream be scheduled / wait until the previous kernel of the
+// stream has completed and its writes are visible
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 // One thread per 16-byte granule of the current chunk, indexed in the caller's token-major
 // order (row, head, granule) so that the reads of the new chunk are fully coalesced.
 __global__ void __launch_bounds__(256) current_kernel(const CurrentArgs a) {
+  pdl_trigger();   // the scoring kernel that follows may start its prologue; it waits for us
   const int gpr = a.head_dim / 8;
   const uint32_t per_row = (uint32_t)(a.heads * gpr);
   const uint32_t total = (uint32_t)a.rows * per_row;   // < 2^31 (checked at configuration)
@@ -99,33 +108,42 @@ __global__ void __launch_bounds__(256) scatter_kernel(const ScatterArgs a) {
 }
 
 // One CTA copies one piece (<= 16 KB of keys and 16 KB of values) of one unit of one
-// dynamic head's view.  Units in view order: sink frames (n units each), kept segments
-// (ascending t*n+j), anchor frame (n units); unit u lands at view row CF + u*seg_len.
+// dynamic head's view.  Units in order: the sink frames to copy (n units each), the anchor
+// frame (n units), the kept segments to copy (one unit each, taken from the target's kept
+// list).  View rows after the current chunk: sink frame f at S-slot f, the anchor after the
+// sinks, kept segment i in ring slot (rp0 + i) mod kmax after the anchor.
 __global__ void __launch_bounds__(256) compact_kernel(const CompactArgs a) {
+  pdl_trigger();
+  pdl_wait();      // kept lists and pages come from the kernels before this one
   const CompactItem it = a.items[blockIdx.y];
   const int l = it.layer;
   if (!a.active[l]) return;
   const int u = blockIdx.x / a.splits;
   const int piece = blockIdx.x - u * a.splits;
-  const int n_sink_units = a.n_sink_present[l] * a.n_seg;
-  const int n_keep = a.n_keep[l];
-  const int units = n_sink_units + n_keep + (a.anchor[l] >= 0 ? a.n_seg : 0);
-  if (u >= units) return;
+  const int n_sink_units = a.n_sink_copy[l] * a.n_seg;
+  const int n_anchor_units = a.anchor[l] >= 0 ? a.n_seg : 0;
+  if (u >= n_sink_units + n_anchor_units + a.n_kept_copy[l]) return;
   int frame, seg;
+  int64_t dst_row = a.CF;
   if (u < n_sink_units) {
-    frame = u / a.n_seg;
-    seg = u - frame * a.n_seg;
-  } else if (u < n_sink_units + n_keep) {
-    const int sid = a.kept[(int64_t)it.target * a.kmax + (u - n_sink_units)];
+    frame = a.sink_first[l] + u / a.n_seg;
+    seg = u - (u / a.n_seg) * a.n_seg;
+    dst_row += (int64_t)frame * a.F + (int64_t)seg * a.seg_len;
+  } else if (u < n_sink_units + n_anchor_units) {
+    frame = a.anchor[l];
+    seg = u - n_sink_units;
+    dst_row += (int64_t)a.S * a.F + (int64_t)seg * a.seg_len;
+  } else {
+    const int i = u - n_sink_units - n_anchor_units;
+    const int sid = a.kept[(int64_t)it.target * a.kmax + a.kp0[l] + i];
     frame = sid / a.n_seg;
     seg = sid - frame * a.n_seg;
-  } else {
-    frame = a.anchor[l];
-    seg = u - n_sink_units - n_keep;
+    const int slot = (a.rp0[l] + i) % a.kmax;
+    dst_row += (int64_t)a.S * a.F + a.F + (int64_t)slot * a.seg_len;
   }
   const int slot = ring_slot(frame, a.S, a.cap_nonsink);
   const int64_t src_off = ((int64_t)slot * a.F + (int64_t)seg * a.seg_len) * a.D;
-  const int64_t dst_off = ((int64_t)a.CF + (int64_t)u * a.seg_len) * a.D;
+  const int64_t dst_off = dst_row * a.D;
   const int64_t n = (int64_t)a.seg_len * a.D / 8;      // 16-byte granules per tensor
   const int64_t g0 = (int64_t)piece * (kCompactPiece / 16);
   const uint4* sK = reinterpret_cast<const uint4*>(it.pagesK + src_off);
@@ -174,7 +192,18 @@ void launch_scatter(const ScatterArgs& a, cudaStream_t s) {
 
 void launch_compact(const CompactArgs& a, cudaStream_t s) {
   if (a.n_items == 0 || a.max_units == 0) return;
-  compact_kernel<<<dim3((unsigned)(a.max_units * a.splits), (unsigned)a.n_items), 256, 0, s>>>(a);
+  // programmatic launch: the grid is scheduled while the selection kernel runs
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3((unsigned)(a.max_units * a.splits), (unsigned)a.n_items);
+  cfg.blockDim = dim3(256);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cudaLaunchKernelEx(&cfg, compact_kernel, a);
 }
 
 }  // namespace fk

@@ -7,7 +7,8 @@
 //   view arenas  K and V, [rows][D] bf16 each; head (l, h) owns rows
 //                [row_base, row_base + view_rows), padded to whole 128-key tiles.
 //                Static head view:  [current chunk C*F | sink S*F | anchor F]
-//                Dynamic head view: [current chunk C*F | sink | kept segments | anchor F]
+//                Dynamic head view: [current chunk C*F | sink S*F | anchor F | kept-segment
+//                ring of kmax slots] (attention does not depend on the key order)
 //   page rings   K and V, [ring_slots][F][D] per head that keeps history for scoring
 //                (dynamic heads; every head of layer 0 under layer-0 pooled scoring);
 //                frame f lives in slot f (f < S) or S + (f - S) mod cap_nonsink.
@@ -50,6 +51,12 @@ struct LayerState {
   int n_keep = 0;         // kept segments of each dynamic head (after fk_compress)
   int len_static = 0;     // keys of a static head
   int len_dynamic = 0;    // keys of a dynamic head
+  // incremental compaction: the dynamic views' kept-segment ring holds the kept segments of
+  // frames [ring_first, ring_end), the first of them at ring slot ring_head
+  int ring_first = 0;
+  int ring_end = 0;
+  int ring_head = 0;
+  int sinks_done = 0;     // sink frames already in the dynamic views
 };
 
 struct ProfRec {
@@ -678,6 +685,9 @@ fk_status fk_compress(fk_handle* h, void* stream) {
   ScoreArgs sa{};
   CompactArgs ca{};
   bool any_run = false, any_compact = false;
+  // incremental compaction needs kept sets that never change once decided: per-frame scope
+  const bool inc_compact = h->incremental && h->scope == FK_SCOPE_PER_FRAME;
+  std::vector<int> keep_of(h->L, 0);
   for (int l = 0; l < h->L; ++l) {
     LayerState& ls = h->layers[l];
     const Roles r = roles_of(h, ls.nh);
@@ -696,12 +706,41 @@ fk_status fk_compress(fk_handle* h, void* stream) {
     sa.t_lo[l] = r.t_lo;
     sa.n_scoreable[l] = r.n_scoreable;
     sa.n_keep[l] = keep;
-    ca.n_sink_present[l] = r.n_sink;
-    ca.n_keep[l] = keep;
+    keep_of[l] = keep;
     ca.anchor[l] = r.anchor;
     ca.active[l] = ls.dirty ? 1 : 0;
-    const int units = r.n_sink * h->n + keep + (r.anchor >= 0 ? h->n : 0);
-    ca.max_units = std::max(ca.max_units, ls.dirty ? units : 0);
+    if (!ls.dirty) continue;
+    if (inc_compact) {
+      // sinks not yet in the views
+      ca.sink_first[l] = ls.sinks_done;
+      ca.n_sink_copy[l] = r.n_sink - ls.sinks_done;
+      ls.sinks_done = r.n_sink;
+      // frames below the window leave the ring; the newly decided frames are appended.  A
+      // frame leaves only once the window is full, and then the ring is full again after the
+      // append, so the valid slots are always [0, count) or all kmax: one contiguous key range
+      const int t_hi = r.t_lo + r.n_scoreable;
+      if (r.t_lo > ls.ring_first) {
+        const int gone = std::min(r.t_lo, ls.ring_end) - ls.ring_first;
+        if (gone > 0)
+          ls.ring_head = (int)(((int64_t)ls.ring_head + (int64_t)gone * h->k_frame) % h->kmax);
+        ls.ring_first = r.t_lo;
+        ls.ring_end = std::max(ls.ring_end, r.t_lo);
+      }
+      const int n_add = std::max(0, t_hi - ls.ring_end);
+      ca.n_kept_copy[l] = n_add * h->k_frame;
+      ca.kp0[l] = (ls.ring_end - r.t_lo) * h->k_frame;
+      ca.rp0[l] = (int)(((int64_t)ls.ring_head + (int64_t)(ls.ring_end - ls.ring_first) * h->k_frame) % h->kmax);
+      ls.ring_end = std::max(ls.ring_end, t_hi);
+      if (ls.ring_head != 0 && keep != h->kmax) return FK_ERR_STATE;   // cannot happen (see above)
+    } else {
+      ca.sink_first[l] = 0;
+      ca.n_sink_copy[l] = r.n_sink;
+      ca.n_kept_copy[l] = keep;
+      ca.kp0[l] = 0;
+      ca.rp0[l] = 0;
+    }
+    const int units = ca.n_sink_copy[l] * h->n + ca.n_kept_copy[l] + (r.anchor >= 0 ? h->n : 0);
+    ca.max_units = std::max(ca.max_units, units);
   }
   for (const auto& ci : h->compact_items) any_compact |= ca.active[ci.layer] != 0;
   fk_status st;
@@ -760,7 +799,7 @@ fk_status fk_compress(fk_handle* h, void* stream) {
   for (int l = 0; l < h->L; ++l) {
     LayerState& ls = h->layers[l];
     if (!ls.dirty) continue;
-    ls.n_keep = ca.n_keep[l];
+    ls.n_keep = keep_of[l];
     ls.dirty = false;
     update_lengths(h, l);
   }

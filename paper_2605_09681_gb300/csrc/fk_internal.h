@@ -130,9 +130,14 @@ struct CompactArgs {
   int S, cap_nonsink, kmax;
   int splits;                   // pieces per unit (each at most kCompactPiece bytes per tensor)
   const int* kept;
-  int n_sink_present[kMaxLayers];
-  int n_keep[kMaxLayers];
-  int anchor[kMaxLayers];       // -1 = none
+  // per layer: what this launch copies into the dynamic views [current | sinks | anchor |
+  // kept ring of kmax segment slots]
+  int sink_first[kMaxLayers];   // first sink frame to copy
+  int n_sink_copy[kMaxLayers];  // sink frames to copy
+  int anchor[kMaxLayers];       // anchor frame (copied whole), -1 = none
+  int n_kept_copy[kMaxLayers];  // kept segments to copy
+  int kp0[kMaxLayers];          // their first position in the target's kept list
+  int rp0[kMaxLayers];          // ring slot of the first one (slots wrap modulo kmax)
   unsigned char active[kMaxLayers];
   int max_units;
 };

@@ -132,8 +132,10 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const ScoreArgs 
   const int l = tg.layer;
   const LayerRun run = a.run[l];
   pdl_trigger();
-  if (run.n_run < 2) return;
+  // every CTA waits, even one with nothing to do: this kernel's completion then implies the
+  // completion of the kernels before it, which the next programmatic launch relies on
   pdl_wait();
+  if (run.n_run < 2) return;
   const int n = a.n_seg;
   const int nT = a.n_scoreable[l];
   const int M = nT * n;

@@ -139,6 +139,35 @@ def test_stream_window_small():
     assert _stream(w) == 12
 
 
+def test_incremental_compaction_matches_rebuild():
+    # Incremental mode appends only newly decided segments into a ring of kept-segment slots;
+    # the rebuild copies every kept segment each time.  The views hold the same keys in a
+    # different order (the ring wraps once the 5-frame window is full): key counts agree and
+    # the attention outputs agree up to summation order.
+    from paper_2605_09681_gb300 import ForcingKVCache
+    w = W.ROLLING.with_(name="ring", head_dim=64, tokens_per_frame=120, n_heads=4, window_frames=5,
+                        n_chunks=9, scene_cut_every_chunks=4)
+    hm = W.head_map(w)
+    runs = []
+    for inc in (True, False):
+        fs = W.FrameStream(w, 0)
+        res = []
+        with ForcingKVCache.from_workload(w, hm, incremental=inc) as cache:
+            for c in range(w.n_chunks):
+                k, v = fs.frames(w.frames_per_chunk)
+                cache.append_chunk(0, to_dev(k), to_dev(v))
+                cache.compress()
+                O = cache.attend(0, to_dev(W.queries(w, 0, c, 0)))
+                res.append(([cache.key_count(0, h) for h in range(w.n_heads)],
+                            [cache.kept(0, h) for h in range(w.n_heads)], to_f64(O)))
+            assert cache.sync_status() == 0
+        runs.append(res)
+    for (ka, sa, oa), (kb, sb, ob) in zip(*runs):
+        assert ka == kb and sa == sb
+        err = np.abs(oa - ob)
+        assert err.max() <= ATOL_MAX and err.mean() <= ATOL_MEAN / 4
+
+
 def test_stream_incremental_matches_rescore():
     from paper_2605_09681_gb300 import ForcingKVCache
     w = W.ROLLING.with_(name="inc", head_dim=64, tokens_per_frame=60, n_heads=4, window_frames=6,
