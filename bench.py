@@ -329,6 +329,7 @@ def run_fk(args, rank, world, local_rank):
     cache.close()
     out["incremental"] = run_incremental(args, w, hm, local_rank, to_t(hk).to(dev), to_t(hv).to(dev),
                                          dK, dV, dQ, dO, flush, stream, world, peaks)
+    out["head_profile_480p"] = run_head_profile(args, local_rank, flush, peaks)
     if not args.no_stack:
         out["stack_480p"] = run_stack(local_rank)
     if rank == 0 and not args.no_cpu_baseline:
@@ -409,6 +410,42 @@ def run_incremental(args, w, hm, local_rank, hk, hv, dK, dV, dQ, dO, flush, stre
         "note": "per step: scoring reads C + 1 frames per dynamic head, compaction copies C x k "
                 "segments + the anchor frame per dynamic head (ring-buffer views)",
     }
+
+
+def run_head_profile(args, local_rank, flush, peaks):
+    """Offline head profiling (Eq. 1) over one 480P full attention window: the 4680 queries of
+    a 3-frame chunk against all 34320 keys (3 generated + 1 sink + 17 other + 1 transition
+    frames) of 12 heads, D = 128; device-resident random bf16 inputs (the work does not
+    depend on the values); L2 flushed between launches."""
+    import torch
+
+    from paper_2605_09681_gb300 import head_profile
+
+    F, H, D, C = 1560, 12, 128, 3
+    nq, nk = C * F, 22 * F
+    g = torch.Generator(device="cuda").manual_seed(9)
+    dev = torch.device("cuda", local_rank)
+    Q = torch.randn((nq, H, D), generator=g, device=dev).to(torch.bfloat16)
+    K = torch.randn((nk, H, D), generator=g, device=dev).to(torch.bfloat16)
+    mass, status = head_profile(Q, K, C * F, F, F)
+    reps = max(3, min(args.steps, 20))
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(reps)]
+    torch.cuda.synchronize()
+    for i in range(reps):
+        flush.zero_()
+        evs[i][0].record()
+        head_profile(Q, K, C * F, F, F, mass=mass, status=status)
+        evs[i][1].record()
+    torch.cuda.synchronize()
+    if int(status.item()) != 0:
+        raise SystemExit("device status error in the head-profiling run")
+    ms = sum(a.elapsed_time(b) for a, b in evs) / reps
+    flops = 2.0 * nq * nk * D * H
+    return {"queries": nq, "keys": nk, "heads": H, "head_dim": D, "us": round(ms * 1e3, 2),
+            "qk_tflops": round(flops / (ms * 1e-3) / 1e12, 1),
+            "qk_frac_of_bf16_peak": round(flops / (ms * 1e-3) / 1e12 / peaks["bf16_tflops"], 4),
+            "gexp_per_s": round(nq * nk * H / (ms * 1e-3) / 1e9, 1),
+            "note": "S = Q K^T on tcgen05 plus a softmax with class sums per key; no P V"}
 
 
 def run_stack(local_rank):

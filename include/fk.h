@@ -202,6 +202,31 @@ FK_API fk_status fk_segment_scores_noalloc(const void* K, int n_frames, int toke
                                            int head_dim, int n_segments, float* scores,
                                            void* stream);
 
+/* Offline head profiling (Sec. 4.1, Eq. 1): attention mass per key class.
+ * Q: device [n_queries][n_heads][head_dim] bf16, the queries of the generated chunk.
+ * K: device [n_keys][n_heads][head_dim] bf16, every key of the attention window in the order
+ *    [generated chunk (n_generate) | sink frames (n_sink) | other history | transition frame
+ *    (n_transition, the last frame before the chunk)]; both 16-byte aligned, token-major.
+ * For every head h and query row, the softmax over all n_keys keys (scale 1/sqrt(head_dim))
+ * is split by key class; the row's fractions are summed over the rows and ADDED to
+ * mass[h][0..3] = {A_Total (= rows), A_Generate, A_Transition, A_Sink} (device, double; the
+ * caller zeroes it, so repeated calls accumulate over steps).  A bounded device wait that
+ * expires ORs the value 2 into *status (device int, caller-owned, zeroed by the caller).
+ * Errors: FK_ERR_ARG for null, unaligned or host pointers; FK_ERR_CONFIG for head_dim not 64
+ * or 128, n_heads outside 1..128, empty Q or K, or class counts exceeding n_keys.
+ * Asynchronous on `stream`; allocates nothing; uses the current device. */
+FK_API fk_status fk_head_profile(const void* Q, const void* K, int n_queries, int n_keys,
+                                 int n_heads, int head_dim, int n_generate, int n_sink,
+                                 int n_transition, double* mass, int* status, void* stream);
+
+/* Eq. 1 on host-side masses ([n_heads][4] as written by fk_head_profile): head h is static
+ * (head_is_static[h] = 1) when (A_Generate + A_Transition) / (A_Total - A_Sink) exceeds
+ * alpha_permille / 1000 (alpha = 0.8 in the paper: 800), else dynamic (0).  A head with all
+ * of its mass on the sink frames (A_Total - A_Sink <= 0) is static.  FK_ERR_ARG for null
+ * pointers, FK_ERR_CONFIG for alpha outside 0..1000. */
+FK_API fk_status fk_classify_heads(const double* mass, int n_heads, int alpha_permille,
+                                   uint8_t* head_is_static);
+
 /* Static text for a status code. */
 FK_API const char* fk_status_str(fk_status s);
 

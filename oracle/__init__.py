@@ -4,7 +4,8 @@ Imported by the test suite, the smoke check and the benchmark's CPU-baseline
 leg; never by the library.  See `oracle.forcing_kv` for the definitions.
 """
 from .forcing_kv import *  # noqa: F401,F403
-from .forcing_kv import (ForcingKVOracle, FrameRoles, attention_fp64, bottom_k, cosine_fp64,
+from .forcing_kv import (ForcingKVOracle, FrameRoles, attention_fp64, bottom_k, classify_head,
+                         cosine_fp64, head_attention_mass,
                          dynamic_key_tokens, fixed_point, fmaf_bf16, frame_roles, keep_count,
                          score_from_sums, segment_range, segment_score_contract,
                          segment_sums_contract, static_key_tokens, token_dots_contract)

@@ -29,7 +29,8 @@ Readings taken where the paper is silent (each is listed with its reason in the
 design notes): k = floor(b * n) segments kept per frame with b = 1 - r the keep
 budget; cosine of two segments = Frobenius cosine of the flattened (F/n) x D key
 blocks; the anchor frame is kept whole for dynamic heads and never scored; sink
-frames are never scored and never evicted; the window W counts non-sink history
+frames are never scored and never evicted; a head profiled with all of its mass on the
+sink frames is static (Eq. 1 has a zero denominator there); the window W counts non-sink history
 frames including the anchor; ties in BottomK go to the lower index; the layer-0
 proxy pools the int64 sums over all heads of layer 0.
 
@@ -223,6 +224,49 @@ def attention_fp64(Q: np.ndarray, K: np.ndarray, V: np.ndarray, row_block: int =
         p = np.exp(logits)
         out[r0:r0 + row_block] = (p @ V) / p.sum(axis=1, keepdims=True)
     return out
+
+
+# --------------------------------------------------------------------------------------
+# offline head profiling (Sec. 4.1, Eq. 1)
+# --------------------------------------------------------------------------------------
+def head_attention_mass(Q: np.ndarray, K: np.ndarray, n_generate: int, n_sink: int,
+                        n_transition: int, row_block: int = 256) -> np.ndarray:
+    """Attention mass of one head per key class (Sec. 4.1), in fp64.
+
+    Q [Nq, D], K [Nk, D] with the keys ordered [generated chunk | sink frames | other
+    history | transition frame].  Each query row's softmax over all Nk keys (scale
+    1/sqrt(D)) is summed per class and the rows are summed: returns
+    [A_Total, A_Generate, A_Transition, A_Sink], where A_Total = sum over rows of the whole
+    window's mass (each row contributes 1)."""
+    Q = np.asarray(Q, dtype=np.float64)
+    K = np.asarray(K, dtype=np.float64)
+    nk = K.shape[0]
+    assert n_generate + n_sink + n_transition <= nk
+    scale = 1.0 / np.sqrt(Q.shape[1])
+    gen = slice(0, n_generate)
+    sink = slice(n_generate, n_generate + n_sink)
+    trans = slice(nk - n_transition, nk)
+    total = a_gen = a_trans = a_sink = 0.0
+    for r0 in range(0, Q.shape[0], row_block):
+        logits = (Q[r0:r0 + row_block] @ K.T) * scale
+        logits -= logits.max(axis=1, keepdims=True)
+        p = np.exp(logits)
+        p /= p.sum(axis=1, keepdims=True)
+        total += float(p.sum())
+        a_gen += float(p[:, gen].sum())
+        a_trans += float(p[:, trans].sum()) if n_transition else 0.0
+        a_sink += float(p[:, sink].sum())
+    return np.array([total, a_gen, a_trans, a_sink], dtype=np.float64)
+
+
+def classify_head(mass, alpha: float) -> bool:
+    """Eq. 1: static when (A_Generate + A_Transition) / (A_Total - A_Sink) > alpha.  A head
+    whose whole mass is on the sink frames (denominator <= 0) is read as static."""
+    total, a_gen, a_trans, a_sink = (float(x) for x in mass)
+    window = total - a_sink
+    if window <= 0.0:
+        return True
+    return (a_gen + a_trans) / window > alpha
 
 
 # --------------------------------------------------------------------------------------

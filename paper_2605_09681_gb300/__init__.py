@@ -13,7 +13,8 @@ import numpy as np
 from . import _lib as L
 from ._lib import FkError, KERNEL_KINDS, STATUS_NAMES
 
-__all__ = ["ForcingKVCache", "FkError", "KERNEL_KINDS", "STATUS_NAMES", "load_library"]
+__all__ = ["ForcingKVCache", "FkError", "KERNEL_KINDS", "STATUS_NAMES", "load_library",
+           "head_profile", "classify_heads"]
 
 
 def load_library():
@@ -50,6 +51,44 @@ def _stream(stream) -> int | None:
             return torch.cuda.current_stream().cuda_stream
         return None
     return getattr(stream, "cuda_stream", stream)
+
+
+def head_profile(Q, K, n_generate: int, n_sink: int, n_transition: int, mass=None, status=None,
+                 stream=None):
+    """Offline head profiling (Sec. 4.1, Eq. 1) through fk_head_profile.
+
+    Q [Nq, H, D] and K [Nk, H, D]: contiguous torch.bfloat16 CUDA tensors, keys ordered
+    [generated | sink | other history | transition].  Adds each head's attention mass
+    {A_Total, A_Generate, A_Transition, A_Sink} to `mass` (float64 [H, 4] on the device,
+    created zeroed when None) and returns (mass, status); status is an int32 device tensor
+    whose nonzero value means a bounded device wait expired."""
+    import torch
+    nq, H, D = Q.shape
+    nk = K.shape[0]
+    if tuple(K.shape[1:]) != (H, D):
+        raise ValueError("Q and K disagree on heads / head_dim")
+    if mass is None:
+        mass = torch.zeros((H, 4), dtype=torch.float64, device=Q.device)
+    if status is None:
+        status = torch.zeros(1, dtype=torch.int32, device=Q.device)
+    lib = L.load()
+    _check(lib.fk_head_profile(_ptr(Q), _ptr(K), nq, nk, H, D, n_generate, n_sink, n_transition,
+                               mass.data_ptr(), status.data_ptr(), _stream(stream)),
+           "fk_head_profile")
+    return mass, status
+
+
+def classify_heads(mass, alpha: float = 0.8) -> np.ndarray:
+    """Eq. 1 on masses [H, 4] (host copy): 1 = static, 0 = dynamic (fk_classify_heads)."""
+    m = np.ascontiguousarray(np.asarray(mass, dtype=np.float64))
+    H = m.shape[0]
+    out = np.zeros(H, dtype=np.uint8)
+    lib = L.load()
+    _check(lib.fk_classify_heads(m.ctypes.data_as(ctypes.POINTER(ctypes.c_double)), H,
+                                 int(round(alpha * 1000)),
+                                 out.ctypes.data_as(ctypes.POINTER(ctypes.c_uint8))),
+           "fk_classify_heads")
+    return out
 
 
 class ForcingKVCache:

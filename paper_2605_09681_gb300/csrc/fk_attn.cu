@@ -558,7 +558,236 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
   }
 }
 
+// ---------------------------------------------------------------------------------------
+// Offline head profiling (Sec. 4.1, Eq. 1): per head, the attention mass that the queries of
+// the generated chunk put on the generated chunk, the transition (anchor) frame and the sink
+// frames, out of a full softmax over every key of the attention window.  Keys are ordered
+// [generated | sink | other history | transition].  S = Q K^T runs on the tensor cores
+// (tcgen05, S double-buffered in 256 TMEM columns); no P V product is needed.  Per row the
+// softmax statistics are kept online (running max, total sum, and the three class sums,
+// rescaled together); the per-row fractions are summed per head in double.
+//   warps 0-3  statistics of rows 0..127 (TMEM lanes), one thread per row;
+//   warp 4     TMA: the query tile once, key tiles into a two-stage ring;
+//   warp 5     tcgen05.mma: S_b = Q K_j^T for b = j mod 2, once the statistics warps have
+//              read S_b of tile j - 2 (they release it right after their TMEM loads).
+constexpr int kProfThreads = 192;
+constexpr int kWarpProfTma = 4;
+constexpr int kWarpProfMma = 5;
+
+template <int D>
+struct ProfLayout {
+  static constexpr int kQ = kAttnBM * D * 2;
+  static constexpr int kK = kAttnBN * D * 2;
+  static constexpr int kOffQ = 0;
+  static constexpr int kOffK = kOffQ + kQ;
+  static constexpr int kOffBar = kOffK + 2 * kK;
+  static constexpr int kSmem = kOffBar + 256 + 1024;   // + alignment slack; two CTAs per SM
+};
+
+template <int D>
+__global__ void __launch_bounds__(kProfThreads, 2)
+profile_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+               const ProfArgs a) {
+  using Lay = ProfLayout<D>;
+  constexpr int kHalves = D / 64;
+  constexpr uint32_t kTmemCols = 256;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  uint8_t* sQ = smem + Lay::kOffQ;
+  uint8_t* sK = smem + Lay::kOffK;
+  AttnBarriers* bar = reinterpret_cast<AttnBarriers*>(smem + Lay::kOffBar);
+  // barrier use: q_full, k_full/k_empty (key ring), s_full[b] (S_b written), p_full[b]
+  // (S_b read by the four statistics warps), fin
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int head = blockIdx.x / a.n_qtiles;
+  const int q0 = (blockIdx.x - head * a.n_qtiles) * kAttnBM;
+  const int nk = a.Nk;
+  const int nt = (nk + kAttnBN - 1) / kAttnBN;
+
+  if (threadIdx.x == 0) {
+    mbar_init(&bar->q_full, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&bar->k_full[i], 1);
+      mbar_init(&bar->k_empty[i], 1);
+      mbar_init(&bar->s_full[i], 1);
+      mbar_init(&bar->p_full[i], 4);
+    }
+    mbar_init(&bar->fin, 1);
+    bar->abort = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == kWarpProfMma) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;"
+                 :: "r"(su32(&bar->tmem_base)), "r"(kTmemCols) : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = bar->tmem_base;
+
+  if (warp == kWarpProfTma) {
+    if (lane == 0) {
+      int lastK[2] = {-1, -1};
+      bool ok = true;
+      mbar_expect_tx(&bar->q_full, Lay::kQ);
+      for (int h = 0; h < kHalves; ++h)
+        tma_load_3d(sQ + h * 16384, &tmQ, &bar->q_full, h * 64, head, q0);
+      for (int j = 0; j < nt; ++j) {
+        const int st = j & 1, u = j >> 1;
+        if (j >= 2 && !wait_phase(&bar->k_empty[st], (u - 1) & 1, bar, a.status)) { ok = false; break; }
+        mbar_expect_tx(&bar->k_full[st], Lay::kK);
+        for (int h = 0; h < kHalves; ++h)
+          tma_load_3d(sK + st * Lay::kK + h * 16384, &tmK, &bar->k_full[st], h * 64, head,
+                      j * kAttnBN);
+        lastK[st] = u;
+      }
+      if (!ok) {   // drain every load this thread issued before the CTA exits
+        wait_phase(&bar->q_full, 0, bar, a.status, false);
+        for (int st = 0; st < 2; ++st)
+          if (lastK[st] >= 0) wait_phase(&bar->k_full[st], lastK[st] & 1, bar, a.status, false);
+      }
+    }
+    __syncwarp();
+  } else if (warp == kWarpProfMma) {
+    if (lane == 0) {
+      constexpr uint32_t kIdQK = idesc_bf16(kAttnBM, kAttnBN, 0);
+      const uint32_t aQ = su32(sQ), aK = su32(sK);
+      bool ok = wait_phase(&bar->q_full, 0, bar, a.status);
+      for (int j = 0; j < nt && ok; ++j) {
+        const int st = j & 1, u = j >> 1;
+        if (!wait_phase(&bar->k_full[st], u & 1, bar, a.status) ||
+            (j >= 2 && !wait_phase(&bar->p_full[st], (u - 1) & 1, bar, a.status))) { ok = false; break; }
+        tc_fence_after();
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk) {
+          const uint64_t da = sdesc(aQ + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024);
+          const uint64_t db = sdesc(aK + st * Lay::kK + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024);
+          umma(tmem + (uint32_t)(st * kAttnBN), da, db, kIdQK, kk > 0 ? 1u : 0u);
+        }
+        umma_commit(&bar->s_full[st]);
+        umma_commit(&bar->k_empty[st]);
+      }
+      umma_commit(&bar->fin);                       // completes once every MMA above is done
+      wait_phase(&bar->fin, 0, bar, a.status, false);
+    }
+    __syncwarp();
+  } else {
+    const int wq = warp;
+    const int row = wq * 32 + lane;
+    const uint32_t lane_base = (uint32_t)(wq * 32) << 16;
+    float m = -INFINITY, l = 0.0f, cg = 0.0f, cs = 0.0f, ct = 0.0f;
+    bool ok = true;
+    for (int j = 0; j < nt; ++j) {
+      const int st = j & 1;
+      if (!warp_wait(&bar->s_full[st], (j >> 1) & 1, bar, a.status)) { ok = false; break; }
+      tc_fence_after();
+#pragma unroll
+      for (int half = 0; half < 2; ++half) {
+        const int kb = j * kAttnBN + half * 64;      // first key of this half
+        const int valid = min(64, nk - kb);          // uniform over the CTA
+        uint32_t sv[64];
+        FK_TMEM_LD64(tmem + lane_base + (uint32_t)(st * kAttnBN + half * 64), sv);
+        tmem_wait_ld();
+        if (half == 1) {                             // S_b is in registers: release it
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&bar->p_full[st]);
+        }
+        if (valid <= 0) continue;
+        float mx = -INFINITY;
+#pragma unroll
+        for (int c = 0; c < 64; ++c)
+          if (c < valid) mx = fmaxf(mx, __uint_as_float(sv[c]));
+        const float m_new = fmaxf(m, mx * a.scale_log2);
+        if (__any_sync(0xffffffffu, m_new > m + kRescaleThreshold)) {   // warp-uniform
+          const float alpha = fast_exp2(m - m_new);  // 0 when m = -inf
+          l *= alpha;
+          cg *= alpha;
+          cs *= alpha;
+          ct *= alpha;
+          m = m_new;
+        }
+        // key classes are contiguous ranges in the order generated, sink, other, transition
+        const int last = kb + valid - 1;
+        const int cls_first = kb < a.g_end ? 0 : kb < a.s_end ? 1 : kb >= a.t_begin ? 3 : 2;
+        const int cls_last = last < a.g_end ? 0 : last < a.s_end ? 1 : last >= a.t_begin ? 3 : 2;
+        if (cls_first == cls_last) {
+          float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+#pragma unroll
+          for (int c = 0; c < 64; ++c)
+            if (c < valid) acc[c & 3] += fast_exp2(fmaf(__uint_as_float(sv[c]), a.scale_log2, -m));
+          const float sum = (acc[0] + acc[1]) + (acc[2] + acc[3]);
+          l += sum;
+          if (cls_first == 0) cg += sum;
+          else if (cls_first == 1) cs += sum;
+          else if (cls_first == 3) ct += sum;
+        } else {
+#pragma unroll
+          for (int c = 0; c < 64; ++c) {
+            if (c < valid) {
+              const int key = kb + c;
+              const float e = fast_exp2(fmaf(__uint_as_float(sv[c]), a.scale_log2, -m));
+              l += e;
+              if (key < a.g_end) cg += e;
+              else if (key < a.s_end) cs += e;
+              else if (key >= a.t_begin) ct += e;
+            }
+          }
+        }
+      }
+    }
+    if (ok) {
+      const bool in = q0 + row < a.Nq;
+      float fg = in ? cg / l : 0.0f, fs = in ? cs / l : 0.0f, ft = in ? ct / l : 0.0f;
+      float rows = in ? 1.0f : 0.0f;
+#pragma unroll
+      for (int sft = 16; sft >= 1; sft >>= 1) {
+        fg += __shfl_xor_sync(0xffffffffu, fg, sft);
+        fs += __shfl_xor_sync(0xffffffffu, fs, sft);
+        ft += __shfl_xor_sync(0xffffffffu, ft, sft);
+        rows += __shfl_xor_sync(0xffffffffu, rows, sft);
+      }
+      if (lane == 0 && rows > 0.0f) {
+        double* mh = a.mass + (int64_t)head * 4;
+        atomicAdd(mh + 0, (double)rows);
+        atomicAdd(mh + 1, (double)fg);
+        atomicAdd(mh + 2, (double)ft);
+        atomicAdd(mh + 3, (double)fs);
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == kWarpProfMma) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" :: "r"(tmem),
+                 "r"(kTmemCols) : "memory");
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_head_profile(int head_dim, const CUtensorMap& tmQ, const CUtensorMap& tmK,
+                                const ProfArgs& a, cudaStream_t s) {
+  const unsigned grid = (unsigned)(a.n_qtiles * a.H);
+  cudaError_t e;
+  if (head_dim == 128) {
+    e = cudaFuncSetAttribute(profile_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             ProfLayout<128>::kSmem);
+    if (e != cudaSuccess) return e;
+    profile_kernel<128><<<grid, kProfThreads, ProfLayout<128>::kSmem, s>>>(tmQ, tmK, a);
+  } else {
+    e = cudaFuncSetAttribute(profile_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             ProfLayout<64>::kSmem);
+    if (e != cudaSuccess) return e;
+    profile_kernel<64><<<grid, kProfThreads, ProfLayout<64>::kSmem, s>>>(tmQ, tmK, a);
+  }
+  return cudaGetLastError();
+}
 
 cudaError_t attention_prepare(int head_dim) {
   if (head_dim == 128)

@@ -383,6 +383,57 @@ fk_status update_current(fk_handle* h, int layer, bool retire, const void* K, co
 
 extern "C" {
 
+fk_status fk_head_profile(const void* Q, const void* K, int n_queries, int n_keys, int n_heads,
+                          int head_dim, int n_generate, int n_sink, int n_transition, double* mass,
+                          int* status, void* stream) {
+  if (!Q || !K || !mass || !status) return FK_ERR_ARG;
+  if (!aligned16(Q) || !aligned16(K) || (reinterpret_cast<uintptr_t>(mass) & 7u) ||
+      (reinterpret_cast<uintptr_t>(status) & 3u))
+    return FK_ERR_ARG;
+  if (head_dim != 64 && head_dim != 128) return FK_ERR_CONFIG;
+  if (n_heads < 1 || n_heads > kMaxHeads || n_queries < 1 || n_keys < 1) return FK_ERR_CONFIG;
+  if (n_generate < 0 || n_sink < 0 || n_transition < 0 ||
+      (int64_t)n_generate + n_sink + n_transition > n_keys)
+    return FK_ERR_CONFIG;
+  const int64_t n_qtiles = (n_queries + kAttnBM - 1) / kAttnBM;
+  if (n_qtiles * n_heads >= ((int64_t)1 << 31)) return FK_ERR_CONFIG;
+  if (!is_device_ptr(Q) || !is_device_ptr(K) || !is_device_ptr(mass) || !is_device_ptr(status))
+    return FK_ERR_ARG;
+  if (!get_encode()) return FK_ERR_CUDA;
+  CUtensorMap tq{}, tk{};
+  fk_status st;
+  if ((st = encode_q(&tq, Q, n_queries, n_heads, head_dim)) != FK_OK) return st;
+  if ((st = encode_q(&tk, K, n_keys, n_heads, head_dim)) != FK_OK) return st;
+  ProfArgs a{};
+  a.Nq = n_queries;
+  a.Nk = n_keys;
+  a.H = n_heads;
+  a.n_qtiles = (int)n_qtiles;
+  a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)head_dim));
+  a.g_end = n_generate;
+  a.s_end = n_generate + n_sink;
+  a.t_begin = n_keys - n_transition;
+  a.mass = mass;
+  a.status = status;
+  return launch_head_profile(head_dim, tq, tk, a, static_cast<cudaStream_t>(stream)) == cudaSuccess
+             ? FK_OK
+             : FK_ERR_CUDA;
+}
+
+fk_status fk_classify_heads(const double* mass, int n_heads, int alpha_permille,
+                            uint8_t* head_is_static) {
+  if (!mass || !head_is_static || n_heads < 0) return FK_ERR_ARG;
+  if (alpha_permille < 0 || alpha_permille > 1000) return FK_ERR_CONFIG;
+  for (int hd = 0; hd < n_heads; ++hd) {
+    const double* m = mass + (int64_t)hd * 4;
+    const double local = m[1] + m[2];          // generated chunk + transition frame
+    const double window = m[0] - m[3];         // whole window minus the sink frames
+    // a head whose mass lies entirely on the sink frames counts as static
+    head_is_static[hd] = (window <= 0.0 || local * 1000.0 > (double)alpha_permille * window) ? 1 : 0;
+  }
+  return FK_OK;
+}
+
 int fk_abi_version(void) { return 1; }
 
 const char* fk_status_str(fk_status s) {

@@ -161,4 +161,18 @@ void launch_attention(int head_dim, const CUtensorMap& tmQ, const CUtensorMap& t
                       const CUtensorMap& tmV, const AttnArgs& a, cudaStream_t s);
 cudaError_t attention_prepare(int head_dim);   // sets the dynamic shared-memory limit
 
+// ------------------------------------------------------------------ head profiling (Eq. 1)
+struct ProfArgs {
+  int Nq, Nk, H, n_qtiles;
+  float scale_log2;             // log2(e) / sqrt(D)
+  int g_end;                    // keys [0, g_end): generated chunk
+  int s_end;                    // keys [g_end, s_end): sink frames
+  int t_begin;                  // keys [t_begin, Nk): transition frame; the rest: other history
+  double* mass;                 // [H][4]: rows, generated, transition, sink (added to)
+  int* status;
+};
+// tmQ / tmK: 3D maps over Q [Nq][H][D] and K [Nk][H][D] (128-row boxes, 128-byte swizzle)
+cudaError_t launch_head_profile(int head_dim, const CUtensorMap& tmQ, const CUtensorMap& tmK,
+                                const ProfArgs& a, cudaStream_t s);
+
 }  // namespace fk

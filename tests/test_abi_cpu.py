@@ -103,3 +103,41 @@ def test_null_handle_calls_are_rejected(lib):
     assert lib.fk_attend(None, 0, None, None, None) == 2
     assert lib.fk_cache_bytes(None) == 0
     lib.fk_destroy(None)
+
+
+def test_classify_heads_matches_oracle(lib):
+    import oracle as O
+    from paper_2605_09681_gb300 import classify_heads
+    rng = np.random.default_rng(7)
+    total = np.full(64, 100.0)
+    parts = rng.dirichlet([1, 1, 1, 1], size=64) * 100.0      # gen, trans, sink, other
+    mass = np.stack([total, parts[:, 0], parts[:, 1], parts[:, 2]], axis=1)
+    mass[0] = [10.0, 6.0, 2.0, 0.0]                              # exactly alpha
+    mass[1] = [10.0, 0.0, 0.0, 10.0]                             # all on the sinks
+    for alpha in (0.5, 0.8, 0.95):
+        got = classify_heads(mass, alpha)
+        ref = np.array([O.classify_head(m, alpha) for m in mass], dtype=np.uint8)
+        assert np.array_equal(got, ref)
+
+
+def test_head_profile_rejects_bad_arguments(lib):
+    # argument checks run on the host before any device query
+    buf = np.zeros(4096, dtype=np.float64)
+    p = buf.ctypes.data
+    ok = dict(n_queries=128, n_keys=256, n_heads=2, head_dim=128, n_generate=64, n_sink=32, n_transition=32)
+
+    def call(**kw):
+        a = dict(ok, **kw)
+        return lib.fk_head_profile(kw.get("Q", p), kw.get("K", p), a["n_queries"], a["n_keys"],
+                                   a["n_heads"], a["head_dim"], a["n_generate"], a["n_sink"],
+                                   a["n_transition"], kw.get("mass", p), kw.get("status", p), None)
+    from paper_2605_09681_gb300._lib import FK_ERR_ARG, FK_ERR_CONFIG
+    assert call(Q=None) == FK_ERR_ARG
+    assert call(mass=None) == FK_ERR_ARG
+    assert call(K=p + 8) == FK_ERR_ARG                            # not 16-byte aligned
+    assert call(head_dim=96) == FK_ERR_CONFIG
+    assert call(n_heads=0) == FK_ERR_CONFIG
+    assert call(n_keys=0) == FK_ERR_CONFIG
+    assert call(n_generate=200, n_sink=40, n_transition=40) == FK_ERR_CONFIG
+    assert call(n_sink=-1) == FK_ERR_CONFIG
+    assert call() == FK_ERR_ARG                                   # host pointers: not device memory

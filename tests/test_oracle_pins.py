@@ -360,3 +360,64 @@ def test_window_drops_old_frames():
     assert orc.nh[0] == 21 and r.window == tuple(range(9, 21)) and r.sink == (0,)
     assert sorted(orc.frames[0]) == [0] + list(range(9, 21))
     assert len(orc.kept(0, 1)) == 11 * 3
+
+
+# ---- offline head profiling (Sec. 4.1, Eq. 1)
+
+def _class_layout(n_gen, n_sink, n_other, n_trans, D, seed):
+    rng = np.random.default_rng(seed)
+    return rng.standard_normal((n_gen + n_sink + n_other + n_trans, D))
+
+
+def test_head_mass_uniform_attention_closed_form():
+    # q = 0: every logit is 0, each row spreads its unit mass evenly over the Nk keys, so each
+    # class receives rows * (class size) / Nk exactly
+    n_gen, n_sink, n_other, n_trans, D, nq = 30, 10, 45, 15, 16, 7
+    K = _class_layout(n_gen, n_sink, n_other, n_trans, D, 0)
+    nk = K.shape[0]
+    m = O.head_attention_mass(np.zeros((nq, D)), K, n_gen, n_sink, n_trans)
+    assert np.allclose(m, [nq, nq * n_gen / nk, nq * n_trans / nk, nq * n_sink / nk], rtol=0, atol=1e-12)
+
+
+def test_head_mass_two_key_values_closed_form():
+    # keys take two values: a on the generated chunk, b everywhere else; one query row q.
+    # The softmax is then n_gen e^{q.a/s} / Z on the chunk and e^{q.b/s} / Z on each other key.
+    D = 8
+    n_gen, n_sink, n_other, n_trans = 5, 3, 7, 4
+    a = np.linspace(-1, 1, D)
+    b = np.cos(np.arange(D))
+    q = np.sin(np.arange(D) * 0.7)
+    K = np.vstack([np.tile(a, (n_gen, 1)), np.tile(b, (n_sink + n_other + n_trans, 1))])
+    ea, eb = np.exp(q @ a / np.sqrt(D)), np.exp(q @ b / np.sqrt(D))
+    Z = n_gen * ea + (n_sink + n_other + n_trans) * eb
+    m = O.head_attention_mass(q[None], K, n_gen, n_sink, n_trans)
+    assert np.allclose(m, [1.0, n_gen * ea / Z, n_trans * eb / Z, n_sink * eb / Z], rtol=1e-13, atol=0)
+
+
+def test_head_mass_class_boundaries_and_permutations():
+    # shuffling keys inside a class leaves the masses unchanged; moving one key across a
+    # class boundary changes exactly the two classes involved
+    n_gen, n_sink, n_other, n_trans, D = 12, 6, 20, 6, 16
+    rng = np.random.default_rng(3)
+    K = _class_layout(n_gen, n_sink, n_other, n_trans, D, 1)
+    Q = rng.standard_normal((9, D)) * 2.0
+    m = O.head_attention_mass(Q, K, n_gen, n_sink, n_trans)
+    P = K.copy()
+    P[:n_gen] = P[rng.permutation(n_gen)]
+    P[n_gen + n_sink + n_other:] = P[n_gen + n_sink + n_other + rng.permutation(n_trans)]
+    assert np.allclose(O.head_attention_mass(Q, P, n_gen, n_sink, n_trans), m, rtol=1e-13, atol=1e-13)
+    m2 = O.head_attention_mass(Q, K, n_gen + 1, n_sink - 1, n_trans)   # key n_gen: sink -> generated
+    logits = Q @ K.T / np.sqrt(D)
+    p = np.exp(logits - logits.max(1, keepdims=True))
+    p /= p.sum(1, keepdims=True)
+    moved = p[:, n_gen].sum()
+    assert np.isclose(m2[1] - m[1], moved, rtol=1e-12) and np.isclose(m[3] - m2[3], moved, rtol=1e-12)
+    assert m2[0] == m[0] and m2[2] == m[2]
+
+
+def test_classify_head_threshold():
+    # Eq. 1 with alpha = 0.8: (gen + trans) / (total - sink)
+    assert O.classify_head([10.0, 6.0, 2.0, 1.0], 0.8)          # 8/9 = 0.889 > 0.8: static
+    assert not O.classify_head([10.0, 4.0, 2.0, 1.0], 0.8)      # 6/9 = 0.667: dynamic
+    assert not O.classify_head([10.0, 6.0, 2.0, 0.0], 0.8)      # exactly 0.8 is not above it
+    assert O.classify_head([10.0, 0.0, 0.0, 10.0], 0.8)         # all mass on the sinks

@@ -254,3 +254,30 @@ def test_480p_stack_full():
     # data and are attended and compared (the other layers replay layer 0's inputs)
     w = W.P480_STACK
     assert _stream(w, track_layers=(0, 13, 29), compare_every=3, step_filter=(0, 3)) > 0
+
+
+@pytest.mark.parametrize("head_dim,F,hist", [(128, 260, 8), (64, 100, 5)])
+def test_head_profile_matches_oracle(head_dim, F, hist):
+    # Eq. 1 masses from the tcgen05 profiling kernel vs the fp64 oracle on the same bf16
+    # inputs; 3-frame chunk, ragged query and key tiles, class boundaries inside key tiles.
+    # A second call adds to the same accumulator.
+    from paper_2605_09681_gb300 import classify_heads, head_profile
+    H = 8
+    q, k, (g, s, t) = W.profile_inputs(11 + head_dim, H, head_dim, F, 3, 1, hist)
+    Qd, Kd = to_dev(q), to_dev(k)
+    mass, status = head_profile(Qd, Kd, g, s, t)
+    torch.cuda.synchronize()
+    got = mass.cpu().numpy()
+    assert int(status.item()) == 0
+    Qf, Kf = W.bf16_bits_to_f32(q), W.bf16_bits_to_f32(k)
+    ref = np.stack([O.head_attention_mass(Qf[:, h], Kf[:, h], g, s, t) for h in range(H)])
+    nq = q.shape[0]
+    assert np.all(got[:, 0] == nq)
+    assert np.abs(got - ref).max() <= 1e-4 * nq, np.abs(got - ref).max()
+    ratio = (ref[:, 1] + ref[:, 2]) / (ref[:, 0] - ref[:, 3])
+    clear = np.abs(ratio - 0.8) > 1e-3
+    assert np.array_equal(classify_heads(got, 0.8)[clear],
+                          np.array([O.classify_head(m, 0.8) for m in ref], dtype=np.uint8)[clear])
+    head_profile(Qd, Kd, g, s, t, mass=mass, status=status)
+    torch.cuda.synchronize()
+    assert np.allclose(mass.cpu().numpy(), 2 * got, rtol=1e-12, atol=0)

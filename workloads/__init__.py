@@ -30,6 +30,7 @@ import numpy as np
 __all__ = [
     "Workload", "TINY", "TINY_PER_FRAME", "P480_LAYER", "P480_STACK", "ROLLING",
     "P1080_LAYER", "WORKLOADS", "normals", "uniforms", "to_bf16_bits", "bf16_bits_to_f32",
+    "profile_inputs",
     "head_map", "FrameStream", "snapshot_inputs", "queries", "step_kv", "stream_key",
 ]
 
@@ -90,6 +91,7 @@ def bf16_bits_to_f32(bits: np.ndarray) -> np.ndarray:
 
 # tensor-kind tags of the generator streams
 _K, _V, _Q, _SCALE, _MAP, _KSTEP, _VSTEP = 1, 2, 3, 4, 5, 6, 7
+_PK, _PQ, _PB, _PT = 11, 12, 13, 14   # head-profiling inputs
 
 
 @dataclass(frozen=True)
@@ -295,3 +297,25 @@ def step_kv(w: Workload, layer: int, chunk: int, step: int, clean_k: np.ndarray,
     k = bf16_bits_to_f32(clean_k).astype(np.float64) + a * ek
     v = bf16_bits_to_f32(clean_v).astype(np.float64) + a * ev
     return to_bf16_bits(k), to_bf16_bits(v)
+
+
+def profile_inputs(seed: int, n_heads: int, head_dim: int, tokens_per_frame: int,
+                   frames_per_chunk: int, n_sink_frames: int, n_history_frames: int):
+    """Seeded inputs of one offline head-profiling pass (one layer, one step).
+
+    Keys of the attention window, token-major [Nk, H, D], in the order [generated chunk (C
+    frames) | sink frames | other history | transition frame (the newest history frame)];
+    queries [C*F, H, D] of the generated chunk.  Head h's queries are beta_h times the
+    generated chunk's own keys plus unit noise (beta_h uniform in [0, 1.4)), and the
+    transition frame's keys are 0.7 x the chunk's last frame plus 0.7 x noise, so that the
+    heads range from attending locally to attending across the whole window.  Returns
+    (Q bits, K bits, (n_generate, n_sink, n_transition)) as bf16 bit patterns."""
+    F, C, S, H, D = tokens_per_frame, frames_per_chunk, n_sink_frames, n_heads, head_dim
+    assert n_history_frames > S
+    n_gen, n_sink, n_trans = C * F, S * F, F
+    nk = n_gen + (n_history_frames - 1) * F + n_trans
+    K = normals(stream_key(seed, _PK), nk * H * D).reshape(nk, H, D)
+    K[nk - F:] = 0.7 * K[n_gen - F:n_gen] + 0.7 * normals(stream_key(seed, _PT), F * H * D).reshape(F, H, D)
+    beta = 1.4 * uniforms(stream_key(seed, _PB), H)
+    Q = beta[None, :, None] * K[:n_gen] + normals(stream_key(seed, _PQ), n_gen * H * D).reshape(n_gen, H, D)
+    return to_bf16_bits(Q), to_bf16_bits(K), (n_gen, n_sink, n_trans)
