@@ -516,9 +516,9 @@ def run_stack(local_rank):
 # is reported only while that source is unchanged.
 NCU_TRAFFIC = {
     "480p_layer": {
-        "attend": ("fk_attn.cu", "a7947bb70908", 121476352),
-        "compact": ("fk_copy.cu", "cba7e7019a47", 75307264),
-        "score": ("fk_score.cu", "630b903cffb0", 43159552),
+        "attend": ("fk_attn.cu", "fc08b6769224", 122271744),
+        "compact": ("fk_copy.cu", "696e1eb5e98a", 76390912),
+        "score": ("fk_score.cu", "584831ae7a26", 43160320),
     },
 }
 
