@@ -224,5 +224,10 @@ class ForcingKVCache:
                                          ctypes.byref(n)), "fk_profile_read")
         return ms.value, n.value
 
+    def set_host_overlap(self, on: bool = True) -> None:
+        """Copy host inputs on the handle's copy stream as soon as a call is made (see
+        fk_set_host_overlap): the caller promises host inputs are final at call time."""
+        _check(self._lib.fk_set_host_overlap(self._h, 1 if on else 0), "fk_set_host_overlap")
+
     def launch_count(self) -> int:
         return int(self._lib.fk_launch_count(self._h))

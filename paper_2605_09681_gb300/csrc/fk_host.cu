@@ -59,6 +59,12 @@ struct LayerState {
   int sinks_done = 0;     // sink frames already in the dynamic views
 };
 
+struct Staging {
+  bf16* buf[2][2] = {};           // [slot][tensor]
+  cudaEvent_t ready[2] = {}, freed[2] = {};
+  int slot = 0;                   // next slot to fill
+};
+
 struct ProfRec {
   int kind;
   cudaEvent_t a, b;
@@ -102,11 +108,13 @@ struct fk_handle {
   int* kept = nullptr;
   unsigned long long* sums = nullptr;
   int* status = nullptr;
-  bf16* stage_q = nullptr;
+  // host-input staging: two slots per kind (K with V; Q), each with a ready event (copy done)
+  // and a freed event (the kernel that read the slot has run); optional copy stream
+  Staging st_kv, st_q;
   bf16* stage_o = nullptr;
-  bf16* stage_k = nullptr;
-  bf16* stage_v = nullptr;
   int64_t stage_frames = 0;        // frames one K/V staging buffer holds
+  cudaStream_t copy_stream = nullptr;
+  bool host_overlap = false;
   ScoreItem* d_score_items = nullptr;
   SelectTarget* d_targets = nullptr;
   CompactItem* d_compact_items = nullptr;
@@ -118,8 +126,9 @@ struct fk_handle {
   int max_run = 0;
   int score_ctas = 0;
   CUtensorMap tmK{}, tmV{};
-  const void* q_cached = nullptr;
-  CUtensorMap tmQ{};
+  const void* q_cached[2] = {};   // two cached Q maps (the two Q staging slots alternate)
+  CUtensorMap tmQ[2]{};
+  int q_next = 0;
   // profiling
   bool prof = false;
   std::vector<ProfRec> prof_pending;
@@ -247,15 +256,37 @@ fk_status dev_alloc(fk_handle* h, size_t bytes, void** out) {
   return FK_OK;
 }
 
-// Copy host input [rows][H][D] into staging when needed; returns the device pointer to use.
-fk_status stage_input(fk_handle* h, const void* src, bf16* stage, size_t bytes, cudaStream_t s,
-                      const bf16** out) {
-  if (is_device_ptr(src)) {
-    *out = static_cast<const bf16*>(src);
-    return FK_OK;
+// Host inputs [rows][H][D] (up to two of `bytes` each) into the next staging slot of `sg`;
+// device inputs pass through.  *slot is the slot used, -1 when nothing was staged; the caller
+// records sg.freed[*slot] on `s` after the kernel that reads it.  By default the copies run on
+// `s` in call order; with host overlap on, they run at once on the copy stream (after the
+// slot's previous reader) and `s` waits for them before the reader.
+fk_status stage_inputs(fk_handle* h, Staging& sg, const void* a, const void* b, size_t bytes,
+                       cudaStream_t s, const bf16** oa, const bf16** ob, int* slot) {
+  const void* src[2] = {a, b};
+  const bf16** out[2] = {oa, ob};
+  bool host[2] = {false, false};
+  for (int i = 0; i < 2; ++i) {
+    if (!src[i]) continue;
+    host[i] = !is_device_ptr(src[i]);
+    if (!host[i]) *out[i] = static_cast<const bf16*>(src[i]);
   }
-  FK_CUDA(cudaMemcpyAsync(stage, src, bytes, cudaMemcpyHostToDevice, s));
-  *out = stage;
+  *slot = -1;
+  if (!host[0] && !host[1]) return FK_OK;
+  const int sl = sg.slot;
+  sg.slot ^= 1;
+  cudaStream_t cs = h->host_overlap ? h->copy_stream : s;
+  if (h->host_overlap) FK_CUDA(cudaStreamWaitEvent(cs, sg.freed[sl], 0));
+  for (int i = 0; i < 2; ++i) {
+    if (!host[i]) continue;
+    FK_CUDA(cudaMemcpyAsync(sg.buf[sl][i], src[i], bytes, cudaMemcpyHostToDevice, cs));
+    *out[i] = sg.buf[sl][i];
+  }
+  if (h->host_overlap) {
+    FK_CUDA(cudaEventRecord(sg.ready[sl], cs));
+    FK_CUDA(cudaStreamWaitEvent(s, sg.ready[sl], 0));
+  }
+  *slot = sl;
   return FK_OK;
 }
 
@@ -340,11 +371,10 @@ fk_status update_current(fk_handle* h, int layer, bool retire, const void* K, co
   retire = retire && ls.has_current;
   if (retire && h->W == 0 && ls.nh + h->C > h->max_hist) return FK_ERR_FULL;
   const bf16 *k = nullptr, *v = nullptr;
+  int slot = -1;
   if (K) {
     const size_t bytes = (size_t)h->CF * h->H * h->D * 2;
-    fk_status st = stage_input(h, K, h->stage_k, bytes, s, &k);
-    if (st != FK_OK) return st;
-    st = stage_input(h, V, h->stage_v, bytes, s, &v);
+    fk_status st = stage_inputs(h, h->st_kv, K, V, bytes, s, &k, &v, &slot);
     if (st != FK_OK) return st;
   }
   if (!retire && !k) return FK_OK;
@@ -370,6 +400,7 @@ fk_status update_current(fk_handle* h, int layer, bool retire, const void* K, co
   }
   fk_status st = launch(h, s, FK_KERNEL_APPEND, [&] { launch_current(a, s); });
   if (st != FK_OK) return st;
+  if (slot >= 0) FK_CUDA(cudaEventRecord(h->st_kv.freed[slot], s));
   if (retire) {
     ls.nh += h->C;
     ls.dirty = true;
@@ -431,6 +462,12 @@ fk_status fk_classify_heads(const double* mass, int n_heads, int alpha_permille,
     // a head whose mass lies entirely on the sink frames counts as static
     head_is_static[hd] = (window <= 0.0 || local * 1000.0 > (double)alpha_permille * window) ? 1 : 0;
   }
+  return FK_OK;
+}
+
+fk_status fk_set_host_overlap(fk_handle* h, int on) {
+  if (!h) return FK_ERR_ARG;
+  h->host_overlap = on != 0;
   return FK_OK;
 }
 
@@ -600,15 +637,28 @@ fk_status fk_create(const fk_config* cfg, fk_handle** out) {
   if ((st = dev_alloc(h, 256, &p)) != FK_OK) return fail(st);
   h->status = static_cast<int*>(p);
   const size_t chunk_bytes = (size_t)h->CF * h->H * h->D * 2;
-  if ((st = dev_alloc(h, chunk_bytes, &p)) != FK_OK) return fail(st);
-  h->stage_q = static_cast<bf16*>(p);
+  for (int sl = 0; sl < 2; ++sl) {
+    for (int i = 0; i < 2; ++i) {
+      if ((st = dev_alloc(h, chunk_bytes, &p)) != FK_OK) return fail(st);
+      h->st_kv.buf[sl][i] = static_cast<bf16*>(p);
+    }
+    if ((st = dev_alloc(h, chunk_bytes, &p)) != FK_OK) return fail(st);
+    h->st_q.buf[sl][0] = static_cast<bf16*>(p);
+  }
   if ((st = dev_alloc(h, chunk_bytes, &p)) != FK_OK) return fail(st);
   h->stage_o = static_cast<bf16*>(p);
-  if ((st = dev_alloc(h, chunk_bytes, &p)) != FK_OK) return fail(st);
-  h->stage_k = static_cast<bf16*>(p);
-  if ((st = dev_alloc(h, chunk_bytes, &p)) != FK_OK) return fail(st);
-  h->stage_v = static_cast<bf16*>(p);
   h->stage_frames = h->C;
+  for (Staging* sg : {&h->st_kv, &h->st_q})
+    for (int sl = 0; sl < 2; ++sl)
+      if (cudaEventCreateWithFlags(&sg->ready[sl], cudaEventDisableTiming) != cudaSuccess ||
+          cudaEventCreateWithFlags(&sg->freed[sl], cudaEventDisableTiming) != cudaSuccess) {
+        cudaGetLastError();
+        return fail(FK_ERR_CUDA);
+      }
+  if (cudaStreamCreateWithFlags(&h->copy_stream, cudaStreamNonBlocking) != cudaSuccess) {
+    cudaGetLastError();
+    return fail(FK_ERR_CUDA);
+  }
 
   // static device tables
   if (h->source == FK_SCORE_LAYER0_POOLED) {
@@ -660,6 +710,12 @@ void fk_destroy(fk_handle* h) {
     cudaEventDestroy(r.b);
   }
   for (auto e : h->ev_free) cudaEventDestroy(e);
+  for (Staging* sg : {&h->st_kv, &h->st_q})
+    for (int sl = 0; sl < 2; ++sl) {
+      if (sg->ready[sl]) cudaEventDestroy(sg->ready[sl]);
+      if (sg->freed[sl]) cudaEventDestroy(sg->freed[sl]);
+    }
+  if (h->copy_stream) cudaStreamDestroy(h->copy_stream);
   for (void* p : h->allocs) cudaFree(p);
   cudaGetLastError();
   delete h;
@@ -689,15 +745,17 @@ fk_status fk_append_frames(fk_handle* h, int layer, const void* K, const void* V
     const int nf = dev_in ? n_frames : (int)std::min<int64_t>(h->stage_frames, n_frames - f0);
     const bf16* k = static_cast<const bf16*>(K) + (size_t)f0 * frame_bytes / 2;
     const bf16* v = static_cast<const bf16*>(V) + (size_t)f0 * frame_bytes / 2;
-    if (!dev_in) {
-      FK_CUDA(cudaMemcpyAsync(h->stage_k, k, nf * frame_bytes, cudaMemcpyHostToDevice, s));
-      FK_CUDA(cudaMemcpyAsync(h->stage_v, v, nf * frame_bytes, cudaMemcpyHostToDevice, s));
-      k = h->stage_k;
-      v = h->stage_v;
+    if (!dev_in) {   // staging slot 0, in order on `s` (see the freed events below)
+      FK_CUDA(cudaMemcpyAsync(h->st_kv.buf[0][0], k, nf * frame_bytes, cudaMemcpyHostToDevice, s));
+      FK_CUDA(cudaMemcpyAsync(h->st_kv.buf[0][1], v, nf * frame_bytes, cudaMemcpyHostToDevice, s));
+      k = h->st_kv.buf[0][0];
+      v = h->st_kv.buf[0][1];
     }
     if ((st = push_history(h, layer, k, v, nf, s)) != FK_OK) return st;
     f0 += nf;
   }
+  if (n_frames > 0 && !dev_in)   // later overlapped copies into either slot wait for this use
+    for (int sl = 0; sl < 2; ++sl) FK_CUDA(cudaEventRecord(h->st_kv.freed[sl], s));
   ls.dirty = true;
   return FK_OK;
 }
@@ -866,13 +924,19 @@ fk_status fk_attend(fk_handle* h, int layer, const void* Q, void* O, void* strea
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   FK_CUDA(cudaSetDevice(h->dev));
   const size_t bytes = (size_t)h->CF * h->H * h->D * 2;
-  const bf16* q;
-  if ((st = stage_input(h, Q, h->stage_q, bytes, s, &q)) != FK_OK) return st;
-  const bool dev_out = is_device_ptr(O);
-  bf16* o = dev_out ? static_cast<bf16*>(O) : h->stage_o;
-  if (q != h->q_cached) {
-    if ((st = encode_q(&h->tmQ, q, h->CF, h->H, h->D)) != FK_OK) return st;
-    h->q_cached = q;
+  const bf16* q = nullptr;
+  int slot = -1;
+  if ((st = stage_inputs(h, h->st_q, Q, nullptr, bytes, s, &q, nullptr, &slot)) != FK_OK) return st;
+  // a host output is staged and copied back on `stream` (measured faster than storing it
+  // from the attention epilogue directly into pinned host memory)
+  const bool copy_back = !is_device_ptr(O);
+  bf16* o = copy_back ? h->stage_o : static_cast<bf16*>(O);
+  int qm = q == h->q_cached[0] ? 0 : q == h->q_cached[1] ? 1 : -1;
+  if (qm < 0) {
+    qm = h->q_next;
+    h->q_next ^= 1;
+    if ((st = encode_q(&h->tmQ[qm], q, h->CF, h->H, h->D)) != FK_OK) return st;
+    h->q_cached[qm] = q;
   }
   AttnArgs a{};
   a.O = o;
@@ -893,9 +957,10 @@ fk_status fk_attend(fk_handle* h, int layer, const void* Q, void* O, void* strea
   for (int i = 0; i < h->H; ++i) a.head_of[i] = order[i];
   const int D = h->D;
   if ((st = launch(h, s, FK_KERNEL_ATTEND,
-                   [&] { launch_attention(D, h->tmQ, h->tmK, h->tmV, a, s); })) != FK_OK)
+                   [&] { launch_attention(D, h->tmQ[qm], h->tmK, h->tmV, a, s); })) != FK_OK)
     return st;
-  if (!dev_out) FK_CUDA(cudaMemcpyAsync(O, o, bytes, cudaMemcpyDeviceToHost, s));
+  if (slot >= 0) FK_CUDA(cudaEventRecord(h->st_q.freed[slot], s));
+  if (copy_back) FK_CUDA(cudaMemcpyAsync(O, o, bytes, cudaMemcpyDeviceToHost, s));
   return FK_OK;
 }
 

@@ -281,3 +281,51 @@ def test_head_profile_matches_oracle(head_dim, F, hist):
     head_profile(Qd, Kd, g, s, t, mass=mass, status=status)
     torch.cuda.synchronize()
     assert np.allclose(mass.cpu().numpy(), 2 * got, rtol=1e-12, atol=0)
+
+
+def test_host_inputs_and_overlap_match_device_inputs():
+    # the same stream driven with device tensors; with pageable host arrays (inputs copied
+    # in call order, output copied back); and with pinned host tensors and host-input overlap
+    # on (inputs copied on the handle's copy stream into two alternating staging slots).  The
+    # overlap run issues every step
+    # before one final synchronize, so copies into a slot really race the kernels still
+    # reading the other slot.  All three produce bit-identical outputs.
+    from paper_2605_09681_gb300 import ForcingKVCache
+    w = W.ROLLING.with_(name="ovl", head_dim=64, tokens_per_frame=120, n_heads=4, window_frames=6,
+                        n_chunks=7)
+    hm = W.head_map(w)
+    pin = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16).pin_memory()
+    runs = {}
+    for mode in ("device", "host", "overlap"):
+        fs = W.FrameStream(w, 0)
+        keep, outs = [], []
+        with ForcingKVCache.from_workload(w, hm) as cache:
+            cache.set_host_overlap(mode == "overlap")
+            for c in range(w.n_chunks):
+                k, v = fs.frames(w.frames_per_chunk)
+                q = W.queries(w, 0, c, 0)
+                if mode == "device":
+                    cache.append_chunk(0, to_dev(k), to_dev(v))
+                    cache.compress()
+                    outs.append(cache.attend(0, to_dev(q)))
+                else:
+                    if mode == "host":
+                        K, V, Q = (np.ascontiguousarray(x) for x in (k, v, q))
+                        Oh = np.zeros(q.shape, dtype=np.uint16)
+                    else:
+                        K, V, Q = pin(k), pin(v), pin(q)
+                        Oh = torch.empty(Q.shape, dtype=torch.bfloat16).pin_memory()
+                    keep += [K, V, Q]
+                    cache.append_chunk(0, K, V)
+                    cache.compress()
+                    cache.set_current(0, K, V)
+                    cache.attend(0, Q, Oh)
+                    outs.append(Oh)
+                    if mode == "host":
+                        torch.cuda.synchronize()
+            torch.cuda.synchronize()
+            assert cache.sync_status() == 0
+            runs[mode] = [W.bf16_bits_to_f32(o) if isinstance(o, np.ndarray) else o.float().cpu().numpy()
+                          for o in outs]
+    for a, b, c in zip(runs["device"], runs["host"], runs["overlap"]):
+        assert np.array_equal(a, b) and np.array_equal(a, c)
