@@ -53,8 +53,10 @@ def _workload(name: str):
     w = W.WORKLOADS[name]
     if w.schedule != "snapshot":
         raise SystemExit("bench workloads are the single-layer cases: 480p_layer, 1080p_layer, tiny")
-    # stream chunks through a window holding exactly the snapshot's history
-    return w.with_(window_frames=max(1, w.n_history_frames - w.n_sink_frames), incremental=False)
+    # stream chunks through a window holding exactly the snapshot's history (a workload with
+    # its own window, such as the comparison rules, keeps it)
+    window = w.window_frames or max(1, w.n_history_frames - w.n_sink_frames)
+    return w.with_(window_frames=window, incremental=False)
 
 
 def _algorithmic(w, key_counts):
@@ -72,8 +74,10 @@ def _algorithmic(w, key_counts):
     n_scoreable = (nh - 1 - lo) if has_anchor else 0
     static = _workload_static(w)
     n_dyn = sum(1 for st in static if not st)
-    score_bytes = n_dyn * (n_scoreable + 1 if n_scoreable else 0) * F * D * 2
-    n_keep = n_scoreable * (w.keep_budget_permille * w.n_segments // 1000)
+    scored = w.selection == "similarity"                 # comparison rules skip scoring
+    score_bytes = n_dyn * (n_scoreable + 1 if n_scoreable else 0) * F * D * 2 if scored else 0
+    k_frame = w.n_segments if w.selection == "all" else w.keep_budget_permille * w.n_segments // 1000
+    n_keep = n_scoreable * k_frame
     unit_tokens = n_sink * F + n_keep * (F // w.n_segments) + (F if has_anchor else 0)
     compact_bytes = n_dyn * 2 * 2 * unit_tokens * D * 2
     append_bytes = 2 * 2 * nq * H * D * 2 + sum(
@@ -282,7 +286,7 @@ def run_fk(args, rank, world, local_rank):
     attn_tflops = alg["attn_flops"] / (attn_ms * 1e-3) / 1e12
     compact_ms, score_ms = per_launch("compact"), per_launch("score")
     compact_gbs = alg["compact_bytes"] / (compact_ms * 1e-3) / 1e9
-    score_gbs = alg["score_bytes"] / (score_ms * 1e-3) / 1e9
+    score_gbs = alg["score_bytes"] / (score_ms * 1e-3) / 1e9 if prof["score"][1] else None
     append_ms = prof["append"][0] / max(1, prof["append"][1])
     append_total = prof["append"][0] / args.steps
     compress_ms = (prof["score"][0] + prof["select"][0] + prof["compact"][0]) / args.steps
@@ -309,7 +313,8 @@ def run_fk(args, rank, world, local_rank):
             "queries": w.n_queries, "sink_frames": w.n_sink_frames,
             "history_frames": w.n_history_frames - w.n_sink_frames,
             "segments": w.n_segments, "keep_budget": w.keep_budget_permille / 1000,
-            "keys_per_head": keys, "rescore": "whole window every step",
+            "keys_per_head": keys, "selection": w.selection,
+            "rescore": "whole window every step" if w.selection == "similarity" else "no scoring (comparison rule)",
             "l2": "flushed between timed steps (512 MiB write outside the step events)",
             "parallelism": "replicas" if world > 1 else "single GPU",
         },
@@ -329,9 +334,10 @@ def run_fk(args, rank, world, local_rank):
             "compact": {"achieved": round(compact_gbs, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
                         "frac": round(compact_gbs / peaks["hbm_gbs"], 4), "bytes": alg["compact_bytes"],
                         "us": round(compact_ms * 1e3, 2), "traffic": traffic.get("compact")},
-            "score": {"achieved": round(score_gbs, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
-                      "frac": round(score_gbs / peaks["hbm_gbs"], 4), "bytes": alg["score_bytes"],
-                      "us": round(score_ms * 1e3, 2), "traffic": traffic.get("score")},
+            "score": ({"achieved": round(score_gbs, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                       "frac": round(score_gbs / peaks["hbm_gbs"], 4), "bytes": alg["score_bytes"],
+                       "us": round(score_ms * 1e3, 2), "traffic": traffic.get("score")}
+                      if score_gbs is not None else None),
             "peak_source": peaks["source"] + " HBM copy bandwidth",
         },
         "kernels_us_per_step": {k: round(prof[k][0] / args.steps * 1e3, 2) for k in prof},
@@ -408,6 +414,8 @@ def run_incremental(args, w, hm, local_rank, hk, hv, dK, dV, dQ, dO, flush, stre
 
     def kern(kind, nbytes):
         ms, n = prof[kind]
+        if not n:
+            return None
         us = ms / n * 1e3
         gbs = nbytes / (us * 1e-6) / 1e9
         return {"bytes": nbytes, "us": round(us, 2), "achieved": round(gbs, 1), "unit": "GB/s",

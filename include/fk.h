@@ -77,6 +77,21 @@ enum {
                                  Sec. 4.3); one kept set is shared by all dynamic heads     */
 };
 
+/* Which segments of a scoreable frame dynamic heads keep.  SIMILARITY is the method (Eq. 3);
+ * the others are the paper's comparison rules, run through the same selection, compaction
+ * and attention for speed comparisons (App. H and Sec. 5.3): ALL keeps every segment (with
+ * n_sink_frames = 3 and window_frames = 4 on all-dynamic heads: the frame-level StreamingLLM
+ * baseline; on neighbour heads with window_frames = L: Dummy Forcing), UNIFORM keeps the k
+ * segments j = floor(i n / k), i < k (with n_segments = tokens_per_frame: uniform token
+ * pruning), RANDOM keeps the k segments with the smallest seeded SplitMix64 values (random
+ * token pruning).  k = floor(b n) as for SIMILARITY (n for ALL). */
+enum {
+  FK_SELECT_SIMILARITY = 0,
+  FK_SELECT_ALL = 1,
+  FK_SELECT_UNIFORM = 2,        /* per-frame scope only */
+  FK_SELECT_RANDOM = 3
+};
+
 typedef struct fk_config {
   int32_t n_layers;             /* 1..256                                                  */
   int32_t n_heads;              /* 1..128                                                  */
@@ -97,6 +112,10 @@ typedef struct fk_config {
   int32_t device;               /* CUDA device ordinal                                     */
   const uint8_t* head_is_static;/* host [n_layers*n_heads]: 1 = static head, 0 = dynamic;
                                    copied by fk_create                                     */
+  int32_t selection;            /* FK_SELECT_* (0 = the method)                            */
+  uint32_t select_seed;         /* seed of FK_SELECT_RANDOM                                */
+  int32_t static_drop_anchor;   /* 1: static heads keep sink + current chunk only (Dummy
+                                   Forcing's local heads); 0: sink + anchor + current (Eq. 2) */
 } fk_config;
 
 typedef struct fk_handle fk_handle;
@@ -242,7 +261,8 @@ FK_API fk_status fk_classify_heads(const double* mass, int n_heads, int alpha_pe
 /* Static text for a status code. */
 FK_API const char* fk_status_str(fk_status s);
 
-/* ABI version of this header: 1. */
+/* ABI version of this header: 2 (fk_config gained selection, select_seed and
+ * static_drop_anchor after head_is_static). */
 FK_API int fk_abi_version(void);
 
 #ifdef __cplusplus

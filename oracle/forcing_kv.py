@@ -176,12 +176,13 @@ def frame_tokens(frame: int, F: int) -> list:
     return list(range(frame * F, (frame + 1) * F))
 
 
-def static_key_tokens(roles: FrameRoles, F: int, current_frames) -> list:
-    """Eq. 2: [sink frames, transition-anchor frame, current chunk] as global key ids."""
+def static_key_tokens(roles: FrameRoles, F: int, current_frames, keep_anchor: bool = True) -> list:
+    """Eq. 2: [sink frames, transition-anchor frame, current chunk] as global key ids
+    (keep_anchor=False: sink and current chunk only, Dummy Forcing's local heads)."""
     ids = []
     for f in roles.sink:
         ids += frame_tokens(f, F)
-    if roles.anchor is not None:
+    if roles.anchor is not None and keep_anchor:
         ids += frame_tokens(roles.anchor, F)
     for f in current_frames:
         ids += frame_tokens(f, F)
@@ -224,6 +225,35 @@ def attention_fp64(Q: np.ndarray, K: np.ndarray, V: np.ndarray, row_block: int =
         p = np.exp(logits)
         out[r0:r0 + row_block] = (p @ V) / p.sum(axis=1, keepdims=True)
     return out
+
+
+# --------------------------------------------------------------------------------------
+# comparison selection rules (App. H, Sec. 5.3): ranking values replacing the scores
+# --------------------------------------------------------------------------------------
+_M64 = (1 << 64) - 1
+
+
+def splitmix64(z: int) -> int:
+    """SplitMix64 (Steele, Lea and Flood, 2014): the finaliser applied to z + golden gamma."""
+    z = (z + 0x9E3779B97F4A7C15) & _M64
+    z = ((z ^ (z >> 30)) * 0xBF58476D1CE4E5B9) & _M64
+    z = ((z ^ (z >> 27)) * 0x94D049BB133111EB) & _M64
+    return z ^ (z >> 31)
+
+
+def rule_value(rule: str, seed: int, t: int, j: int, n: int, k: int) -> float:
+    """Value of segment j of frame t under a comparison rule; BottomK keeps the smallest.
+    all: 0 everywhere (k = n keeps every segment); uniform: 0 on the k evenly spaced segments
+    {floor(i n / k) : i < k}, else 1; random: the top 24 bits of
+    SplitMix64(seed * 2^40 xor t * 2^20 xor j) as a fraction of 2^24."""
+    if rule == "all":
+        return 0.0
+    if rule == "uniform":
+        return 0.0 if k > 0 and j in {i * n // k for i in range(k)} else 1.0
+    if rule == "random":
+        key = ((seed << 40) ^ (t << 20) ^ j) & _M64
+        return (splitmix64(key) >> 40) / 16777216.0
+    raise ValueError(rule)
 
 
 # --------------------------------------------------------------------------------------
@@ -286,7 +316,8 @@ class ForcingKVOracle:
     def __init__(self, *, n_layers, n_heads, head_dim, tokens_per_frame, frames_per_chunk,
                  n_sink_frames, window_frames, n_segments, keep_budget_permille,
                  select_scope="per_frame", score_source="per_head", head_is_static,
-                 track_layers=None):
+                 track_layers=None, selection="similarity", select_seed=0,
+                 static_drop_anchor=False):
         self.L, self.H, self.D = n_layers, n_heads, head_dim
         self.F, self.C = tokens_per_frame, frames_per_chunk
         self.S, self.W = n_sink_frames, window_frames
@@ -298,6 +329,10 @@ class ForcingKVOracle:
         if score_source not in ("per_head", "layer0_pooled"):
             raise ValueError(score_source)
         self.scope, self.source = select_scope, score_source
+        if selection not in ("similarity", "all", "uniform", "random"):
+            raise ValueError(selection)
+        self.selection, self.seed = selection, int(select_seed) & 0xFFFFFFFF
+        self.keep_anchor_static = not static_drop_anchor
         self.static = np.asarray(head_is_static, dtype=np.uint8).reshape(n_layers, n_heads)
         self.layers = list(range(n_layers)) if track_layers is None else sorted(track_layers)
         if score_source == "layer0_pooled" and 0 not in self.layers:
@@ -314,7 +349,9 @@ class ForcingKVOracle:
                    n_sink_frames=w.n_sink_frames, window_frames=w.window_frames,
                    n_segments=w.n_segments, keep_budget_permille=w.keep_budget_permille,
                    select_scope=w.select_scope, score_source=w.score_source,
-                   head_is_static=head_is_static, track_layers=track_layers)
+                   head_is_static=head_is_static, track_layers=track_layers,
+                   selection=w.selection, select_seed=w.select_seed,
+                   static_drop_anchor=w.static_drop_anchor)
 
     def _push_history(self, layer, K, V):
         F = self.F
@@ -365,11 +402,21 @@ class ForcingKVOracle:
             return 0, None
         return layer, head
 
+    def _k_frame(self) -> int:
+        return self.n if self.selection == "all" else keep_count(self.b, self.n)
+
     def scores(self, layer, head, exact: bool = False) -> dict:
         """Eq. 3 scores {t: [s_t^(0..n-1)]} over the scoreable frames; contract fp32 by
-        default, fp64 definition with exact=True."""
+        default, fp64 definition with exact=True.  Under a comparison rule: the rule's
+        ranking values instead."""
         sl, sh = self._score_layer_head(layer, head)
         out = {}
+        if self.selection != "similarity":
+            k = self._k_frame()
+            for t in self.roles(sl).scoreable:
+                out[t] = np.array([rule_value(self.selection, self.seed, t, j, self.n, k)
+                                   for j in range(self.n)], dtype=np.float32)
+            return out
         for t in self.roles(sl).scoreable:
             row = []
             for j in range(self.n):
@@ -384,7 +431,7 @@ class ForcingKVOracle:
             return []
         sc = self.scores(layer, head, exact=exact)
         if self.scope == "per_frame":
-            k = keep_count(self.b, self.n)
+            k = self._k_frame()
             ids = []
             for t, row in sc.items():
                 ids += [t * self.n + j for j in bottom_k(row, range(self.n), k)]
@@ -394,7 +441,8 @@ class ForcingKVOracle:
             for j in range(self.n):
                 cand_s.append(row[j])
                 cand_i.append(t * self.n + j)
-        return bottom_k(cand_s, cand_i, keep_count(self.b, len(cand_i)))
+        n_keep = len(cand_i) if self.selection == "all" else keep_count(self.b, len(cand_i))
+        return bottom_k(cand_s, cand_i, n_keep)
 
     # ---- Eq. 2 / Eq. 4 key sets and attention ----
     def current_frames(self, layer):
@@ -405,7 +453,7 @@ class ForcingKVOracle:
         roles = self.roles(layer)
         cur = self.current_frames(layer)
         if self.static[layer, head]:
-            return static_key_tokens(roles, self.F, cur)
+            return static_key_tokens(roles, self.F, cur, self.keep_anchor_static)
         if kept is None:
             kept = self.kept(layer, head)
         return dynamic_key_tokens(roles, self.F, self.n, kept, cur)

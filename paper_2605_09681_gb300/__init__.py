@@ -100,7 +100,8 @@ class ForcingKVCache:
     def __init__(self, *, n_layers, n_heads, head_dim, tokens_per_frame, frames_per_chunk,
                  n_sink_frames, window_frames, n_segments, keep_budget_permille,
                  head_is_static, select_scope="per_frame", score_source="per_head",
-                 incremental=False, max_history_frames=64, device=0):
+                 incremental=False, max_history_frames=64, device=0, selection="similarity",
+                 select_seed=0, static_drop_anchor=False):
         self._lib = L.load()
         self._h = ctypes.c_void_p()
         hm = np.ascontiguousarray(np.asarray(head_is_static, dtype=np.uint8).reshape(-1))
@@ -113,7 +114,8 @@ class ForcingKVCache:
             {"per_frame": L.FK_SCOPE_PER_FRAME, "pooled": L.FK_SCOPE_POOLED}[select_scope],
             {"per_head": L.FK_SCORE_PER_HEAD, "layer0_pooled": L.FK_SCORE_LAYER0_POOLED}[score_source],
             1 if incremental else 0, max_history_frames, device,
-            hm.ctypes.data_as(ctypes.POINTER(ctypes.c_uint8)))
+            hm.ctypes.data_as(ctypes.POINTER(ctypes.c_uint8)),
+            L.FK_SELECT[selection], select_seed & 0xFFFFFFFF, 1 if static_drop_anchor else 0)
         self.n_layers, self.n_heads, self.head_dim = n_layers, n_heads, head_dim
         self.F, self.C, self.n_segments = tokens_per_frame, frames_per_chunk, n_segments
         self.device = device
@@ -127,7 +129,9 @@ class ForcingKVCache:
                   n_segments=w.n_segments, keep_budget_permille=w.keep_budget_permille,
                   head_is_static=head_is_static, select_scope=w.select_scope,
                   score_source=w.score_source, incremental=w.incremental,
-                  max_history_frames=max(1, w.max_history_frames()), device=device)
+                  max_history_frames=max(1, w.max_history_frames()), device=device,
+                  selection=w.selection, select_seed=w.select_seed,
+                  static_drop_anchor=w.static_drop_anchor)
         kw.update(over)
         return cls(**kw)
 

@@ -15,6 +15,7 @@ STATUS_NAMES = {0: "FK_OK", 1: "FK_ERR_CONFIG", 2: "FK_ERR_ARG", 3: "FK_ERR_STAT
                 8: "FK_ERR_NOMEM"}
 FK_SCOPE_PER_FRAME, FK_SCOPE_POOLED = 0, 1
 FK_SCORE_PER_HEAD, FK_SCORE_LAYER0_POOLED = 0, 1
+FK_SELECT = {"similarity": 0, "all": 1, "uniform": 2, "random": 3}
 KERNEL_KINDS = {"append": 0, "score": 1, "select": 2, "compact": 3, "attend": 4}
 
 EXPORTS = [
@@ -35,6 +36,8 @@ class FkConfig(ctypes.Structure):
         ("select_scope", ctypes.c_int32), ("score_source", ctypes.c_int32),
         ("incremental", ctypes.c_int32), ("max_history_frames", ctypes.c_int32),
         ("device", ctypes.c_int32), ("head_is_static", ctypes.POINTER(ctypes.c_uint8)),
+        ("selection", ctypes.c_int32), ("select_seed", ctypes.c_uint32),
+        ("static_drop_anchor", ctypes.c_int32),
     ]
 
 

@@ -60,8 +60,10 @@ __global__ void __launch_bounds__(256) current_kernel(const CurrentArgs a) {
       const int f = a.nh_old + row / a.F;
       const int p = row - (row / a.F) * a.F;
       const bool sink = f < a.S;
-      to_page = a.pageK[h] != nullptr && (sink || f >= lo_new);   // frames replaced within
-      to_slot = a.is_static[h] && (sink || f == nh_new - 1);      // the retire are skipped
+      // frames replaced within the retire are skipped; static views hold the sinks and
+      // (unless they drop it) the new anchor frame
+      to_page = a.pageK[h] != nullptr && (sink || f >= lo_new);
+      to_slot = a.is_static[h] && (sink || (a.static_anchor && f == nh_new - 1));
       po = ((int64_t)ring_slot(f, a.S, a.cap_nonsink) * a.F + p) * a.head_dim + c * 8;
       so = ((int64_t)a.rows + (int64_t)(sink ? f : a.S) * a.F + p) * a.head_dim + c * 8;
     }
@@ -107,22 +109,17 @@ __global__ void __launch_bounds__(256) scatter_kernel(const ScatterArgs a) {
   }
 }
 
-// One CTA copies one piece (<= 16 KB of keys and 16 KB of values) of one unit of one
-// dynamic head's view.  Units in order: the sink frames to copy (n units each), the anchor
-// frame (n units), the kept segments to copy (one unit each, taken from the target's kept
+// Source and destination element offsets of unit u of a dynamic head's compaction; false
+// when u is past the layer's units.  Units in order: the sink frames to copy (n units each),
+// the anchor frame (n units), the kept segments to copy (one unit each, from the target's kept
 // list).  View rows after the current chunk: sink frame f at S-slot f, the anchor after the
 // sinks, kept segment i in ring slot (rp0 + i) mod kmax after the anchor.
-__global__ void __launch_bounds__(256) compact_kernel(const CompactArgs a) {
-  pdl_trigger();
-  pdl_wait();      // kept lists and pages come from the kernels before this one
-  const CompactItem it = a.items[blockIdx.y];
+__device__ __forceinline__ bool unit_offsets(const CompactArgs& a, const CompactItem& it, int u,
+                                             int64_t& src_off, int64_t& dst_off) {
   const int l = it.layer;
-  if (!a.active[l]) return;
-  const int u = blockIdx.x / a.splits;
-  const int piece = blockIdx.x - u * a.splits;
   const int n_sink_units = a.n_sink_copy[l] * a.n_seg;
   const int n_anchor_units = a.anchor[l] >= 0 ? a.n_seg : 0;
-  if (u >= n_sink_units + n_anchor_units + a.n_kept_copy[l]) return;
+  if (u >= n_sink_units + n_anchor_units + a.n_kept_copy[l]) return false;
   int frame, seg;
   int64_t dst_row = a.CF;
   if (u < n_sink_units) {
@@ -142,30 +139,64 @@ __global__ void __launch_bounds__(256) compact_kernel(const CompactArgs a) {
     dst_row += (int64_t)a.S * a.F + a.F + (int64_t)slot * a.seg_len;
   }
   const int slot = ring_slot(frame, a.S, a.cap_nonsink);
-  const int64_t src_off = ((int64_t)slot * a.F + (int64_t)seg * a.seg_len) * a.D;
-  const int64_t dst_off = dst_row * a.D;
-  const int64_t n = (int64_t)a.seg_len * a.D / 8;      // 16-byte granules per tensor
-  const int64_t g0 = (int64_t)piece * (kCompactPiece / 16);
-  const uint4* sK = reinterpret_cast<const uint4*>(it.pagesK + src_off);
-  const uint4* sV = reinterpret_cast<const uint4*>(it.pagesV + src_off);
-  uint4* dK = reinterpret_cast<uint4*>(it.viewK + dst_off);
-  uint4* dV = reinterpret_cast<uint4*>(it.viewV + dst_off);
+  src_off = ((int64_t)slot * a.F + (int64_t)seg * a.seg_len) * a.D;
+  dst_off = dst_row * a.D;
+  return true;
+}
+
+// One CTA copies 16 KB of keys and 16 KB of values of one dynamic head's view: one piece of
+// one unit (units_per_cta = 1, a unit spans `splits` pieces), or units_per_cta whole small
+// units (token-level segments), each thread resolving the unit of every granule it moves.
+__global__ void __launch_bounds__(256) compact_kernel(const CompactArgs a) {
+  pdl_trigger();
+  pdl_wait();      // kept lists and pages come from the kernels before this one
+  const CompactItem it = a.items[blockIdx.y];
+  if (!a.active[it.layer]) return;
+  const int blk = blockIdx.x / a.splits;
+  const int piece = blockIdx.x - blk * a.splits;
+  const int G = a.units_per_cta;
+  const int64_t n = (int64_t)a.seg_len * a.D / 8;      // 16-byte granules per unit and tensor
   constexpr int kPer = kCompactPiece / 16 / 256;         // granules per thread and tensor
   uint4 k[kPer], v[kPer];
+  uint4* dK[kPer];
+  uint4* dV[kPer];
+  if (G == 1) {
+    int64_t src_off, dst_off;
+    if (!unit_offsets(a, it, blk, src_off, dst_off)) return;
+    const int64_t g0 = (int64_t)piece * (kCompactPiece / 16);
+    const uint4* sK = reinterpret_cast<const uint4*>(it.pagesK + src_off);
+    const uint4* sV = reinterpret_cast<const uint4*>(it.pagesV + src_off);
 #pragma unroll
-  for (int r = 0; r < kPer; ++r) {
-    const int64_t i = g0 + threadIdx.x + r * 256;
-    if (i < n) {
-      k[r] = ld_stream(sK + i);
-      v[r] = ld_stream(sV + i);
+    for (int r = 0; r < kPer; ++r) {
+      const int64_t i = g0 + threadIdx.x + r * 256;
+      dK[r] = nullptr;
+      if (i < n) {
+        k[r] = ld_stream(sK + i);
+        v[r] = ld_stream(sV + i);
+        dK[r] = reinterpret_cast<uint4*>(it.viewK + dst_off) + i;
+        dV[r] = reinterpret_cast<uint4*>(it.viewV + dst_off) + i;
+      }
+    }
+  } else {
+#pragma unroll
+    for (int r = 0; r < kPer; ++r) {
+      const int64_t gi = threadIdx.x + r * 256;          // granule of this CTA's G units
+      dK[r] = nullptr;
+      int64_t src_off, dst_off;
+      if (gi < G * n && unit_offsets(a, it, blk * G + (int)(gi / n), src_off, dst_off)) {
+        const int64_t i = gi - (gi / n) * n;
+        k[r] = ld_stream(reinterpret_cast<const uint4*>(it.pagesK + src_off) + i);
+        v[r] = ld_stream(reinterpret_cast<const uint4*>(it.pagesV + src_off) + i);
+        dK[r] = reinterpret_cast<uint4*>(it.viewK + dst_off) + i;
+        dV[r] = reinterpret_cast<uint4*>(it.viewV + dst_off) + i;
+      }
     }
   }
 #pragma unroll
   for (int r = 0; r < kPer; ++r) {
-    const int64_t i = g0 + threadIdx.x + r * 256;
-    if (i < n) {
-      st_v4(dK + i, k[r]);
-      st_v4(dV + i, v[r]);
+    if (dK[r]) {
+      st_v4(dK[r], k[r]);
+      st_v4(dV[r], v[r]);
     }
   }
 }
@@ -194,7 +225,8 @@ void launch_compact(const CompactArgs& a, cudaStream_t s) {
   if (a.n_items == 0 || a.max_units == 0) return;
   // programmatic launch: the grid is scheduled while the selection kernel runs
   cudaLaunchConfig_t cfg{};
-  cfg.gridDim = dim3((unsigned)(a.max_units * a.splits), (unsigned)a.n_items);
+  const int blocks = (a.max_units + a.units_per_cta - 1) / a.units_per_cta;
+  cfg.gridDim = dim3((unsigned)(blocks * a.splits), (unsigned)a.n_items);
   cfg.blockDim = dim3(256);
   cfg.dynamicSmemBytes = 0;
   cfg.stream = s;

@@ -96,6 +96,9 @@ struct fk_handle {
   int scope = 0, source = 0, incremental = 0, max_hist = 0, dev = 0;
   int seg = 0, CF = 0;
   int cap_nonsink = 0, ring_slots = 0, k_frame = 0, kmax = 0, chunks = 0;
+  int selection = FK_SELECT_SIMILARITY;
+  uint32_t select_seed = 0;
+  bool drop_anchor = false;        // static heads keep sink + current chunk only
   std::vector<HeadBuf> heads;      // [L*H]
   std::vector<LayerState> layers;  // [L]
   // device memory
@@ -185,15 +188,17 @@ Roles roles_of(const fk_handle* h, int nh) {
 
 int keep_total(const fk_handle* h, int n_scoreable) {
   if (h->scope == FK_SCOPE_PER_FRAME) return n_scoreable * h->k_frame;
+  if (h->selection == FK_SELECT_ALL) return n_scoreable * h->n;
   return (int)(((int64_t)h->b * n_scoreable * h->n) / 1000);
 }
 
 void update_lengths(fk_handle* h, int l) {
   LayerState& ls = h->layers[l];
   const Roles r = roles_of(h, ls.nh);
-  const int base = h->CF + r.n_sink * h->F + (r.anchor >= 0 ? h->F : 0);
-  ls.len_static = base;
-  ls.len_dynamic = base + ls.n_keep * h->seg;
+  const int base = h->CF + r.n_sink * h->F;
+  const int anchor_rows = r.anchor >= 0 ? h->F : 0;
+  ls.len_static = base + (h->drop_anchor ? 0 : anchor_rows);
+  ls.len_dynamic = base + anchor_rows + ls.n_keep * h->seg;
 }
 
 // ---- profiling and launch accounting
@@ -341,7 +346,7 @@ fk_status push_history(fk_handle* h, int layer, const bf16* tokK, const bf16* to
         pa.dstV[hd] = hb.pageV + ring_slot(h, f) * frame_elems;
         any_p = true;
       }
-      if (hb.is_static && (sink || is_anchor)) {
+      if (hb.is_static && (sink || (is_anchor && !h->drop_anchor))) {
         const int64_t row = h->CF + (int64_t)(sink ? f : h->S) * h->F;
         va.dstK[hd] = hb.viewK + row * h->D;
         va.dstV[hd] = hb.viewV + row * h->D;
@@ -389,6 +394,7 @@ fk_status update_current(fk_handle* h, int layer, bool retire, const void* K, co
   a.W = h->W;
   a.cap_nonsink = h->cap_nonsink;
   a.retire = retire ? 1 : 0;
+  a.static_anchor = h->drop_anchor ? 0 : 1;
   a.nh_old = ls.nh;
   for (int hd = 0; hd < h->H; ++hd) {
     const HeadBuf& hb = h->heads[layer * h->H + hd];
@@ -471,7 +477,7 @@ fk_status fk_set_host_overlap(fk_handle* h, int on) {
   return FK_OK;
 }
 
-int fk_abi_version(void) { return 1; }
+int fk_abi_version(void) { return 2; }
 
 const char* fk_status_str(fk_status s) {
   switch (s) {
@@ -502,6 +508,9 @@ fk_status fk_validate_config(const fk_config* c) {
     return FK_ERR_CONFIG;
   if (c->incremental != 0 && c->incremental != 1) return FK_ERR_CONFIG;
   if (c->window_frames == 0 && c->max_history_frames < 1) return FK_ERR_CONFIG;
+  if (c->selection < FK_SELECT_SIMILARITY || c->selection > FK_SELECT_RANDOM) return FK_ERR_CONFIG;
+  if (c->selection == FK_SELECT_UNIFORM && c->select_scope != FK_SCOPE_PER_FRAME) return FK_ERR_CONFIG;
+  if (c->static_drop_anchor != 0 && c->static_drop_anchor != 1) return FK_ERR_CONFIG;
   const int64_t cf = (int64_t)c->frames_per_chunk * c->tokens_per_frame;
   if (cf > (1 << 24) || (int64_t)c->tokens_per_frame * c->head_dim > (1 << 28)) return FK_ERR_CONFIG;
   // 16-byte granules of one chunk (all heads) are indexed with 32-bit integers
@@ -541,7 +550,10 @@ fk_status fk_create(const fk_config* cfg, fk_handle** out) {
   h->cap_nonsink = h->W > 0 ? h->W : std::max(0, h->max_hist - h->S);
   if (h->cap_nonsink < 1) h->cap_nonsink = 1;
   h->ring_slots = h->S + h->cap_nonsink;
-  h->k_frame = (h->b * h->n) / 1000;
+  h->selection = cfg->selection;
+  h->select_seed = cfg->select_seed;
+  h->drop_anchor = cfg->static_drop_anchor != 0;
+  h->k_frame = h->selection == FK_SELECT_ALL ? h->n : (h->b * h->n) / 1000;
   h->kmax = std::max(1, keep_total(h, h->cap_nonsink - 1));
   h->chunks = (h->seg + kScoreTokensPerCta - 1) / kScoreTokensPerCta;
   h->max_run = h->cap_nonsink;
@@ -803,7 +815,14 @@ fk_status fk_compress(fk_handle* h, void* stream) {
     const int keep = keep_total(h, r.n_scoreable);
     // scoring run of the layer whose keys score (every layer per head; layer 0 pooled)
     const bool scores_here = pooled_src ? l == 0 : true;
-    if (ls.dirty && scores_here) {
+    if (ls.dirty && scores_here && h->selection != FK_SELECT_SIMILARITY) {
+      // comparison rules: no scoring; the selection kernel ranks the whole window by the
+      // rule's values
+      if (r.n_scoreable > 0) {
+        sa.run[l] = {r.t_lo, r.n_scoreable + 1};
+        any_run = true;
+      }
+    } else if (ls.dirty && scores_here) {
       const int t_first = h->incremental ? std::max(r.t_lo, ls.scored_upto) : r.t_lo;
       const int last_t = r.t_lo + r.n_scoreable - 1;
       if (r.n_scoreable > 0 && t_first <= last_t) {
@@ -886,7 +905,11 @@ fk_status fk_compress(fk_handle* h, void* stream) {
     sa.scores = h->scores;
     sa.kept = h->kept;
     sa.status = h->status;
-    if ((st = launch(h, s, FK_KERNEL_SCORE, [&] { launch_score(sa, s); })) != FK_OK) return st;
+    sa.rule = h->selection;
+    sa.seed = h->select_seed;
+    if (h->selection == FK_SELECT_SIMILARITY &&
+        (st = launch(h, s, FK_KERNEL_SCORE, [&] { launch_score(sa, s); })) != FK_OK)
+      return st;
     const int nt = (int)h->targets.size();
     if ((st = launch(h, s, FK_KERNEL_SELECT, [&] { launch_select(sa, nt, s); })) != FK_OK) return st;
   }
@@ -901,7 +924,9 @@ fk_status fk_compress(fk_handle* h, void* stream) {
     ca.S = h->S;
     ca.cap_nonsink = h->cap_nonsink;
     ca.kmax = h->kmax;
-    ca.splits = (int)((int64_t(h->seg) * h->D * 2 + kCompactPiece - 1) / kCompactPiece);
+    const int64_t unit_bytes = (int64_t)h->seg * h->D * 2;
+    ca.splits = (int)((unit_bytes + kCompactPiece - 1) / kCompactPiece);
+    ca.units_per_cta = unit_bytes < kCompactPiece ? (int)(kCompactPiece / unit_bytes) : 1;
     ca.kept = h->kept;
     if ((st = launch(h, s, FK_KERNEL_COMPACT, [&] { launch_compact(ca, s); })) != FK_OK) return st;
   }

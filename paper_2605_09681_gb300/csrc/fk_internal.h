@@ -42,6 +42,7 @@ struct CurrentArgs {
   int F, S, W, cap_nonsink;
   int retire;                   // 1: the previous current chunk joins the history
   int nh_old;                   // history frames before the retire
+  int static_anchor;            // 1: static views keep the anchor frame (Eq. 2)
   bf16* viewK[kMaxHeads];       // view fronts (current chunk rows)
   bf16* viewV[kMaxHeads];
   bf16* pageK[kMaxHeads];       // page rings (nullptr: head keeps no history pages)
@@ -95,6 +96,8 @@ struct ScoreArgs {
   int act_first_item[kMaxLayers];   // first score item of the layer
   long long act_start[kMaxLayers];  // first frame-chunk of the layer in the flattened range
   int scope;                    // FK_SCOPE_*
+  int rule;                     // FK_SELECT_*: similarity scores, or a comparison rule's values
+  unsigned int seed;            // FK_SELECT_RANDOM
   int k_frame;                  // kept per frame (per-frame scope)
   int kmax;                     // capacity of one kept list
   unsigned long long* sums;     // scratch [target][max_run][n_seg][2] : {N(t), D(t-1,t)}, zero between launches
@@ -129,6 +132,7 @@ struct CompactArgs {
   int F, D, n_seg, seg_len, CF;
   int S, cap_nonsink, kmax;
   int splits;                   // pieces per unit (each at most kCompactPiece bytes per tensor)
+  int units_per_cta;            // whole units per CTA when a unit is smaller (then splits = 1)
   const int* kept;
   // per layer: what this launch copies into the dynamic views [current | sinks | anchor |
   // kept ring of kmax segment slots]

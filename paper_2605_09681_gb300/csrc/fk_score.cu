@@ -15,6 +15,7 @@
 // atomic) finishes s = D / sqrt(N_t N_{t+1}) in IEEE double, stores the fp32 scores per frame
 // slot, ranks the scoreable candidates by (score, segment id) and stream-compacts the kept
 // segment ids with warp ballots and prefix sums.
+#include <algorithm>
 #include <mutex>
 
 #include "fk_internal.h"
@@ -119,6 +120,127 @@ __device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_
 __device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
+// SplitMix64 (Steele, Lea and Flood, 2014): the 64-bit finaliser of a Weyl sequence.
+__device__ __forceinline__ unsigned long long splitmix64(unsigned long long z) {
+  z += 0x9E3779B97F4A7C15ull;
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+// Ranking value of candidate (t, j) under a comparison rule (BottomK keeps the smallest):
+// ALL 0 for every segment (with k = n all are kept); UNIFORM 0 on the k segments
+// j = floor(i n / k), i < k, else 1; RANDOM a uniform value in [0, 1) with 24 random bits,
+// SplitMix64 of seed * 2^40 + t * 2^20 + j.
+__device__ __forceinline__ float rule_value(int rule, unsigned int seed, int t, int j, int n, int k) {
+  if (rule == FK_SELECT_UNIFORM) {
+    if (k <= 0) return 1.0f;
+    const long long i = ((long long)j * k + n - 1) / n;     // smallest i with i n / k >= j
+    return (i < k && (i * n) / k == j) ? 0.0f : 1.0f;
+  }
+  if (rule == FK_SELECT_RANDOM) {
+    const unsigned long long key = ((unsigned long long)seed << 40) ^ ((unsigned long long)t << 20) ^
+                                   (unsigned long long)j;
+    return (float)(splitmix64(key) >> 40) * (1.0f / 16777216.0f);
+  }
+  return 0.0f;
+}
+
+// Up to this many segments per frame the per-frame ranking compares every pair; above it
+// (token-level rules) each frame is sorted in shared memory.
+constexpr int kRankDirect = 64;
+__host__ __device__ constexpr int select_sort_len(int n) {   // next power of two >= n
+  int p = 1;
+  while (p < n) p <<= 1;
+  return p;
+}
+__host__ __device__ constexpr size_t select_sort_off(int max_run, int n) {   // 8-byte aligned
+  return ((size_t)max_run * n * sizeof(float) + 7) / 8 * 8;
+}
+
+// BottomK of one frame with many segments (token-level rules): sort (value, id) keys in
+// shared memory (bitonic), flag the k smallest ids, write them in ascending id order as
+// frame-t segment ids into out[0 .. min(k, bound)).  Block-uniform arguments.
+__device__ void sort_select_frame(const float* vals, int n, int k, int t, int* out, int bound,
+                                  unsigned long long* key, int* flag, int* warp_tot, int* base_off) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int P = select_sort_len(n);
+  for (int i = threadIdx.x; i < P; i += blockDim.x) {
+    unsigned long long kv = ~0ull;
+    if (i < n) {
+      float v = vals[i];
+      if (v == 0.0f) v = 0.0f;                       // -0 ranks as +0
+      const uint32_t u = __float_as_uint(v);
+      const uint32_t ord = (u & 0x80000000u) ? ~u : (u | 0x80000000u);   // order-preserving
+      kv = ((unsigned long long)ord << 32) | (unsigned)i;
+    }
+    key[i] = kv;
+  }
+  for (int j = threadIdx.x; j < n; j += blockDim.x) flag[j] = 0;
+  __syncthreads();
+  for (int size = 2; size <= P; size <<= 1) {
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      for (int i = threadIdx.x; i < P / 2; i += blockDim.x) {
+        const int lo = 2 * stride * (i / stride) + (i % stride), hi = lo + stride;
+        const unsigned long long x = key[lo], y = key[hi];
+        if ((x > y) == ((lo & size) == 0)) {
+          key[lo] = y;
+          key[hi] = x;
+        }
+      }
+      __syncthreads();
+    }
+  }
+  for (int i = threadIdx.x; i < k && i < n; i += blockDim.x) flag[(int)(key[i] & 0xFFFFFFFFu)] = 1;
+  if (threadIdx.x == 0) *base_off = 0;
+  __syncthreads();
+  for (int b0 = 0; b0 < n; b0 += blockDim.x) {
+    const int j = b0 + threadIdx.x;
+    const bool keep = j < n && flag[j];
+    const unsigned mask = __ballot_sync(0xffffffffu, keep);
+    if (lane == 0) warp_tot[warp] = __popc(mask);
+    __syncthreads();
+    int woff = *base_off;
+    for (int w = 0; w < warp; ++w) woff += warp_tot[w];
+    const int pos = woff + __popc(mask & ((1u << lane) - 1u));
+    if (keep && pos < bound) out[pos] = t * n + j;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      int tot = 0;
+      for (int w = 0; w < (int)(blockDim.x >> 5); ++w) tot += warp_tot[w];
+      *base_off += tot;
+    }
+    __syncthreads();
+  }
+}
+
+// Selection kernel for a comparison rule with many segments per frame (per-frame scope): one
+// CTA per (target, frame of the window); the rule's values need no scores, so the frames are
+// independent.
+__global__ void __launch_bounds__(kSelectThreads) select_frames_kernel(const ScoreArgs a) {
+  extern __shared__ float vals[];
+  __shared__ int warp_tot[kSelectThreads / 32];
+  __shared__ int base_off;
+  const int tgi = blockIdx.x, f = blockIdx.y;
+  const int l = a.targets[tgi].layer;
+  pdl_trigger();
+  pdl_wait();
+  if (a.run[l].n_run < 2 || f >= a.n_scoreable[l]) return;
+  const int n = a.n_seg, k = a.k_frame, t = a.t_lo[l] + f;
+  float* sc = a.scores + (int64_t)tgi * a.ring_slots * n + (int64_t)ring_slot(t, a.S, a.cap_nonsink) * n;
+  for (int j = threadIdx.x; j < n; j += blockDim.x) {
+    const float v = rule_value(a.rule, a.seed, t, j, n, k);
+    vals[j] = v;
+    sc[j] = v;
+  }
+  unsigned long long* key = reinterpret_cast<unsigned long long*>(
+      reinterpret_cast<uint8_t*>(vals) + ((size_t)n * sizeof(float) + 7) / 8 * 8);
+  int* flag = reinterpret_cast<int*>(key + select_sort_len(n));
+  __syncthreads();
+  sort_select_frame(vals, n, k, t, a.kept + (int64_t)tgi * a.kmax + (int64_t)f * k,
+                    a.n_keep[l] - f * k, key, flag, warp_tot, &base_off);
+}
+
 // Selection kernel: one CTA per selection target.  Finishes the pairs (t, t+1) scored by
 // this launch from the target's int64 sums, clears the sums for the next launch, then
 // BottomK over the scoreable frames compacted in ascending segment-id order; the window's
@@ -142,6 +264,16 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const ScoreArgs 
   const int t_lo = a.t_lo[l];
   float* sc = a.scores + (int64_t)tgi * a.ring_slots * n;
   unsigned long long* sums = a.sums + (int64_t)tgi * a.max_run * n * 2;
+  if (a.rule != FK_SELECT_SIMILARITY) {
+    // comparison rules: the ranking values come from the rule, not from scores
+    for (int idx = threadIdx.x; idx < M; idx += blockDim.x) {
+      const int t = t_lo + idx / n, jj = idx - (idx / n) * n;
+      const float v = rule_value(a.rule, a.seed, t, jj, n, a.k_frame);
+      ssc[idx] = v;
+      sc[ring_slot(t, a.S, a.cap_nonsink) * n + jj] = v;
+    }
+    __syncthreads();
+  } else {
   // 1. finish: s = D / sqrt(N_t N_{t+1}) in IEEE double, stored per frame slot and staged
   //    for the ranking when the frame is in the window
   const int pairs = (run.n_run - 1) * n;
@@ -162,12 +294,24 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const ScoreArgs 
   }
   __syncthreads();   // every sum has been read
   for (int i = threadIdx.x; i < run.n_run * n * 2; i += blockDim.x) sums[i] = 0ull;
+  }
 
   // 2. BottomK: rank by (score, segment id) within the frame (per-frame scope) or over the
   //    whole window (pooled scope), then stream-compact with warp ballots
   const int K = a.n_keep[l];
   int* out = a.kept + (int64_t)tgi * a.kmax;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (a.scope == FK_SCOPE_PER_FRAME && n > kRankDirect) {
+    // many segments per frame (token-level rules): sort each frame in shared memory;
+    // frame f's kept ids fill out[f k .. f k + k)
+    unsigned long long* key = reinterpret_cast<unsigned long long*>(
+        reinterpret_cast<uint8_t*>(ssc) + select_sort_off(a.max_run, n));
+    int* flag = reinterpret_cast<int*>(key + select_sort_len(n));
+    for (int f = 0; f < nT; ++f)
+      sort_select_frame(ssc + f * n, n, a.k_frame, t_lo + f, out + f * a.k_frame, K - f * a.k_frame,
+                        key, flag, warp_tot, &base_off);
+    return;
+  }
   if (threadIdx.x == 0) base_off = 0;
   __syncthreads();
   for (int b0 = 0; b0 < M; b0 += blockDim.x) {
@@ -409,7 +553,12 @@ constexpr size_t score_smem_bytes_d(int max_run) {
 size_t score_smem_bytes(int head_dim, int max_run) {
   return head_dim == 128 ? score_smem_bytes_d<128>(max_run) : score_smem_bytes_d<64>(max_run);
 }
-size_t select_smem_bytes(int max_run, int n_seg) { return (size_t)max_run * n_seg * sizeof(float); }
+size_t select_smem_bytes(int max_run, int n_seg) {
+  size_t b = (size_t)max_run * n_seg * sizeof(float);
+  if (n_seg > kRankDirect)   // sort keys and flags of one frame
+    b = select_sort_off(max_run, n_seg) + (size_t)select_sort_len(n_seg) * 8 + (size_t)n_seg * 4;
+  return b;
+}
 
 // launch with the programmatic-dependent-launch attribute: the kernel's prologue may
 // overlap the previous kernel's tail; its pdl_wait() orders it after that kernel
@@ -467,7 +616,26 @@ void launch_score(const ScoreArgs& a, cudaStream_t s) {
 }
 
 void launch_select(const ScoreArgs& a, int n_targets, cudaStream_t s) {
-  if (n_targets <= 0 || a.total_units <= 0) return;
+  if (n_targets <= 0) return;
+  if (a.rule != FK_SELECT_SIMILARITY && a.scope == FK_SCOPE_PER_FRAME && a.n_seg > kRankDirect) {
+    int frames = 0;
+    for (int l = 0; l < kMaxLayers; ++l) frames = std::max(frames, a.n_scoreable[l]);
+    if (frames <= 0) return;
+    const size_t smem = ((size_t)a.n_seg * sizeof(float) + 7) / 8 * 8 +
+                        (size_t)select_sort_len(a.n_seg) * 8 + (size_t)a.n_seg * 4;
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3((unsigned)n_targets, (unsigned)frames);
+    cfg.blockDim = dim3(kSelectThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cudaLaunchKernelEx(&cfg, select_frames_kernel, a);
+    return;
+  }
   launch_pdl(select_kernel, (unsigned)n_targets, kSelectThreads, select_smem_bytes(a.max_run, a.n_seg), s, a);
 }
 

@@ -46,8 +46,13 @@ def _cfg(**kw):
 
 def test_config_struct_layout():
     from paper_2605_09681_gb300._lib import FkConfig
-    assert ctypes.sizeof(FkConfig) == 64
+    assert ctypes.sizeof(FkConfig) == 80
     assert FkConfig.head_is_static.offset == 56
+    assert (FkConfig.selection.offset, FkConfig.select_seed.offset, FkConfig.static_drop_anchor.offset) == (64, 68, 72)
+
+
+def test_abi_version(lib):
+    assert lib.fk_abi_version() == 2
 
 
 @pytest.mark.parametrize("bad", [
@@ -55,7 +60,8 @@ def test_config_struct_layout():
     dict(n_layers=257), dict(tokens_per_frame=61), dict(n_segments=0), dict(frames_per_chunk=0),
     dict(keep_budget_permille=1001), dict(keep_budget_permille=-1), dict(select_scope=2),
     dict(score_source=5), dict(incremental=2), dict(window_frames=-1), dict(n_sink_frames=-1),
-    dict(window_frames=0, max_history_frames=0),
+    dict(window_frames=0, max_history_frames=0), dict(selection=4), dict(selection=-1),
+    dict(selection=2, select_scope=1, n_segments=1), dict(static_drop_anchor=2),
 ])
 def test_validate_rejects_bad_configs(lib, bad):
     c, _keep = _cfg(**bad)
@@ -67,7 +73,10 @@ def test_validate_accepts_paper_configs(lib):
                dict(head_dim=128, n_heads=12, tokens_per_frame=8160, max_history_frames=10),
                dict(window_frames=12, keep_budget_permille=600),
                dict(n_segments=1, select_scope=1, keep_budget_permille=500, n_sink_frames=0),
-               dict(n_layers=30, n_heads=12, score_source=1, incremental=1, max_history_frames=21)]:
+               dict(n_layers=30, n_heads=12, score_source=1, incremental=1, max_history_frames=21),
+               dict(selection=1, n_sink_frames=3, window_frames=4),
+               dict(selection=1, window_frames=2, static_drop_anchor=1),
+               dict(selection=2, n_segments=60), dict(selection=3, select_seed=7, n_segments=60)]:
         c, _keep = _cfg(**kw)
         assert lib.fk_validate_config(ctypes.byref(c)) == 0, kw
 
@@ -76,7 +85,7 @@ def test_null_config_and_status_strings(lib):
     assert lib.fk_validate_config(None) == 2
     for s in range(9):
         assert lib.fk_status_str(s)
-    assert lib.fk_abi_version() == 1
+    assert lib.fk_abi_version() == 2
 
 
 @pytest.mark.skipif(os.path.exists("/dev/nvidia0"), reason="checks the no-GPU error path")

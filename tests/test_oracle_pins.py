@@ -421,3 +421,45 @@ def test_classify_head_threshold():
     assert not O.classify_head([10.0, 4.0, 2.0, 1.0], 0.8)      # 6/9 = 0.667: dynamic
     assert not O.classify_head([10.0, 6.0, 2.0, 0.0], 0.8)      # exactly 0.8 is not above it
     assert O.classify_head([10.0, 0.0, 0.0, 10.0], 0.8)         # all mass on the sinks
+
+
+# ---- comparison selection rules (App. H, Sec. 5.3)
+
+def test_splitmix64_published_vector():
+    # first output of SplitMix64 from state 0 (the generator's published reference output)
+    assert O.splitmix64(0) == 0xE220A8397B1DCDAF
+
+
+def test_rule_uniform_keeps_evenly_spaced_segments():
+    for n, k in [(6, 4), (6, 3), (1560, 1092), (10, 10), (7, 1)]:
+        kept = [j for j in range(n) if O.rule_value("uniform", 0, 3, j, n, k) == 0.0]
+        assert kept == sorted({i * n // k for i in range(k)}) and len(kept) == k
+    assert O.rule_value("uniform", 0, 0, 0, 6, 0) == 1.0
+
+
+def test_rule_random_is_seeded_uniform():
+    vals = np.array([O.rule_value("random", 7, t, j, 1560, 1092) for t in range(3) for j in range(1560)])
+    assert np.all((vals >= 0) & (vals < 1)) and abs(vals.mean() - 0.5) < 0.02
+    assert np.all(vals * 16777216 == np.floor(vals * 16777216))          # 24-bit values
+    again = [O.rule_value("random", 7, 1, j, 1560, 1092) for j in range(5)]
+    other = [O.rule_value("random", 8, 1, j, 1560, 1092) for j in range(5)]
+    assert again == [O.rule_value("random", 7, 1, j, 1560, 1092) for j in range(5)] and again != other
+
+
+def test_rule_workloads_key_sets():
+    # StreamingLLM: every head = 3 sinks + 4 recent frames + chunk; Dummy Forcing L = 2:
+    # local heads = sink + chunk, neighbour heads = sink + 2 recent frames + chunk
+    F = 12
+    for w, want_static, want_dynamic in [
+            (W.STREAMINGLLM_480P, None, (3 + 4 + 3) * F),
+            (W.DUMMY_FORCING_480P, (1 + 3) * F, (1 + 2 + 3) * F)]:
+        w = w.with_(tokens_per_frame=F, n_heads=4, head_dim=16,
+                    n_segments=6 if w.n_segments == 6 else F)
+        hm = W.head_map(w)
+        orc = O.ForcingKVOracle.from_workload(w, hm)
+        hk, hv, ck, cv, q = W.snapshot_inputs(w)
+        orc.append_frames(0, hk, hv)
+        orc.set_current(0, ck, cv)
+        for h in range(4):
+            n = orc.view_length(0, h)
+            assert n == (want_static if hm[0, h] else want_dynamic), (w.name, h, n)

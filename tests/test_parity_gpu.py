@@ -329,3 +329,12 @@ def test_host_inputs_and_overlap_match_device_inputs():
                           for o in outs]
     for a, b, c in zip(runs["device"], runs["host"], runs["overlap"]):
         assert np.array_equal(a, b) and np.array_equal(a, c)
+
+
+@pytest.mark.parametrize("name", ["full_kv_480p", "streamingllm_480p", "dummy_forcing_480p",
+                                  "uniform_tokens_480p", "random_tokens_480p"])
+def test_comparison_rules_480p(name):
+    # the paper's comparison rules through the same selection, compaction and attention
+    # kernels: kept sets and ranking values bit-exact, attention within tolerance
+    w = W.WORKLOADS[name]
+    run_snapshot(w, rows=sample_rows(w.n_queries, 64))

@@ -30,7 +30,8 @@ import numpy as np
 __all__ = [
     "Workload", "TINY", "TINY_PER_FRAME", "P480_LAYER", "P480_STACK", "ROLLING",
     "P1080_LAYER", "WORKLOADS", "normals", "uniforms", "to_bf16_bits", "bf16_bits_to_f32",
-    "profile_inputs",
+    "profile_inputs", "FULL_KV_480P", "STREAMINGLLM_480P", "DUMMY_FORCING_480P", "UNIFORM_TOKENS_480P",
+    "RANDOM_TOKENS_480P",
     "head_map", "FrameStream", "snapshot_inputs", "queries", "step_kv", "stream_key",
 ]
 
@@ -128,6 +129,9 @@ class Workload:
     static_heads: tuple = ()             # fixed static heads (empty = seeded map)
     static_fraction: float = 0.5
     exact_half_static: bool = True       # seeded permutation with exactly H/2 static
+    selection: str = "similarity"        # "similarity" | "all" | "uniform" | "random"
+    select_seed: int = 0
+    static_drop_anchor: bool = False
     seed: int = 0
     description: str = ""
 
@@ -195,7 +199,33 @@ P1080_LAYER = Workload(
     description="1080P single layer: 12 heads, D=128, 8160 tokens/frame (68x120), 24480 queries, "
                 "1 sink + 9 history frames, 70% dynamic budget")
 
-WORKLOADS = {w.name: w for w in (TINY, TINY_PER_FRAME, P480_LAYER, P480_STACK, ROLLING, P1080_LAYER)}
+# The paper's comparison rules (App. H, Sec. 5.3) on the 480P layer snapshot, for speed
+# comparisons through the same kernels (their quality claims need model weights).
+FULL_KV_480P = P480_LAYER.with_(
+    name="full_kv_480p", selection="all", exact_half_static=False, static_fraction=0.0,
+    description="the uncompressed cache on the 480P layer: every head keeps every frame of the "
+                "window (the paper's full-KV reference)")
+STREAMINGLLM_480P = P480_LAYER.with_(
+    name="streamingllm_480p", n_sink_frames=3, window_frames=4, selection="all",
+    exact_half_static=False, static_fraction=0.0,
+    description="frame-level StreamingLLM on the 480P layer: every head keeps 3 sink frames and "
+                "the 4 most recent history frames")
+DUMMY_FORCING_480P = P480_LAYER.with_(
+    name="dummy_forcing_480p", window_frames=2, selection="all", static_drop_anchor=True,
+    description="Dummy Forcing (L = 2) on the 480P layer: local heads keep the sink and the chunk, "
+                "neighbour heads the sink and the last 2 history frames")
+UNIFORM_TOKENS_480P = P480_LAYER.with_(
+    name="uniform_tokens_480p", n_segments=1560, selection="uniform",
+    description="uniform token pruning on the 480P layer's dynamic heads: 1092 evenly spaced "
+                "tokens of each history frame (70%)")
+RANDOM_TOKENS_480P = P480_LAYER.with_(
+    name="random_tokens_480p", n_segments=1560, selection="random", select_seed=7,
+    description="random token pruning on the 480P layer's dynamic heads: 1092 seeded random "
+                "tokens of each history frame (70%)")
+
+WORKLOADS = {w.name: w for w in (TINY, TINY_PER_FRAME, P480_LAYER, P480_STACK, ROLLING, P1080_LAYER,
+                                 FULL_KV_480P, STREAMINGLLM_480P, DUMMY_FORCING_480P,
+                                 UNIFORM_TOKENS_480P, RANDOM_TOKENS_480P)}
 
 
 def head_map(w: Workload) -> np.ndarray:
