@@ -539,8 +539,8 @@ def run_stack(local_rank):
 NCU_TRAFFIC = {
     "480p_layer": {
         "attend": ("fk_attn.cu", "fc08b6769224", 122271744),
-        "compact": ("fk_copy.cu", "696e1eb5e98a", 76390912),
-        "score": ("fk_score.cu", "584831ae7a26", 43160320),
+        "compact": ("fk_copy.cu", "7bff156f176c", 76305408),
+        "score": ("fk_score.cu", "cb7cdc3bafa2", 43160576),
     },
 }
 

@@ -209,6 +209,14 @@ FK_API fk_status fk_profile_reset(fk_handle* h);
  * FK_ERR_ARG for a null handle. */
 FK_API fk_status fk_set_host_overlap(fk_handle* h, int on);
 
+/* Failure-detection self-test (no counterpart in the paper): launches a one-thread kernel
+ * that waits, with the same bounded-wait primitive as the hot-path kernels, on an mbarrier
+ * that nothing completes; after limit_us microseconds (1..2,000,000) the wait gives up and
+ * records the expiry in the handle's status word, so the next fk_sync_status returns
+ * FK_ERR_TIMEOUT and clears it.  No fault: the CUDA context stays usable.  Asynchronous on
+ * `stream`.  FK_ERR_ARG for a null handle or a limit out of range. */
+FK_API fk_status fk_wait_selftest(fk_handle* h, int limit_us, void* stream);
+
 /* Kernels launched by this handle since creation (all kinds). */
 FK_API int64_t fk_launch_count(const fk_handle* h);
 

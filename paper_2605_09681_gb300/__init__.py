@@ -228,6 +228,11 @@ class ForcingKVCache:
                                          ctypes.byref(n)), "fk_profile_read")
         return ms.value, n.value
 
+    def wait_selftest(self, limit_us: int = 20000, stream=None) -> None:
+        """Run the bounded-wait self-test (fk_wait_selftest): the next sync_status() reports
+        FK_ERR_TIMEOUT."""
+        _check(self._lib.fk_wait_selftest(self._h, int(limit_us), _stream(stream)), "fk_wait_selftest")
+
     def set_host_overlap(self, on: bool = True) -> None:
         """Copy host inputs on the handle's copy stream as soon as a call is made (see
         fk_set_host_overlap): the caller promises host inputs are final at call time."""

@@ -471,6 +471,16 @@ fk_status fk_classify_heads(const double* mass, int n_heads, int alpha_permille,
   return FK_OK;
 }
 
+fk_status fk_wait_selftest(fk_handle* h, int limit_us, void* stream) {
+  if (!h) return FK_ERR_ARG;
+  if (limit_us < 1 || limit_us > 2000000) return FK_ERR_ARG;
+  FK_CUDA(cudaSetDevice(h->dev));
+  return launch_wait_selftest((uint64_t)limit_us * 1000ull, h->status,
+                              static_cast<cudaStream_t>(stream)) == cudaSuccess
+             ? FK_OK
+             : FK_ERR_CUDA;
+}
+
 fk_status fk_set_host_overlap(fk_handle* h, int on) {
   if (!h) return FK_ERR_ARG;
   h->host_overlap = on != 0;

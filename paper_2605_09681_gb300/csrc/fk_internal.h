@@ -111,6 +111,8 @@ struct ScoreArgs {
 };
 void launch_score(const ScoreArgs& a, cudaStream_t s);
 void launch_select(const ScoreArgs& a, int n_targets, cudaStream_t s);
+// one-thread kernel whose bounded wait expires after limit_ns (failure-detection self-test)
+cudaError_t launch_wait_selftest(uint64_t limit_ns, int* status, cudaStream_t s);
 // dynamic shared memory limits and the persistent grid size (CTAs resident at once)
 cudaError_t score_prepare(int head_dim, int max_run, int n_seg, int* max_ctas);
 // frame-chunks in flight per scoring CTA (one bulk copy each)

@@ -102,11 +102,12 @@ __device__ __forceinline__ bool mbar_test(uint32_t bar, uint32_t parity) {
   return ok != 0;
 }
 // bounded wait for the phase of parity `parity`; false when the limit expired
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity,
+                                          uint64_t limit_ns = kWaitLimitNs) {
   if (mbar_test(bar, parity)) return true;
   const uint64_t t0 = now_ns();
   while (!mbar_test(bar, parity))
-    if (now_ns() - t0 > kWaitLimitNs) return false;
+    if (now_ns() - t0 > limit_ns) return false;
   return true;
 }
 // one contiguous global -> shared copy on the TMA engine, completing on `bar`
@@ -578,7 +579,23 @@ cudaError_t launch_pdl(Kern kern, unsigned grid, unsigned threads, size_t smem, 
   return cudaLaunchKernelEx(&cfg, kern, a);
 }
 
+// Self-test of the bounded wait: one thread waits on an mbarrier that nothing arrives on,
+// with the kernels' wait primitive and a short limit, then records the expiry in the status
+// word exactly as the production kernels do and returns.
+__global__ void wait_selftest_kernel(uint64_t limit_ns, int* status) {
+  __shared__ __align__(8) uint64_t bar;
+  const uint32_t b = su32_shared(&bar);
+  mbar_init(b, 1);
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  if (!mbar_wait(b, 0, limit_ns)) atomicOr(status, kStatusTimeout);
+}
+
 }  // namespace
+
+cudaError_t launch_wait_selftest(uint64_t limit_ns, int* status, cudaStream_t s) {
+  wait_selftest_kernel<<<1, 1, 0, s>>>(limit_ns, status);
+  return cudaGetLastError();
+}
 
 cudaError_t score_prepare(int head_dim, int max_run, int n_seg, int* max_ctas) {
   const int smem = (int)score_smem_bytes(head_dim, max_run);

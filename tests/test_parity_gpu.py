@@ -338,3 +338,20 @@ def test_comparison_rules_480p(name):
     # kernels: kept sets and ranking values bit-exact, attention within tolerance
     w = W.WORKLOADS[name]
     run_snapshot(w, rows=sample_rows(w.n_queries, 64))
+
+
+def test_bounded_wait_expiry_is_reported_and_context_survives():
+    # a wait on an mbarrier that nothing completes gives up after its limit, the status word
+    # reports FK_ERR_TIMEOUT once, and the same handle then runs the hot path normally
+    from paper_2605_09681_gb300 import ForcingKVCache
+    from paper_2605_09681_gb300._lib import FK_ERR_TIMEOUT
+    import time
+    w = W.TINY_PER_FRAME
+    hm = W.head_map(w)
+    with ForcingKVCache.from_workload(w, hm) as cache:
+        t0 = time.perf_counter()
+        cache.wait_selftest(20000)                   # 20 ms
+        assert cache.sync_status() == FK_ERR_TIMEOUT
+        assert time.perf_counter() - t0 >= 0.019
+        assert cache.sync_status() == 0              # cleared once read
+    run_snapshot(w)                                  # the context is still usable
