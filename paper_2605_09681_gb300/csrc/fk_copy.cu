@@ -158,38 +158,45 @@ __global__ void __launch_bounds__(256) compact_kernel(const CompactArgs a) {
   const int64_t n = (int64_t)a.seg_len * a.D / 8;      // 16-byte granules per unit and tensor
   constexpr int kPer = kCompactPiece / 16 / 256;         // granules per thread and tensor
   uint4 k[kPer], v[kPer];
-  uint4* dK[kPer];
-  uint4* dV[kPer];
   if (G == 1) {
     int64_t src_off, dst_off;
     if (!unit_offsets(a, it, blk, src_off, dst_off)) return;
     const int64_t g0 = (int64_t)piece * (kCompactPiece / 16);
     const uint4* sK = reinterpret_cast<const uint4*>(it.pagesK + src_off);
     const uint4* sV = reinterpret_cast<const uint4*>(it.pagesV + src_off);
+    uint4* dK = reinterpret_cast<uint4*>(it.viewK + dst_off);
+    uint4* dV = reinterpret_cast<uint4*>(it.viewV + dst_off);
 #pragma unroll
     for (int r = 0; r < kPer; ++r) {
       const int64_t i = g0 + threadIdx.x + r * 256;
-      dK[r] = nullptr;
       if (i < n) {
         k[r] = ld_stream(sK + i);
         v[r] = ld_stream(sV + i);
-        dK[r] = reinterpret_cast<uint4*>(it.viewK + dst_off) + i;
-        dV[r] = reinterpret_cast<uint4*>(it.viewV + dst_off) + i;
       }
     }
-  } else {
 #pragma unroll
     for (int r = 0; r < kPer; ++r) {
-      const int64_t gi = threadIdx.x + r * 256;          // granule of this CTA's G units
-      dK[r] = nullptr;
-      int64_t src_off, dst_off;
-      if (gi < G * n && unit_offsets(a, it, blk * G + (int)(gi / n), src_off, dst_off)) {
-        const int64_t i = gi - (gi / n) * n;
-        k[r] = ld_stream(reinterpret_cast<const uint4*>(it.pagesK + src_off) + i);
-        v[r] = ld_stream(reinterpret_cast<const uint4*>(it.pagesV + src_off) + i);
-        dK[r] = reinterpret_cast<uint4*>(it.viewK + dst_off) + i;
-        dV[r] = reinterpret_cast<uint4*>(it.viewV + dst_off) + i;
+      const int64_t i = g0 + threadIdx.x + r * 256;
+      if (i < n) {
+        st_v4(dK + i, k[r]);
+        st_v4(dV + i, v[r]);
       }
+    }
+    return;
+  }
+  uint4* dK[kPer];
+  uint4* dV[kPer];
+#pragma unroll
+  for (int r = 0; r < kPer; ++r) {
+    const int64_t gi = threadIdx.x + r * 256;            // granule of this CTA's G units
+    dK[r] = nullptr;
+    int64_t src_off, dst_off;
+    if (gi < G * n && unit_offsets(a, it, blk * G + (int)(gi / n), src_off, dst_off)) {
+      const int64_t i = gi - (gi / n) * n;
+      k[r] = ld_stream(reinterpret_cast<const uint4*>(it.pagesK + src_off) + i);
+      v[r] = ld_stream(reinterpret_cast<const uint4*>(it.pagesV + src_off) + i);
+      dK[r] = reinterpret_cast<uint4*>(it.viewK + dst_off) + i;
+      dV[r] = reinterpret_cast<uint4*>(it.viewV + dst_off) + i;
     }
   }
 #pragma unroll
