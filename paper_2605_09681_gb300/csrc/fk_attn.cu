@@ -277,12 +277,19 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
   AttnBarriers* bar = reinterpret_cast<AttnBarriers*>(smem + Lay::kOffBar);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int hi = blockIdx.x / a.n_qtiles;
-  const int q0 = (blockIdx.x - hi * a.n_qtiles) * (2 * kAttnBM);
+  // CTA = (head slot, pair of query tiles, key split).  Split `split` of kv_splits covers key
+  // tiles [j0, j1) of the head: the CTA sees it as a head of nk keys starting at row0.
+  const int split = blockIdx.x % a.kv_splits;
+  const int rest = blockIdx.x / a.kv_splits;
+  const int hi = rest / a.n_qtiles;
+  const int q0 = (rest - hi * a.n_qtiles) * (2 * kAttnBM);
   const int head = a.head_of[hi];
-  const int nk = a.n_keys[head];
-  const int row0 = a.row_base[head];
-  const int nt = (nk + kAttnBN - 1) / kAttnBN;
+  const int nk_head = a.n_keys[head];
+  const int nt_head = (nk_head + kAttnBN - 1) / kAttnBN;
+  const int j0 = split * nt_head / a.kv_splits, j1 = (split + 1) * nt_head / a.kv_splits;
+  const int nk = min(nk_head, j1 * kAttnBN) - j0 * kAttnBN;
+  const int row0 = a.row_base[head] + j0 * kAttnBN;
+  const int nt = j1 - j0;
 
   if (threadIdx.x == 0) {
     mbar_init(&bar->q_full, 1);
@@ -524,7 +531,25 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
       if (lane == 0) mbar_arrive(&bar->p_full[t]);
     }
     // ---------------------------------------------------------------- epilogue
-    if (ok && warp_wait(&bar->o_done, 0, bar, a.status)) {
+    if (ok && a.kv_splits > 1 && warp_wait(&bar->o_done, 0, bar, a.status)) {
+      // one key split: unnormalised O and the row's (m, l), merged by merge_kernel
+      tc_fence_after();
+      const int q = q0 + t * kAttnBM + row;
+      const int64_t slot = ((int64_t)split * a.Nq + q) * a.H + head;
+      float* prow = a.part_o + slot * D;
+#pragma unroll
+      for (int c = 0; c < D / 32; ++c) {
+        uint32_t o[32];
+        FK_TMEM_LD32(tO + c * 32, o);
+        tmem_wait_ld();
+        if (q < a.Nq) {
+#pragma unroll
+          for (int e = 0; e < 32; e += 4)
+            *reinterpret_cast<uint4*>(prow + c * 32 + e) = make_uint4(o[e], o[e + 1], o[e + 2], o[e + 3]);
+        }
+      }
+      if (q < a.Nq) a.part_ml[slot] = make_float2(m, l);
+    } else if (ok && warp_wait(&bar->o_done, 0, bar, a.status)) {
       tc_fence_after();
       const float inv = 1.0f / l;
       const int q = q0 + t * kAttnBM + row;
@@ -789,6 +814,47 @@ cudaError_t launch_head_profile(int head_dim, const CUtensorMap& tmQ, const CUte
   return cudaGetLastError();
 }
 
+namespace {
+
+// Merge of the key splits of one query row and head (one warp): with M = max_s m_s (log2
+// domain), O = sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M) l_s, stored as bf16.
+template <int D>
+__global__ void __launch_bounds__(256) merge_kernel(const float* part_o, const float2* part_ml,
+                                                    bf16* O, int Nq, int H, int splits) {
+  constexpr int kPer = D / 32;
+  const int64_t w = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (w >= (int64_t)Nq * H) return;
+  float M = -INFINITY;
+  for (int sp = 0; sp < splits; ++sp) M = fmaxf(M, part_ml[sp * (int64_t)Nq * H + w].x);
+  float L = 0.0f, acc[kPer];
+#pragma unroll
+  for (int d = 0; d < kPer; ++d) acc[d] = 0.0f;
+  for (int sp = 0; sp < splits; ++sp) {
+    const int64_t slot = sp * (int64_t)Nq * H + w;
+    const float2 ml = part_ml[slot];
+    const float wgt = fast_exp2(ml.x - M);
+    L = fmaf(wgt, ml.y, L);
+    const float* src = part_o + slot * D + lane * kPer;
+#pragma unroll
+    for (int d = 0; d < kPer; ++d) acc[d] = fmaf(wgt, src[d], acc[d]);
+  }
+  const float inv = 1.0f / L;
+  bf16* dst = O + w * D + lane * kPer;
+#pragma unroll
+  for (int d = 0; d < kPer; d += 2)
+    *reinterpret_cast<uint32_t*>(dst + d) = pack_bf16(acc[d] * inv, acc[d + 1] * inv);
+}
+
+}  // namespace
+
+void launch_merge(int head_dim, const AttnArgs& a, cudaStream_t s) {
+  const int64_t warps = (int64_t)a.Nq * a.H;
+  const unsigned grid = (unsigned)((warps * 32 + 255) / 256);
+  if (head_dim == 128) merge_kernel<128><<<grid, 256, 0, s>>>(a.part_o, a.part_ml, a.O, a.Nq, a.H, a.kv_splits);
+  else merge_kernel<64><<<grid, 256, 0, s>>>(a.part_o, a.part_ml, a.O, a.Nq, a.H, a.kv_splits);
+}
+
 cudaError_t attention_prepare(int head_dim) {
   if (head_dim == 128)
     return cudaFuncSetAttribute(attn_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -799,7 +865,7 @@ cudaError_t attention_prepare(int head_dim) {
 
 void launch_attention(int head_dim, const CUtensorMap& tmQ, const CUtensorMap& tmK,
                       const CUtensorMap& tmV, const AttnArgs& a, cudaStream_t s) {
-  const unsigned grid = (unsigned)(a.n_qtiles * a.H);
+  const unsigned grid = (unsigned)(a.n_qtiles * a.H * a.kv_splits);
   if (head_dim == 128)
     attn_kernel<128><<<grid, kAttnThreads, Layout<128>::kSmem, s>>>(tmQ, tmK, tmV, a);
   else

@@ -21,6 +21,7 @@
 #include <cstring>
 #include <mutex>
 #include <new>
+#include <queue>
 #include <vector>
 
 #include <cudaTypedefs.h>
@@ -87,6 +88,37 @@ bool get_encode() {
 
 int64_t round_up(int64_t x, int64_t m) { return (x + m - 1) / m * m; }
 
+// Key splits of one attention launch.  The CTAs (one per SM) are dispatched longest first;
+// the makespan on n_sms SMs is estimated greedily in units of key tiles (plus a fixed cost
+// per CTA), without and with 2 key splits (plus the merge pass); equal-length heads whose CTAs
+// fill 1.5 waves are where the split pays.
+int choose_kv_splits(int n_sms, int n_qtiles, int CF, int H, int D, const int* n_keys) {
+  const double kOverheadTiles = 3.0, kTileUs = 1.65, kHbmBytesPerUs = 6.0e6;
+  auto makespan = [&](int sp) {
+    std::vector<double> d;
+    for (int hd = 0; hd < H; ++hd) {
+      const int nt = (n_keys[hd] + kAttnBN - 1) / kAttnBN;
+      if (nt < sp) return 1e30;
+      for (int q = 0; q < n_qtiles; ++q)
+        for (int k = 0; k < sp; ++k) d.push_back((double)((k + 1) * nt / sp - k * nt / sp) + kOverheadTiles);
+    }
+    std::sort(d.begin(), d.end(), std::greater<double>());
+    std::priority_queue<double, std::vector<double>, std::greater<double>> load;
+    for (int i = 0; i < n_sms; ++i) load.push(0.0);
+    double span = 0.0;
+    for (double x : d) {
+      const double t = load.top() + x;
+      load.pop();
+      load.push(t);
+      span = std::max(span, t);
+    }
+    return span;
+  };
+  const double merge_tiles =
+      ((double)kMaxKvSplits * CF * H * D * 4 + (double)CF * H * D * 2) / kHbmBytesPerUs / kTileUs;
+  return makespan(2) + merge_tiles < 0.95 * makespan(1) ? 2 : 1;
+}
+
 }  // namespace
 
 struct fk_handle {
@@ -118,6 +150,12 @@ struct fk_handle {
   int64_t stage_frames = 0;        // frames one K/V staging buffer holds
   cudaStream_t copy_stream = nullptr;
   bool host_overlap = false;
+  // attention key splits: scratch for split outputs, SM count, last decision per layer
+  float* part_o = nullptr;
+  float2* part_ml = nullptr;
+  int n_sms = 0;
+  std::vector<std::vector<int>> split_keys;   // [L]: key counts the cached decision was made for
+  std::vector<int> split_choice;              // [L]
   ScoreItem* d_score_items = nullptr;
   SelectTarget* d_targets = nullptr;
   CompactItem* d_compact_items = nullptr;
@@ -669,6 +707,18 @@ fk_status fk_create(const fk_config* cfg, fk_handle** out) {
   }
   if ((st = dev_alloc(h, chunk_bytes, &p)) != FK_OK) return fail(st);
   h->stage_o = static_cast<bf16*>(p);
+  if ((st = dev_alloc(h, (size_t)kMaxKvSplits * h->CF * h->H * h->D * sizeof(float), &p)) != FK_OK)
+    return fail(st);
+  h->part_o = static_cast<float*>(p);
+  if ((st = dev_alloc(h, (size_t)kMaxKvSplits * h->CF * h->H * sizeof(float2), &p)) != FK_OK)
+    return fail(st);
+  h->part_ml = static_cast<float2*>(p);
+  if (cudaDeviceGetAttribute(&h->n_sms, cudaDevAttrMultiProcessorCount, h->dev) != cudaSuccess) {
+    cudaGetLastError();
+    return fail(FK_ERR_CUDA);
+  }
+  h->split_keys.assign(h->L, {});
+  h->split_choice.assign(h->L, 1);
   h->stage_frames = h->C;
   for (Staging* sg : {&h->st_kv, &h->st_q})
     for (int sl = 0; sl < 2; ++sl)
@@ -990,10 +1040,21 @@ fk_status fk_attend(fk_handle* h, int layer, const void* Q, void* O, void* strea
   std::stable_sort(order.begin(), order.end(),
                    [&](int x, int y) { return a.n_keys[x] > a.n_keys[y]; });
   for (int i = 0; i < h->H; ++i) a.head_of[i] = order[i];
+  std::vector<int> keys(a.n_keys, a.n_keys + h->H);
+  if (keys != h->split_keys[layer]) {
+    h->split_choice[layer] = choose_kv_splits(h->n_sms, a.n_qtiles, h->CF, h->H, h->D, a.n_keys);
+    h->split_keys[layer] = keys;
+  }
+  a.kv_splits = h->split_choice[layer];
+  a.part_o = h->part_o;
+  a.part_ml = h->part_ml;
   const int D = h->D;
-  if ((st = launch(h, s, FK_KERNEL_ATTEND,
-                   [&] { launch_attention(D, h->tmQ[qm], h->tmK, h->tmV, a, s); })) != FK_OK)
+  if ((st = launch(h, s, FK_KERNEL_ATTEND, [&] {
+         launch_attention(D, h->tmQ[qm], h->tmK, h->tmV, a, s);
+         if (a.kv_splits > 1) launch_merge(D, a, s);
+       })) != FK_OK)
     return st;
+  if (a.kv_splits > 1) h->launches++;   // the merge pass
   if (slot >= 0) FK_CUDA(cudaEventRecord(h->st_q.freed[slot], s));
   if (copy_back) FK_CUDA(cudaMemcpyAsync(O, o, bytes, cudaMemcpyDeviceToHost, s));
   return FK_OK;

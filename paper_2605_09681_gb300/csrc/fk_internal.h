@@ -158,6 +158,9 @@ struct AttnArgs {
   int n_qtiles;
   float scale_log2;             // log2(e) / sqrt(D)
   int* status;
+  int kv_splits;                // key splits per (head, query-tile pair): 1, or 2 with a merge
+  float* part_o;                // [kv_splits][Nq][H][D] unnormalised split outputs (kv_splits > 1)
+  float2* part_ml;              // [kv_splits][Nq][H] {running max (log2 domain), row sum}
   int head_of[kMaxHeads];       // CTA order: head index of the i-th (longest-first) head
   int row_base[kMaxHeads];      // first row of the head's packed view in the view arena
   int n_keys[kMaxHeads];        // keys the head attends to
@@ -166,6 +169,9 @@ struct AttnArgs {
 void launch_attention(int head_dim, const CUtensorMap& tmQ, const CUtensorMap& tmK,
                       const CUtensorMap& tmV, const AttnArgs& a, cudaStream_t s);
 cudaError_t attention_prepare(int head_dim);   // sets the dynamic shared-memory limit
+// combine the key splits of every (row, head) into O (bf16)
+void launch_merge(int head_dim, const AttnArgs& a, cudaStream_t s);
+constexpr int kMaxKvSplits = 2;
 
 // ------------------------------------------------------------------ head profiling (Eq. 1)
 struct ProfArgs {
