@@ -260,7 +260,9 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   return *reinterpret_cast<const uint32_t*>(&p);
 }
 
-template <int D>
+// kSplit: a launch with key splits (kv_splits > 1); the unsplit instantiation carries none of
+// the split bookkeeping.
+template <int D, bool kSplit>
 __global__ void __launch_bounds__(kAttnThreads, 1)
 attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
             const __grid_constant__ CUtensorMap tmV, const AttnArgs a) {
@@ -279,17 +281,20 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   // CTA = (head slot, pair of query tiles, key split).  Split `split` of kv_splits covers key
   // tiles [j0, j1) of the head: the CTA sees it as a head of nk keys starting at row0.
-  const int split = blockIdx.x % a.kv_splits;
-  const int rest = blockIdx.x / a.kv_splits;
+  const int split = kSplit ? blockIdx.x % a.kv_splits : 0;
+  const int rest = kSplit ? blockIdx.x / a.kv_splits : blockIdx.x;
   const int hi = rest / a.n_qtiles;
   const int q0 = (rest - hi * a.n_qtiles) * (2 * kAttnBM);
   const int head = a.head_of[hi];
-  const int nk_head = a.n_keys[head];
-  const int nt_head = (nk_head + kAttnBN - 1) / kAttnBN;
-  const int j0 = split * nt_head / a.kv_splits, j1 = (split + 1) * nt_head / a.kv_splits;
-  const int nk = min(nk_head, j1 * kAttnBN) - j0 * kAttnBN;
-  const int row0 = a.row_base[head] + j0 * kAttnBN;
-  const int nt = j1 - j0;
+  int nk = a.n_keys[head];
+  int row0 = a.row_base[head];
+  if constexpr (kSplit) {
+    const int nt_head = (nk + kAttnBN - 1) / kAttnBN;
+    const int j0 = split * nt_head / a.kv_splits, j1 = (split + 1) * nt_head / a.kv_splits;
+    nk = min(nk, j1 * kAttnBN) - j0 * kAttnBN;
+    row0 += j0 * kAttnBN;
+  }
+  const int nt = (nk + kAttnBN - 1) / kAttnBN;
 
   if (threadIdx.x == 0) {
     mbar_init(&bar->q_full, 1);
@@ -531,7 +536,7 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
       if (lane == 0) mbar_arrive(&bar->p_full[t]);
     }
     // ---------------------------------------------------------------- epilogue
-    if (ok && a.kv_splits > 1 && warp_wait(&bar->o_done, 0, bar, a.status)) {
+    if (kSplit && ok && warp_wait(&bar->o_done, 0, bar, a.status)) {
       // one key split: unnormalised O and the row's (m, l), merged by merge_kernel
       tc_fence_after();
       const int q = q0 + t * kAttnBM + row;
@@ -549,7 +554,7 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
         }
       }
       if (q < a.Nq) a.part_ml[slot] = make_float2(m, l);
-    } else if (ok && warp_wait(&bar->o_done, 0, bar, a.status)) {
+    } else if (!kSplit && ok && warp_wait(&bar->o_done, 0, bar, a.status)) {
       tc_fence_after();
       const float inv = 1.0f / l;
       const int q = q0 + t * kAttnBM + row;
@@ -856,20 +861,31 @@ void launch_merge(int head_dim, const AttnArgs& a, cudaStream_t s) {
 }
 
 cudaError_t attention_prepare(int head_dim) {
-  if (head_dim == 128)
-    return cudaFuncSetAttribute(attn_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  cudaError_t e;
+  if (head_dim == 128) {
+    e = cudaFuncSetAttribute(attn_kernel<128, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             Layout<128>::kSmem);
+    if (e != cudaSuccess) return e;
+    return cudaFuncSetAttribute(attn_kernel<128, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 Layout<128>::kSmem);
-  return cudaFuncSetAttribute(attn_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  }
+  e = cudaFuncSetAttribute(attn_kernel<64, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           Layout<64>::kSmem);
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(attn_kernel<64, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                               Layout<64>::kSmem);
 }
 
 void launch_attention(int head_dim, const CUtensorMap& tmQ, const CUtensorMap& tmK,
                       const CUtensorMap& tmV, const AttnArgs& a, cudaStream_t s) {
   const unsigned grid = (unsigned)(a.n_qtiles * a.H * a.kv_splits);
-  if (head_dim == 128)
-    attn_kernel<128><<<grid, kAttnThreads, Layout<128>::kSmem, s>>>(tmQ, tmK, tmV, a);
-  else
-    attn_kernel<64><<<grid, kAttnThreads, Layout<64>::kSmem, s>>>(tmQ, tmK, tmV, a);
+  if (head_dim == 128) {
+    if (a.kv_splits > 1) attn_kernel<128, true><<<grid, kAttnThreads, Layout<128>::kSmem, s>>>(tmQ, tmK, tmV, a);
+    else attn_kernel<128, false><<<grid, kAttnThreads, Layout<128>::kSmem, s>>>(tmQ, tmK, tmV, a);
+  } else {
+    if (a.kv_splits > 1) attn_kernel<64, true><<<grid, kAttnThreads, Layout<64>::kSmem, s>>>(tmQ, tmK, tmV, a);
+    else attn_kernel<64, false><<<grid, kAttnThreads, Layout<64>::kSmem, s>>>(tmQ, tmK, tmV, a);
+  }
 }
 
 }  // namespace fk
