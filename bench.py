@@ -538,7 +538,7 @@ def run_stack(local_rank):
 # is reported only while that source is unchanged.
 NCU_TRAFFIC = {
     "480p_layer": {
-        "attend": ("fk_attn.cu", "fc08b6769224", 122271744),
+        "attend": ("fk_attn.cu", "ab1645e4ffd2", 121940224),
         "compact": ("fk_copy.cu", "7bff156f176c", 76305408),
         "score": ("fk_score.cu", "cb7cdc3bafa2", 43160576),
     },
