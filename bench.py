@@ -539,7 +539,7 @@ def run_stack(local_rank):
 NCU_TRAFFIC = {
     "480p_layer": {
         "attend": ("fk_attn.cu", "ab1645e4ffd2", 121940224),
-        "compact": ("fk_copy.cu", "7bff156f176c", 76305408),
+        "compact": ("fk_copy.cu", "b4908ca5adab", 76899072),
         "score": ("fk_score.cu", "cb7cdc3bafa2", 43160576),
     },
 }
