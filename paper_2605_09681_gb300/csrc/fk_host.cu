@@ -14,7 +14,8 @@
 //                frame f lives in slot f (f < S) or S + (f - S) mod cap_nonsink.
 //   scores       fp32 [target][ring_slots][n]; kept lists int32 [target][kmax];
 //                int64 scoring sums (scratch); status word;
-//                host-input staging.
+//                host staging (two slots of K, V and Q; O) and the attention key-split
+//                scratch (fp32 partial outputs and row statistics of two splits).
 #include <algorithm>
 #include <cmath>
 #include <cstdio>

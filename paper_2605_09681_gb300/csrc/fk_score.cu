@@ -1,19 +1,21 @@
-// Segment-wise similarity scoring and BottomK selection (Sec. 4.3, Eq. 3) in one launch.
+// Segment-wise similarity scoring (Sec. 4.3, Eq. 3) and BottomK selection: the scoring kernel,
+// then the selection kernel chained to it by programmatic dependent launch.
 //
 // Work unit: one frame-chunk, i.e. 32 tokens of one segment of one scored (layer, head) in
 // one frame of the run.  The units of all scored heads, ordered (layer, item, segment,
 // token chunk, frame), are split into equal contiguous ranges, one per CTA of a persistent
 // grid, so every CTA streams the same number of key bytes (no partial last wave).  A range
-// walks consecutive frames of a token chunk through a cp.async shared-memory ring, loading
-// one extra frame at its start as the partner of its first pair; every other key byte is
+// walks consecutive frames of a token chunk; thread 0 streams each frame-chunk (8 KB
+// contiguous) with one bulk copy into a shared-memory ring completed on mbarriers, loading one
+// extra frame at the range's start as the partner of its first pair; every other key byte is
 // read once.  Per token it forms the score-contract quantities (fp32 channel dot in a fixed
 // fma/butterfly order, scaled by 2^24 and truncated to int64, carried as two exact int32
 // halves): the squared norm n_p(t) and the dot d_p(t-1, t).  Warp sums go into shared-memory
 // int32 accumulators (at most 32 tokens per run, so no overflow) and each run adds them as
-// int64 into the target's global int64 sums (exact integer adds, so the order is free).  The
-// CTA whose run completes a selection target's last frame-chunks (counted with a global
-// atomic) finishes s = D / sqrt(N_t N_{t+1}) in IEEE double, stores the fp32 scores per frame
-// slot, ranks the scoreable candidates by (score, segment id) and stream-compacts the kept
+// int64 into the target's global int64 sums (exact integer adds, so the order is free); no
+// CTA waits for another.  The selection kernel (one CTA per target) then finishes
+// s = D / sqrt(N_t N_{t+1}) in IEEE double, stores the fp32 scores per frame slot, clears the
+// sums, ranks the scoreable candidates by (score, segment id) and stream-compacts the kept
 // segment ids with warp ballots and prefix sums.
 #include <algorithm>
 #include <mutex>
