@@ -540,7 +540,7 @@ NCU_TRAFFIC = {
     "480p_layer": {
         "attend": ("fk_attn.cu", "ab1645e4ffd2", 121940224),
         "compact": ("fk_copy.cu", "b4908ca5adab", 76899072),
-        "score": ("fk_score.cu", "cd1c927e77bd", 43160576),
+        "score": ("fk_score.cu", "b939942305b6", 43160576),
     },
 }
 
