@@ -266,6 +266,7 @@ def run_fk(args, rank, world, local_rank):
     e_begin.record(stream)
     for i in range(args.steps):
         step(i, host=True)
+    cache.wait_outputs()                 # every step's output copy-back inside the interval
     e_end.record(stream)
     torch.cuda.synchronize()
     barrier(world)
@@ -321,8 +322,11 @@ def run_fk(args, rank, world, local_rank):
         "gpu_launches": int(launches),
         "e2e": {"value": round(e2e_value, 3), "unit": "TFLOP/s", "ms_per_step": round(e2e_ms / args.steps, 4),
                 "h2d_bytes_per_step": 3 * nbytes, "d2h_bytes_per_step": nbytes,
-                "note": "pinned host K, V, Q in and O out every step through the C ABI; host-input "
-                        "copies overlap queued work (fk_set_host_overlap); one continuous interval"},
+                "note": "pinned host K, V, Q in and O out every step through the C ABI; host copies "
+                        "overlap queued work (fk_set_host_overlap, outputs joined by fk_wait_outputs "
+                        "before the end event); one continuous interval over all steps",
+                "l2": "not flushed between steps (each step touches ~0.4 GB of inputs, views and "
+                      "pages, more than the L2); the device-timed value flushes before every step"},
         "roofline": {
             "bound": "tensor", "kernel": "attention (tcgen05)", "achieved": round(attn_tflops, 2),
             "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",

@@ -18,10 +18,10 @@
  *   - Tensors K, V, Q, O are bf16, token-major [tokens][n_heads][head_dim], row-major
  *     and contiguous ("the [seq, heads, dim] layout"), 16-byte aligned.
  *   - A tensor pointer may be device memory or host memory (pinned or pageable).  Host
- *     inputs are copied into library-owned device staging buffers on `stream` (or on the
- *     handle's copy stream, see fk_set_host_overlap); a host output is written by an
- *     asynchronous device-to-host copy on `stream`, so the caller synchronizes `stream`
- *     before reading it.  Caller-owned device inputs must
+ *     inputs are copied into library-owned device staging buffers on `stream`; a host output
+ *     is written by an asynchronous device-to-host copy on `stream`, so the caller
+ *     synchronizes `stream` before reading it (with fk_set_host_overlap on, the copies run on
+ *     the handle's copy streams instead; see there).  Caller-owned device inputs must
  *     stay valid until the work queued on `stream` by the call has run.
  *   - `stream` is a cudaStream_t passed as void* (NULL = the legacy default stream).
  *   - Frames are numbered globally from 0 in append order.  The history is every frame
@@ -198,16 +198,23 @@ FK_API fk_status fk_profile_enable(fk_handle* h, int on);
 FK_API fk_status fk_profile_read(fk_handle* h, int kind, double* total_ms, int64_t* launches);
 FK_API fk_status fk_profile_reset(fk_handle* h);
 
-/* Host-input overlap.  Off (the default): a host input (K, V of fk_append_chunk /
- * fk_set_current, Q of fk_attend) is copied into staging on `stream`, in call order.  On: it is
- * copied at once on a copy stream owned by the handle, into one of two staging slots per
- * input kind, so the copy overlaps the work already queued on `stream`; the kernel that reads
- * it waits for the copy, and the next copy into a slot waits for the kernel that read it
- * before.  With overlap on, the caller guarantees that a host input is final when the call
- * is made (written by the CPU, not by device work still pending on any stream) and unchanged
- * until `stream` has run the call's work.  Host outputs (O) are always copied on `stream`.
- * FK_ERR_ARG for a null handle. */
+/* Host-transfer overlap.  Off (the default): a host input (K, V of fk_append_chunk /
+ * fk_set_current, Q of fk_attend) is copied into staging on `stream`, in call order, and a
+ * host output (O of fk_attend) is copied back on `stream`.  On: a host input is copied at once
+ * on a copy stream owned by the handle, into one of two staging slots per input kind, so the
+ * copy overlaps the work already queued on `stream` (the kernel that reads it waits for the
+ * copy; the next copy into a slot waits for the kernel that read it before); and a host
+ * output is copied back on a second copy stream of the handle after the attention kernel, so
+ * it overlaps the work queued after the call.  With overlap on, the caller guarantees that a
+ * host input is final when the call is made (written by the CPU, not by device work still
+ * pending on any stream) and unchanged until `stream` has run the call's work, and reads a
+ * host output only after fk_wait_outputs (or fk_sync_status) on `stream` and a
+ * synchronization of `stream`.  FK_ERR_ARG for a null handle. */
 FK_API fk_status fk_set_host_overlap(fk_handle* h, int on);
+
+/* Make `stream` wait for every host-output copy still pending on the handle's copy stream
+ * (host overlap on); a no-op otherwise.  FK_ERR_ARG for a null handle. */
+FK_API fk_status fk_wait_outputs(fk_handle* h, void* stream);
 
 /* Failure-detection self-test (no counterpart in the paper): launches a one-thread kernel
  * that waits, with the same bounded-wait primitive as the hot-path kernels, on an mbarrier

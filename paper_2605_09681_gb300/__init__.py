@@ -234,9 +234,14 @@ class ForcingKVCache:
         _check(self._lib.fk_wait_selftest(self._h, int(limit_us), _stream(stream)), "fk_wait_selftest")
 
     def set_host_overlap(self, on: bool = True) -> None:
-        """Copy host inputs on the handle's copy stream as soon as a call is made (see
-        fk_set_host_overlap): the caller promises host inputs are final at call time."""
+        """Overlap host transfers with queued work (see fk_set_host_overlap): host inputs must
+        be final at call time; host outputs are complete after wait_outputs() (or
+        sync_status()) and a synchronization of the stream."""
         _check(self._lib.fk_set_host_overlap(self._h, 1 if on else 0), "fk_set_host_overlap")
+
+    def wait_outputs(self, stream=None) -> None:
+        """Make the stream wait for pending host-output copies (fk_wait_outputs)."""
+        _check(self._lib.fk_wait_outputs(self._h, _stream(stream)), "fk_wait_outputs")
 
     def launch_count(self) -> int:
         return int(self._lib.fk_launch_count(self._h))

@@ -24,7 +24,7 @@ EXPORTS = [
     "fk_key_count", "fk_get_kept", "fk_get_scores", "fk_sync_status", "fk_profile_enable",
     "fk_profile_read", "fk_profile_reset", "fk_launch_count", "fk_status_str", "fk_abi_version",
     "fk_segment_scores_noalloc", "fk_head_profile", "fk_classify_heads", "fk_set_host_overlap",
-    "fk_wait_selftest",
+    "fk_wait_selftest", "fk_wait_outputs",
 ]
 
 
@@ -85,6 +85,7 @@ def load(path: str | None = None) -> ctypes.CDLL:
         "fk_launch_count": (ctypes.c_int64, [vp]),
         "fk_set_host_overlap": (st, [vp, i32]),
         "fk_wait_selftest": (st, [vp, i32, vp]),
+        "fk_wait_outputs": (st, [vp, vp]),
         "fk_status_str": (cp, [i32]),
         "fk_abi_version": (i32, []),
         "fk_segment_scores_noalloc": (st, [vp, i32, i32, i32, i32, vp, vp]),

@@ -147,7 +147,12 @@ struct fk_handle {
   // host-input staging: two slots per kind (K with V; Q), each with a ready event (copy done)
   // and a freed event (the kernel that read the slot has run); optional copy stream
   Staging st_kv, st_q;
-  bf16* stage_o = nullptr;
+  // output staging: two slots; with host overlap on, copied back on copy_out_stream
+  bf16* stage_o[2] = {};
+  cudaEvent_t o_ready[2] = {}, o_copied[2] = {};
+  int o_slot = 0;
+  bool o_pending[2] = {};
+  cudaStream_t copy_out_stream = nullptr;
   int64_t stage_frames = 0;        // frames one K/V staging buffer holds
   cudaStream_t copy_stream = nullptr;
   bool host_overlap = false;
@@ -526,6 +531,15 @@ fk_status fk_set_host_overlap(fk_handle* h, int on) {
   return FK_OK;
 }
 
+fk_status fk_wait_outputs(fk_handle* h, void* stream) {
+  if (!h) return FK_ERR_ARG;
+  FK_CUDA(cudaSetDevice(h->dev));
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  for (int sl = 0; sl < 2; ++sl)
+    if (h->o_pending[sl]) FK_CUDA(cudaStreamWaitEvent(s, h->o_copied[sl], 0));
+  return FK_OK;
+}
+
 int fk_abi_version(void) { return 2; }
 
 const char* fk_status_str(fk_status s) {
@@ -706,8 +720,15 @@ fk_status fk_create(const fk_config* cfg, fk_handle** out) {
     if ((st = dev_alloc(h, chunk_bytes, &p)) != FK_OK) return fail(st);
     h->st_q.buf[sl][0] = static_cast<bf16*>(p);
   }
-  if ((st = dev_alloc(h, chunk_bytes, &p)) != FK_OK) return fail(st);
-  h->stage_o = static_cast<bf16*>(p);
+  for (int sl = 0; sl < 2; ++sl) {
+    if ((st = dev_alloc(h, chunk_bytes, &p)) != FK_OK) return fail(st);
+    h->stage_o[sl] = static_cast<bf16*>(p);
+    if (cudaEventCreateWithFlags(&h->o_ready[sl], cudaEventDisableTiming) != cudaSuccess ||
+        cudaEventCreateWithFlags(&h->o_copied[sl], cudaEventDisableTiming) != cudaSuccess) {
+      cudaGetLastError();
+      return fail(FK_ERR_CUDA);
+    }
+  }
   if ((st = dev_alloc(h, (size_t)kMaxKvSplits * h->CF * h->H * h->D * sizeof(float), &p)) != FK_OK)
     return fail(st);
   h->part_o = static_cast<float*>(p);
@@ -728,7 +749,8 @@ fk_status fk_create(const fk_config* cfg, fk_handle** out) {
         cudaGetLastError();
         return fail(FK_ERR_CUDA);
       }
-  if (cudaStreamCreateWithFlags(&h->copy_stream, cudaStreamNonBlocking) != cudaSuccess) {
+  if (cudaStreamCreateWithFlags(&h->copy_stream, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaStreamCreateWithFlags(&h->copy_out_stream, cudaStreamNonBlocking) != cudaSuccess) {
     cudaGetLastError();
     return fail(FK_ERR_CUDA);
   }
@@ -789,6 +811,11 @@ void fk_destroy(fk_handle* h) {
       if (sg->freed[sl]) cudaEventDestroy(sg->freed[sl]);
     }
   if (h->copy_stream) cudaStreamDestroy(h->copy_stream);
+  if (h->copy_out_stream) cudaStreamDestroy(h->copy_out_stream);
+  for (int sl = 0; sl < 2; ++sl) {
+    if (h->o_ready[sl]) cudaEventDestroy(h->o_ready[sl]);
+    if (h->o_copied[sl]) cudaEventDestroy(h->o_copied[sl]);
+  }
   for (void* p : h->allocs) cudaFree(p);
   cudaGetLastError();
   delete h;
@@ -1016,7 +1043,14 @@ fk_status fk_attend(fk_handle* h, int layer, const void* Q, void* O, void* strea
   // a host output is staged and copied back on `stream` (measured faster than storing it
   // from the attention epilogue directly into pinned host memory)
   const bool copy_back = !is_device_ptr(O);
-  bf16* o = copy_back ? h->stage_o : static_cast<bf16*>(O);
+  const int osl = h->o_slot;
+  bf16* o = static_cast<bf16*>(O);
+  if (copy_back) {
+    h->o_slot ^= 1;
+    o = h->stage_o[osl];
+    // the slot's previous copy-back (two host-output calls ago) must have read it
+    if (h->o_pending[osl]) FK_CUDA(cudaStreamWaitEvent(s, h->o_copied[osl], 0));
+  }
   int qm = q == h->q_cached[0] ? 0 : q == h->q_cached[1] ? 1 : -1;
   if (qm < 0) {
     qm = h->q_next;
@@ -1057,7 +1091,18 @@ fk_status fk_attend(fk_handle* h, int layer, const void* Q, void* O, void* strea
     return st;
   if (a.kv_splits > 1) h->launches++;   // the merge pass
   if (slot >= 0) FK_CUDA(cudaEventRecord(h->st_q.freed[slot], s));
-  if (copy_back) FK_CUDA(cudaMemcpyAsync(O, o, bytes, cudaMemcpyDeviceToHost, s));
+  if (copy_back) {
+    if (h->host_overlap) {   // copy back off the caller's stream; fk_wait_outputs joins it
+      FK_CUDA(cudaEventRecord(h->o_ready[osl], s));
+      FK_CUDA(cudaStreamWaitEvent(h->copy_out_stream, h->o_ready[osl], 0));
+      FK_CUDA(cudaMemcpyAsync(O, o, bytes, cudaMemcpyDeviceToHost, h->copy_out_stream));
+      FK_CUDA(cudaEventRecord(h->o_copied[osl], h->copy_out_stream));
+      h->o_pending[osl] = true;
+    } else {
+      FK_CUDA(cudaMemcpyAsync(O, o, bytes, cudaMemcpyDeviceToHost, s));
+      h->o_pending[osl] = false;
+    }
+  }
   return FK_OK;
 }
 
@@ -1142,6 +1187,8 @@ fk_status fk_sync_status(fk_handle* h, void* stream) {
   if (!h) return FK_ERR_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   FK_CUDA(cudaSetDevice(h->dev));
+  fk_status st = fk_wait_outputs(h, stream);   // overlapped output copies complete too
+  if (st != FK_OK) return st;
   int word = 0;
   FK_CUDA(cudaMemcpyAsync(&word, h->status, sizeof(int), cudaMemcpyDeviceToHost, s));
   FK_CUDA(cudaStreamSynchronize(s));

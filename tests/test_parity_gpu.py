@@ -323,7 +323,8 @@ def test_host_inputs_and_overlap_match_device_inputs():
                     outs.append(Oh)
                     if mode == "host":
                         torch.cuda.synchronize()
-            torch.cuda.synchronize()
+            cache.wait_outputs()
+            torch.cuda.current_stream().synchronize()   # stream order alone covers the outputs
             assert cache.sync_status() == 0
             runs[mode] = [W.bf16_bits_to_f32(o) if isinstance(o, np.ndarray) else o.float().cpu().numpy()
                           for o in outs]
