@@ -228,6 +228,57 @@ def attention_fp64(Q: np.ndarray, K: np.ndarray, V: np.ndarray, row_block: int =
 
 
 # --------------------------------------------------------------------------------------
+# FP8 attention (App. on quantization: FP8 attention on the compressed cache).  The paper
+# names the technique only; the reading taken here: Q K^T on OCP FP8 E4M3 operands, P V
+# unquantised.  K is rounded to e4m3 unscaled (the scoring precondition |K| <= 256 keeps
+# it inside the e4m3 range, largest finite 448); each query row (token, head) is scaled
+# by a power of two 2^-e, e the smallest integer with max|q| <= 448 * 2^e, so scaling and
+# unscaling are exact and the only rounding is the e4m3 rounding itself.
+# --------------------------------------------------------------------------------------
+E4M3_MAX = 448.0
+E4M3_MIN_EXP = -6            # smallest normal binade 2^-6; subnormals step by 2^-9
+E4M3_MANT_BITS = 3
+
+
+def e4m3_round(x) -> np.ndarray:
+    """Nearest OCP FP8 E4M3 value of each element (ties to the even mantissa), saturating
+    to +-448; fp64 in, fp64 out.  The grid spacing in binade [2^b, 2^(b+1)) is
+    2^(max(b, -6) - 3)."""
+    x = np.asarray(x, dtype=np.float64)
+    a = np.abs(x)
+    _, ex = np.frexp(a)                          # a = m 2^ex, 0.5 <= m < 1: binade b = ex - 1
+    b = np.maximum(ex.astype(np.int64) - 1, E4M3_MIN_EXP)
+    spacing = np.ldexp(1.0, b - E4M3_MANT_BITS)
+    r = np.rint(a / spacing) * spacing           # a / spacing is exact; rint ties to even
+    r = np.minimum(r, E4M3_MAX)
+    return np.copysign(r, x)
+
+
+def q_row_exponent(amax: float) -> int:
+    """Smallest integer e with amax <= 448 * 2^e (0 for amax = 0), clamped to [-120, 120]."""
+    amax = float(amax)
+    if amax == 0.0:
+        return 0
+    m, ex = np.frexp(amax)                       # amax = m 2^ex; 448 = 0.875 * 2^9
+    e = int(ex) - 9 if m <= 0.875 else int(ex) - 8
+    return max(-120, min(120, e))
+
+
+def quantize_q_rows(Q: np.ndarray) -> tuple[np.ndarray, np.ndarray]:
+    """Per-row FP8 quantization of queries: (e4m3 values of Q_r 2^-e_r as fp64, e_r)."""
+    Q = np.asarray(Q, dtype=np.float64)
+    e = np.array([q_row_exponent(np.abs(r).max()) if r.size else 0 for r in Q], dtype=np.int64)
+    return e4m3_round(Q * np.ldexp(1.0, -e)[:, None]), e
+
+
+def attention_fp8_qk(Q: np.ndarray, K: np.ndarray, V: np.ndarray) -> np.ndarray:
+    """FP8 attention: softmax(2^e_r (Q8_r . K8) / sqrt(D)) V in fp64, with Q8, e from
+    `quantize_q_rows`, K8 = e4m3_round(K) and V as given."""
+    q8, e = quantize_q_rows(Q)
+    return attention_fp64(q8 * np.ldexp(1.0, e)[:, None], e4m3_round(K), V)
+
+
+# --------------------------------------------------------------------------------------
 # comparison selection rules (App. H, Sec. 5.3): ranking values replacing the scores
 # --------------------------------------------------------------------------------------
 _M64 = (1 << 64) - 1
@@ -317,7 +368,7 @@ class ForcingKVOracle:
                  n_sink_frames, window_frames, n_segments, keep_budget_permille,
                  select_scope="per_frame", score_source="per_head", head_is_static,
                  track_layers=None, selection="similarity", select_seed=0,
-                 static_drop_anchor=False):
+                 static_drop_anchor=False, attn_precision="bf16"):
         self.L, self.H, self.D = n_layers, n_heads, head_dim
         self.F, self.C = tokens_per_frame, frames_per_chunk
         self.S, self.W = n_sink_frames, window_frames
@@ -333,6 +384,9 @@ class ForcingKVOracle:
             raise ValueError(selection)
         self.selection, self.seed = selection, int(select_seed) & 0xFFFFFFFF
         self.keep_anchor_static = not static_drop_anchor
+        if attn_precision not in ("bf16", "fp8_qk"):
+            raise ValueError(attn_precision)
+        self.attn_precision = attn_precision
         self.static = np.asarray(head_is_static, dtype=np.uint8).reshape(n_layers, n_heads)
         self.layers = list(range(n_layers)) if track_layers is None else sorted(track_layers)
         if score_source == "layer0_pooled" and 0 not in self.layers:
@@ -351,7 +405,7 @@ class ForcingKVOracle:
                    select_scope=w.select_scope, score_source=w.score_source,
                    head_is_static=head_is_static, track_layers=track_layers,
                    selection=w.selection, select_seed=w.select_seed,
-                   static_drop_anchor=w.static_drop_anchor)
+                   static_drop_anchor=w.static_drop_anchor, attn_precision=w.attn_precision)
 
     def _push_history(self, layer, K, V):
         F = self.F
@@ -479,14 +533,16 @@ class ForcingKVOracle:
         return Ks, Vs
 
     def attend(self, layer, Q_bits, heads=None, rows=None, kept=None) -> np.ndarray:
-        """O [rows, H, D] fp64: each head's queries over its Eq. 2 / Eq. 4 key set."""
+        """O [rows, H, D] fp64: each head's queries over its Eq. 2 / Eq. 4 key set (Q K^T
+        on e4m3 operands when the attention precision is "fp8_qk")."""
         Q = _bf16_to_f32(Q_bits)
         rows = np.arange(Q.shape[0]) if rows is None else np.asarray(rows)
         heads = range(self.H) if heads is None else heads
         O = np.full((len(rows), self.H, self.D), np.nan)
         for h in heads:
             K, V = self.gather_kv(layer, h, None if kept is None else kept.get(h))
-            O[:, h, :] = attention_fp64(Q[rows, h, :], K, V)
+            att = attention_fp8_qk if self.attn_precision == "fp8_qk" else attention_fp64
+            O[:, h, :] = att(Q[rows, h, :], K, V)
         return O
 
     def view_length(self, layer, head) -> int:

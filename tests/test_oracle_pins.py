@@ -463,3 +463,83 @@ def test_rule_workloads_key_sets():
         for h in range(4):
             n = orc.view_length(0, h)
             assert n == (want_static if hm[0, h] else want_dynamic), (w.name, h, n)
+
+
+# ---------------------------------------------------------------- FP8 attention (e4m3 Q K^T)
+def _e4m3_codes():
+    """Every finite OCP FP8 E4M3 value, decoded from its bit fields: sign, 4 exponent bits
+    with bias 7 (0 = subnormal, m 2^-9), 3 mantissa bits; S.1111.111 is NaN."""
+    vals = []
+    for code in range(256):
+        s, e, m = code >> 7, (code >> 3) & 15, code & 7
+        if e == 15 and m == 7:
+            continue
+        v = m * 2.0 ** -9 if e == 0 else (1 + m / 8) * 2.0 ** (e - 7)
+        vals.append(-v if s else v)
+    return np.array(vals)
+
+
+def test_e4m3_grid_round_trips():
+    v = _e4m3_codes()
+    assert v.max() == 448.0 and np.min(np.abs(v[v != 0])) == 2.0 ** -9
+    assert np.array_equal(O.e4m3_round(v), v)
+
+
+def test_e4m3_midpoints_round_to_even_mantissa():
+    pos = np.unique(_e4m3_codes()[_e4m3_codes() >= 0])
+    mid = (pos[:-1] + pos[1:]) / 2
+    got = O.e4m3_round(mid)
+    # the even neighbour: mantissa field (value / spacing) even in the neighbours' binade
+    for lo, hi, g in zip(pos[:-1], pos[1:], got):
+        spacing = hi - lo
+        even = lo if round(lo / spacing) % 2 == 0 else hi
+        assert g == even, (lo, hi, g)
+    assert np.array_equal(O.e4m3_round(-mid), -got)
+
+
+def test_e4m3_matches_torch_cast_on_every_bf16_in_range():
+    bits = np.arange(1 << 16, dtype=np.uint32)
+    f = (bits << 16).astype(np.uint32).view(np.float32)
+    f = f[np.isfinite(f) & (np.abs(f) <= 448.0)]
+    ref = torch.from_numpy(f).to(torch.float8_e4m3fn).float().numpy().astype(np.float64)
+    assert np.array_equal(O.e4m3_round(f.astype(np.float64)), ref)
+
+
+def test_e4m3_saturates():
+    assert np.array_equal(O.e4m3_round([449.0, 464.0, 1e6, -500.0]), [448.0, 448.0, 448.0, -448.0])
+
+
+def test_q_row_exponent_is_the_smallest_fitting_power():
+    rng = np.random.default_rng(5)
+    amax = np.concatenate([rng.lognormal(0, 6, 2000), [448.0, 449.0, 224.0, 896.0, 1.0, 2.0 ** -100]])
+    for a in amax:
+        e = O.q_row_exponent(a)
+        assert a <= 448.0 * 2.0 ** e and a > 448.0 * 2.0 ** (e - 1), (a, e)
+    assert (O.q_row_exponent(0.0), O.q_row_exponent(448.0), O.q_row_exponent(449.0),
+            O.q_row_exponent(1.0)) == (0, 0, 1, -8)
+
+
+def test_fp8_attention_is_exact_on_e4m3_inputs():
+    # Q rows and K already on the (row-scaled) e4m3 grid: quantization changes nothing
+    rng = np.random.default_rng(6)
+    grid = _e4m3_codes()
+    grid = grid[(np.abs(grid) >= 2.0 ** -3) & (np.abs(grid) <= 8)]
+    Q = rng.choice(grid, size=(40, 64)) * np.ldexp(1.0, rng.integers(-3, 4, size=40))[:, None]
+    K = rng.choice(grid, size=(300, 64))
+    V = rng.standard_normal((300, 64))
+    assert np.array_equal(O.attention_fp8_qk(Q, K, V), O.attention_fp64(Q, K, V))
+
+
+def test_fp8_attention_quantizes_within_e4m3_error():
+    rng = np.random.default_rng(7)
+    Q = rng.standard_normal((64, 128)) * np.ldexp(1.0, rng.integers(-6, 1, size=64))[:, None]
+    K = rng.standard_normal((500, 128))
+    V = rng.standard_normal((500, 128))
+    q8, e = O.quantize_q_rows(Q)
+    deq = q8 * np.ldexp(1.0, e)[:, None]
+    # relative rounding error of e4m3 normals <= 2^-4; every row uses the full range
+    normal = np.abs(deq) >= 2.0 ** -6 * np.ldexp(1.0, e)[:, None]
+    assert np.all(np.abs(deq - Q)[normal] <= np.abs(Q)[normal] * 2.0 ** -4 + 1e-300)
+    assert np.all(np.abs(q8).max(axis=1) >= 224.0)   # amax 2^-e in (224, 448], then rounded
+    ref, got = O.attention_fp64(Q, K, V), O.attention_fp8_qk(Q, K, V)
+    assert 1e-5 < np.abs(got - ref).max() < 0.1

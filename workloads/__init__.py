@@ -132,6 +132,7 @@ class Workload:
     selection: str = "similarity"        # "similarity" | "all" | "uniform" | "random"
     select_seed: int = 0
     static_drop_anchor: bool = False
+    attn_precision: str = "bf16"         # "bf16" | "fp8_qk" (Q K^T on e4m3 operands)
     seed: int = 0
     description: str = ""
 
@@ -223,9 +224,19 @@ RANDOM_TOKENS_480P = P480_LAYER.with_(
     description="random token pruning on the 480P layer's dynamic heads: 1092 seeded random "
                 "tokens of each history frame (70%)")
 
+# FP8 attention on the compressed cache (the paper's quantization appendix): Q K^T on e4m3.
+P480_LAYER_FP8 = P480_LAYER.with_(
+    name="480p_layer_fp8", attn_precision="fp8_qk",
+    description="the 480P layer with Q K^T on FP8 E4M3 operands (per-row power-of-two query "
+                "scales, unscaled keys), P V in bf16")
+P1080_LAYER_FP8 = P1080_LAYER.with_(
+    name="1080p_layer_fp8", attn_precision="fp8_qk",
+    description="the 1080P layer with Q K^T on FP8 E4M3 operands, P V in bf16")
+
 WORKLOADS = {w.name: w for w in (TINY, TINY_PER_FRAME, P480_LAYER, P480_STACK, ROLLING, P1080_LAYER,
                                  FULL_KV_480P, STREAMINGLLM_480P, DUMMY_FORCING_480P,
-                                 UNIFORM_TOKENS_480P, RANDOM_TOKENS_480P)}
+                                 UNIFORM_TOKENS_480P, RANDOM_TOKENS_480P, P480_LAYER_FP8,
+                                 P1080_LAYER_FP8)}
 
 
 def head_map(w: Workload) -> np.ndarray:
