@@ -353,6 +353,9 @@ def run_fk(args, rank, world, local_rank):
     cache.close()
     out["incremental"] = run_incremental(args, w, hm, local_rank, to_t(hk).to(dev), to_t(hv).to(dev),
                                          dK, dV, dQ, dO, flush, stream, world, peaks)
+    if w.head_dim == 128:
+        out["fp8_qk"] = run_fp8(args, w, hm, local_rank, to_t(hk).to(dev), to_t(hv).to(dev),
+                                dK, dV, dQ, dO, flush, stream, world, peaks, attn_ms)
     out["head_profile_480p"] = run_head_profile(args, local_rank, flush, peaks)
     if not args.no_stack:
         out["stack_480p"] = run_stack(local_rank)
@@ -435,6 +438,86 @@ def run_incremental(args, w, hm, local_rank, hk, hv, dK, dV, dQ, dO, flush, stre
         "compact": kern("compact", compact_bytes),
         "note": "per step: scoring reads C + 1 frames per dynamic head, compaction copies C x k "
                 "segments + the anchor frame per dynamic head (ring-buffer views)",
+    }
+
+
+def run_fp8(args, w, hm, local_rank, hk, hv, dK, dV, dQ, dO, flush, stream, world, peaks,
+            bf16_attn_ms):
+    """The same stream with Q K^T on E4M3 operands (FK_ATTN_FP8_QK): every step quantizes the
+    chunk's queries and, after the append and compression, every key row of the layer's views;
+    under denoising steps (fk_set_current) only the current chunk's key rows would be redone."""
+    import torch
+
+    from paper_2605_09681_gb300 import ForcingKVCache
+
+    wf = w.with_(attn_precision="fp8_qk")
+    n_pool = len(dK)
+    cache = ForcingKVCache.from_workload(wf, hm, device=local_rank)
+    cache.append_frames(0, hk, hv)
+    cache.set_current(0, dK[0], dV[0])
+    cache.compress()
+
+    def step(i):
+        j = i % n_pool
+        cache.append_chunk(0, dK[j], dV[j])
+        cache.compress()
+        cache.attend(0, dQ[j], dO)
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize()
+    keys = [cache.key_count(0, h) for h in range(w.n_heads)]
+
+    def timed():
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(args.steps)]
+        barrier(world)
+        torch.cuda.synchronize()
+        for i in range(args.steps):
+            flush.zero_()
+            evs[i][0].record(stream)
+            step(i)
+            evs[i][1].record(stream)
+        torch.cuda.synchronize()
+        barrier(world)
+        return sum(a.elapsed_time(b) for a, b in evs)
+
+    total_ms = reduce_max(timed(), world)
+    cache.profile_enable(True)
+    cache.profile_reset()
+    timed()
+    kinds = ("append", "score", "select", "compact", "quant", "attend")
+    prof = {k: cache.profile_read(k) for k in kinds}
+    if cache.sync_status() != 0:
+        raise SystemExit("device status error in the FP8 run")
+    cache.close()
+    alg = _algorithmic(w, keys)
+    D, nq = w.head_dim, w.n_queries
+    attn_ms = prof["attend"][0] / max(1, prof["attend"][1])
+    attn_tflops = alg["attn_flops"] / (attn_ms * 1e-3) / 1e12
+    # half the flops (Q K^T) at the E4M3 rate (twice bf16, the nominal ratio), half (P V) at
+    # the bf16 rate: the mixed peak is 4/3 of the measured bf16 peak
+    mixed_peak = peaks["bf16_tflops"] * 4.0 / 3.0
+    # quantization bytes per step: bf16 read + E4M3 write of every key row and query row,
+    # plus the query exponents
+    quant_bytes = (sum(keys) + nq * w.n_heads) * D * 3 + nq * w.n_heads
+    quant_ms = prof["quant"][0] / args.steps
+    quant_gbs = quant_bytes / (quant_ms * 1e-3) / 1e9
+    return {
+        "workload": wf.name if wf.name.endswith("fp8") else wf.name + " (fp8_qk)",
+        "ms_per_step": round(total_ms / args.steps, 4),
+        "value": round(world * alg["attn_flops"] * args.steps / (total_ms * 1e-3) / 1e12, 3),
+        "unit": "TFLOP/s",
+        "kernels_us_per_step": {k: round(prof[k][0] / args.steps * 1e3, 2) for k in kinds},
+        "attention": {"us": round(attn_ms * 1e3, 2), "achieved": round(attn_tflops, 1),
+                      "unit": "TFLOP/s", "peak": round(mixed_peak, 1),
+                      "frac": round(attn_tflops / mixed_peak, 4),
+                      "speedup_vs_bf16_kernel": round(bf16_attn_ms / attn_ms, 3)},
+        "quant": {"bytes": quant_bytes, "us": round(quant_ms * 1e3, 2), "achieved": round(quant_gbs, 1),
+                  "unit": "GB/s", "frac": round(quant_gbs / peaks["hbm_gbs"], 4),
+                  "launches_per_step": prof["quant"][1] / args.steps},
+        "note": "same algorithmic FLOPs as the bf16 step; Q K^T on E4M3 (kind::f8f6f4), P V bf16; "
+                "the attention is compared with the 4/3 x bf16 mixed peak",
     }
 
 

@@ -92,6 +92,19 @@ enum {
   FK_SELECT_RANDOM = 3
 };
 
+/* Operand precision of the chunk attention's Q K^T product (the paper's quantization
+ * appendix: FP8 attention on the compressed cache).  BF16: Q, K, V in bf16 (the method).
+ * FP8_QK: Q K^T on OCP FP8 E4M3 operands with f32 accumulation; P V stays bf16.  Keys are
+ * rounded to E4M3 unscaled (the scoring precondition |K| <= 256 keeps them inside the E4M3
+ * range, largest finite 448; larger values saturate); each query row (token, head) is scaled
+ * by 2^-e, e the smallest integer with max |q| <= 448 * 2^e, and the logits are scaled back
+ * by 2^e, so the E4M3 rounding (to nearest, ties to even) is the only inexact step before
+ * the softmax.  fk_quantize_e4m3 applies the same rounding.  FP8_QK requires head_dim 128. */
+enum {
+  FK_ATTN_BF16 = 0,
+  FK_ATTN_FP8_QK = 1
+};
+
 typedef struct fk_config {
   int32_t n_layers;             /* 1..256                                                  */
   int32_t n_heads;              /* 1..128                                                  */
@@ -116,6 +129,7 @@ typedef struct fk_config {
   uint32_t select_seed;         /* seed of FK_SELECT_RANDOM                                */
   int32_t static_drop_anchor;   /* 1: static heads keep sink + current chunk only (Dummy
                                    Forcing's local heads); 0: sink + anchor + current (Eq. 2) */
+  int32_t attn_precision;       /* FK_ATTN_* (0 = bf16)                                    */
 } fk_config;
 
 typedef struct fk_handle fk_handle;
@@ -193,7 +207,9 @@ FK_API fk_status fk_sync_status(fk_handle* h, void* stream);
  * stream.  fk_profile_read synchronizes and returns, per kernel kind, the total device
  * milliseconds and the number of launches since the last reset. */
 enum { FK_KERNEL_APPEND = 0, FK_KERNEL_SCORE = 1, FK_KERNEL_SELECT = 2, FK_KERNEL_COMPACT = 3,
-       FK_KERNEL_ATTEND = 4, FK_KERNEL_KINDS = 5 };
+       FK_KERNEL_ATTEND = 4, FK_KERNEL_QUANT = 5, FK_KERNEL_KINDS = 6 };
+/* FK_KERNEL_QUANT: the E4M3 quantization of queries and of changed key rows that precedes
+ * the attention kernel under FK_ATTN_FP8_QK. */
 FK_API fk_status fk_profile_enable(fk_handle* h, int on);
 FK_API fk_status fk_profile_read(fk_handle* h, int kind, double* total_ms, int64_t* launches);
 FK_API fk_status fk_profile_reset(fk_handle* h);
@@ -273,11 +289,24 @@ FK_API fk_status fk_head_profile(const void* Q, const void* K, int n_queries, in
 FK_API fk_status fk_classify_heads(const double* mass, int n_heads, int alpha_permille,
                                    uint8_t* head_is_static);
 
+/* E4M3 quantization of bf16 rows, as the FP8_QK attention applies it (see FK_ATTN_FP8_QK).
+ * X: device [rows][dim] bf16; q8: device [rows][dim] bytes, OCP FP8 E4M3 codes; both 16-byte
+ * aligned.  row_scaled = 1 (queries): row r is multiplied by 2^-e_r, e_r the smallest integer
+ * with max_c |X[r][c]| <= 448 * 2^e_r (0 for an all-zero row; clamped to [-120, 120]), then
+ * rounded to the nearest E4M3 value (ties to even, saturating at +-448); exps (device int8
+ * [rows]) receives e_r.  row_scaled = 0 (keys): every element is rounded unscaled and exps may
+ * be NULL.  dim: 64 or 128 when row_scaled, else a multiple of 8 from 8 to 1024; rows >= 0.
+ * FK_ERR_ARG for null, unaligned or host pointers, FK_ERR_CONFIG for sizes out of range.
+ * Asynchronous on `stream`; allocates nothing; uses the current device. */
+FK_API fk_status fk_quantize_e4m3(const void* X, int64_t rows, int dim, int row_scaled,
+                                  void* q8, int8_t* exps, void* stream);
+
 /* Static text for a status code. */
 FK_API const char* fk_status_str(fk_status s);
 
-/* ABI version of this header: 2 (fk_config gained selection, select_seed and
- * static_drop_anchor after head_is_static). */
+/* ABI version of this header: 3 (fk_config gained selection, select_seed and
+ * static_drop_anchor after head_is_static in version 2, attn_precision in version 3;
+ * FK_KERNEL_QUANT was added in version 3). */
 FK_API int fk_abi_version(void);
 
 #ifdef __cplusplus

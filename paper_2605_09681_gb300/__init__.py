@@ -14,7 +14,7 @@ from . import _lib as L
 from ._lib import FkError, KERNEL_KINDS, STATUS_NAMES
 
 __all__ = ["ForcingKVCache", "FkError", "KERNEL_KINDS", "STATUS_NAMES", "load_library",
-           "head_profile", "classify_heads"]
+           "head_profile", "classify_heads", "quantize_e4m3"]
 
 
 def load_library():
@@ -78,6 +78,25 @@ def head_profile(Q, K, n_generate: int, n_sink: int, n_transition: int, mass=Non
     return mass, status
 
 
+def quantize_e4m3(X, row_scaled: bool, q8=None, exps=None, stream=None):
+    """E4M3 codes of a bf16 CUDA tensor [..., dim] as the FP8 attention path forms them
+    (fk_quantize_e4m3): row_scaled=True scales each row by its power-of-two exponent (queries),
+    False rounds unscaled (keys).  Returns (q8 uint8 tensor of X's shape, int8 exponents per
+    row or None)."""
+    import torch
+    dim = X.shape[-1]
+    rows = X.numel() // dim if dim else 0
+    if q8 is None:
+        q8 = torch.empty(X.shape, dtype=torch.uint8, device=X.device)
+    if row_scaled and exps is None:
+        exps = torch.empty(rows, dtype=torch.int8, device=X.device)
+    lib = L.load()
+    _check(lib.fk_quantize_e4m3(_ptr(X), rows, dim, 1 if row_scaled else 0, q8.data_ptr(),
+                                exps.data_ptr() if exps is not None else None, _stream(stream)),
+           "fk_quantize_e4m3")
+    return q8, exps
+
+
 def classify_heads(mass, alpha: float = 0.8) -> np.ndarray:
     """Eq. 1 on masses [H, 4] (host copy): 1 = static, 0 = dynamic (fk_classify_heads)."""
     m = np.ascontiguousarray(np.asarray(mass, dtype=np.float64))
@@ -101,7 +120,7 @@ class ForcingKVCache:
                  n_sink_frames, window_frames, n_segments, keep_budget_permille,
                  head_is_static, select_scope="per_frame", score_source="per_head",
                  incremental=False, max_history_frames=64, device=0, selection="similarity",
-                 select_seed=0, static_drop_anchor=False):
+                 select_seed=0, static_drop_anchor=False, attn_precision="bf16"):
         self._lib = L.load()
         self._h = ctypes.c_void_p()
         hm = np.ascontiguousarray(np.asarray(head_is_static, dtype=np.uint8).reshape(-1))
@@ -115,7 +134,8 @@ class ForcingKVCache:
             {"per_head": L.FK_SCORE_PER_HEAD, "layer0_pooled": L.FK_SCORE_LAYER0_POOLED}[score_source],
             1 if incremental else 0, max_history_frames, device,
             hm.ctypes.data_as(ctypes.POINTER(ctypes.c_uint8)),
-            L.FK_SELECT[selection], select_seed & 0xFFFFFFFF, 1 if static_drop_anchor else 0)
+            L.FK_SELECT[selection], select_seed & 0xFFFFFFFF, 1 if static_drop_anchor else 0,
+            L.FK_ATTN[attn_precision])
         self.n_layers, self.n_heads, self.head_dim = n_layers, n_heads, head_dim
         self.F, self.C, self.n_segments = tokens_per_frame, frames_per_chunk, n_segments
         self.device = device
@@ -131,7 +151,7 @@ class ForcingKVCache:
                   score_source=w.score_source, incremental=w.incremental,
                   max_history_frames=max(1, w.max_history_frames()), device=device,
                   selection=w.selection, select_seed=w.select_seed,
-                  static_drop_anchor=w.static_drop_anchor)
+                  static_drop_anchor=w.static_drop_anchor, attn_precision=w.attn_precision)
         kw.update(over)
         return cls(**kw)
 

@@ -16,7 +16,8 @@ STATUS_NAMES = {0: "FK_OK", 1: "FK_ERR_CONFIG", 2: "FK_ERR_ARG", 3: "FK_ERR_STAT
 FK_SCOPE_PER_FRAME, FK_SCOPE_POOLED = 0, 1
 FK_SCORE_PER_HEAD, FK_SCORE_LAYER0_POOLED = 0, 1
 FK_SELECT = {"similarity": 0, "all": 1, "uniform": 2, "random": 3}
-KERNEL_KINDS = {"append": 0, "score": 1, "select": 2, "compact": 3, "attend": 4}
+FK_ATTN = {"bf16": 0, "fp8_qk": 1}
+KERNEL_KINDS = {"append": 0, "score": 1, "select": 2, "compact": 3, "attend": 4, "quant": 5}
 
 EXPORTS = [
     "fk_validate_config", "fk_create", "fk_destroy", "fk_append_frames", "fk_append_chunk",
@@ -24,7 +25,7 @@ EXPORTS = [
     "fk_key_count", "fk_get_kept", "fk_get_scores", "fk_sync_status", "fk_profile_enable",
     "fk_profile_read", "fk_profile_reset", "fk_launch_count", "fk_status_str", "fk_abi_version",
     "fk_segment_scores_noalloc", "fk_head_profile", "fk_classify_heads", "fk_set_host_overlap",
-    "fk_wait_selftest", "fk_wait_outputs",
+    "fk_wait_selftest", "fk_wait_outputs", "fk_quantize_e4m3",
 ]
 
 
@@ -38,7 +39,7 @@ class FkConfig(ctypes.Structure):
         ("incremental", ctypes.c_int32), ("max_history_frames", ctypes.c_int32),
         ("device", ctypes.c_int32), ("head_is_static", ctypes.POINTER(ctypes.c_uint8)),
         ("selection", ctypes.c_int32), ("select_seed", ctypes.c_uint32),
-        ("static_drop_anchor", ctypes.c_int32),
+        ("static_drop_anchor", ctypes.c_int32), ("attn_precision", ctypes.c_int32),
     ]
 
 
@@ -92,6 +93,7 @@ def load(path: str | None = None) -> ctypes.CDLL:
         "fk_head_profile": (st, [vp, vp, i32, i32, i32, i32, i32, i32, i32, vp, vp, vp]),
         "fk_classify_heads": (st, [ctypes.POINTER(ctypes.c_double), i32, i32,
                                    ctypes.POINTER(ctypes.c_uint8)]),
+        "fk_quantize_e4m3": (st, [vp, ctypes.c_int64, i32, i32, vp, vp, vp]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)

@@ -13,6 +13,10 @@
 //                      lazily rescaled running max, writes P as bf16 pairs over S's first
 //                      64 columns with tcgen05.st, and finally normalises O and stores it.
 // TMEM columns: S0 0-127, S1 128-255, O0 256.., O1 256+D.. (512 allocated).
+// FP8_QK variant (D = 128): Q and K tiles hold E4M3 codes (one 128-byte swizzle atom per
+// row), S = Q K^T runs as tcgen05.mma kind::f8f6f4 (K = 32 per instruction), and each
+// softmax thread scales its row's logits by 2^e_row (the query row's quantization exponent)
+// along with 1/sqrt(D); P V is unchanged (bf16).
 // Every mbarrier wait is bounded (%globaltimer); on expiry the CTA records
 // FK_ERR_TIMEOUT in the status word, drains its own TMA loads and MMAs and frees TMEM.
 #include "fk_internal.h"
@@ -37,13 +41,14 @@ struct AttnBarriers {
   volatile int abort;
 };
 
-template <int D>
+template <int D, bool kFp8 = false>
 struct Layout {
-  static constexpr int kQ = kAttnBM * D * 2;      // one 128-row query tile
-  static constexpr int kKV = kAttnBN * D * 2;     // one 128-key K or V tile
+  static constexpr int kQ = kAttnBM * D * (kFp8 ? 1 : 2);   // one 128-row query tile
+  static constexpr int kK = kAttnBN * D * (kFp8 ? 1 : 2);   // one 128-key K tile
+  static constexpr int kKV = kAttnBN * D * 2;               // one 128-key V tile (bf16)
   static constexpr int kOffQ = 0;                 // two query tiles
   static constexpr int kOffK = kOffQ + 2 * kQ;    // two K stages
-  static constexpr int kOffV = kOffK + 2 * kKV;   // two V stages
+  static constexpr int kOffV = kOffK + 2 * kK;    // two V stages
   static constexpr int kOffBar = kOffV + 2 * kKV;
   static constexpr int kUsed = kOffBar + 256;
   // at least ~116 KB so that one CTA occupies an SM (its 512 TMEM columns are then free)
@@ -139,6 +144,11 @@ __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, int b_mn) {
   return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)b_mn << 16) |
          ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
 }
+// Instruction descriptor, kind::f8f6f4: f32 accumulate, A and B E4M3 (type code 0 at bits
+// 7 and 10), both K-major.
+__host__ __device__ constexpr uint32_t idesc_e4m3(int M, int N) {
+  return (1u << 4) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
 
 __device__ __forceinline__ void umma(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
                                      uint32_t accumulate) {
@@ -154,6 +164,14 @@ __device__ __forceinline__ void umma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64
       "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
       " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}\n"
       :: "r"(d_tmem), "r"(a_tmem), "l"(b), "r"(idesc), "r"(accumulate) : "memory");
+}
+// D[tmem] (+)= A[smem] * B[smem]^T on E4M3 operands (both K-major, K = 32 per instruction)
+__device__ __forceinline__ void umma_f8(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
+                                        uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n}\n"
+      :: "r"(d_tmem), "l"(a), "l"(b), "r"(idesc), "r"(accumulate) : "memory");
 }
 __device__ __forceinline__ void umma_commit(uint64_t* b) {
   asm volatile(
@@ -261,12 +279,13 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
 }
 
 // kSplit: a launch with key splits (kv_splits > 1); the unsplit instantiation carries none of
-// the split bookkeeping.
-template <int D, bool kSplit>
+// the split bookkeeping.  kFp8: Q K^T on E4M3 operands (D = 128).
+template <int D, bool kSplit, bool kFp8>
 __global__ void __launch_bounds__(kAttnThreads, 1)
 attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
             const __grid_constant__ CUtensorMap tmV, const AttnArgs a) {
-  using Lay = Layout<D>;
+  static_assert(!kFp8 || D == 128, "FP8_QK: one 128-byte swizzle atom per Q / K row");
+  using Lay = Layout<D, kFp8>;
   constexpr int kHalves = D / 64;                 // 64-column (128-byte) swizzle atoms
   constexpr uint32_t kTmemCols = 512;
   constexpr uint32_t kColO = 2 * kAttnBN;         // S0 = cols 0..127, S1 = 128..255, O0, O1 after
@@ -327,17 +346,26 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
       int lastK[2] = {-1, -1}, lastV[2] = {-1, -1};
       bool ok = true;
       mbar_expect_tx(&bar->q_full, 2 * Lay::kQ);
-      for (int t = 0; t < 2; ++t)
-        for (int h = 0; h < kHalves; ++h)
-          tma_load_3d(sQ + t * Lay::kQ + h * 16384, &tmQ, &bar->q_full, h * 64, head,
-                      q0 + t * kAttnBM);
+      for (int t = 0; t < 2; ++t) {
+        if constexpr (kFp8) {
+          tma_load_3d(sQ + t * Lay::kQ, &tmQ, &bar->q_full, 0, head, q0 + t * kAttnBM);
+        } else {
+          for (int h = 0; h < kHalves; ++h)
+            tma_load_3d(sQ + t * Lay::kQ + h * 16384, &tmQ, &bar->q_full, h * 64, head,
+                        q0 + t * kAttnBM);
+        }
+      }
       for (int j = 0; j < nt && ok; ++j) {
         const int st = j & 1, u = j >> 1;
         if (j >= 2 && !wait_phase(&bar->k_empty[st], (u - 1) & 1, bar, a.status)) { ok = false; break; }
-        mbar_expect_tx(&bar->k_full[st], Lay::kKV);
-        for (int h = 0; h < kHalves; ++h)
-          tma_load_2d(sK + st * Lay::kKV + h * 16384, &tmK, &bar->k_full[st], h * 64,
-                      row0 + j * kAttnBN);
+        mbar_expect_tx(&bar->k_full[st], Lay::kK);
+        if constexpr (kFp8) {
+          tma_load_2d(sK + st * Lay::kK, &tmK, &bar->k_full[st], 0, row0 + j * kAttnBN);
+        } else {
+          for (int h = 0; h < kHalves; ++h)
+            tma_load_2d(sK + st * Lay::kK + h * 16384, &tmK, &bar->k_full[st], h * 64,
+                        row0 + j * kAttnBN);
+        }
         lastK[st] = u;
         if (j >= 2 && !wait_phase(&bar->v_empty[st], (u - 1) & 1, bar, a.status)) { ok = false; break; }
         mbar_expect_tx(&bar->v_full[st], Lay::kKV);
@@ -362,16 +390,26 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
     // is complete too: the softmax of tile j+1 may rescale O_t without a further wait, and
     // S_t(j+1) overwriting P_t(j) (same columns) happens after PV_t(j) has read it.
     if (lane == 0) {
-      constexpr uint32_t kIdQK = idesc_bf16(kAttnBM, kAttnBN, 0);
+      constexpr uint32_t kIdQK = kFp8 ? idesc_e4m3(kAttnBM, kAttnBN) : idesc_bf16(kAttnBM, kAttnBN, 0);
       constexpr uint32_t kIdPV = idesc_bf16(kAttnBM, D, 1);
       const uint32_t aQ = su32(sQ), aK = su32(sK), aV = su32(sV);
       auto qk = [&](int j, int t) {
         const int st = j & 1;
+        if constexpr (kFp8) {
+          // 128 codes per row = one swizzle atom: four K = 32 steps of 32 bytes
 #pragma unroll
-        for (int kk = 0; kk < D / 16; ++kk) {
-          const uint64_t da = sdesc(aQ + t * Lay::kQ + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024);
-          const uint64_t db = sdesc(aK + st * Lay::kKV + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024);
-          umma(tmem + (uint32_t)(t * kAttnBN), da, db, kIdQK, kk > 0 ? 1u : 0u);
+          for (int kk = 0; kk < 4; ++kk) {
+            const uint64_t da = sdesc(aQ + t * Lay::kQ + kk * 32, 16, 1024);
+            const uint64_t db = sdesc(aK + st * Lay::kK + kk * 32, 16, 1024);
+            umma_f8(tmem + (uint32_t)(t * kAttnBN), da, db, kIdQK, kk > 0 ? 1u : 0u);
+          }
+        } else {
+#pragma unroll
+          for (int kk = 0; kk < D / 16; ++kk) {
+            const uint64_t da = sdesc(aQ + t * Lay::kQ + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024);
+            const uint64_t db = sdesc(aK + st * Lay::kK + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024);
+            umma(tmem + (uint32_t)(t * kAttnBN), da, db, kIdQK, kk > 0 ? 1u : 0u);
+          }
         }
         umma_commit(&bar->s_full[t]);
       };
@@ -426,6 +464,14 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
     const uint32_t lane_base = (uint32_t)(wq * 32) << 16;
     const uint32_t tS = tmem + lane_base + (uint32_t)(t * kAttnBN);
     const uint32_t tO = tmem + lane_base + kColO + (uint32_t)(t * D);
+    // logit scale of this row in the log2 domain: log2(e) / sqrt(D), times 2^e_row for E4M3
+    // queries (e_row in [-120, 120]: the product is exact)
+    float sl2 = a.scale_log2;
+    if constexpr (kFp8) {
+      const int qr = q0 + t * kAttnBM + row;
+      const int e = qr < a.Nq ? (int)a.q_exp[(int64_t)qr * a.H + head] : 0;
+      sl2 *= __uint_as_float((uint32_t)(127 + e) << 23);
+    }
     float m = -INFINITY, l = 0.0f;
     bool ok = true;
     for (int j = 0; j < nt; ++j) {
@@ -433,7 +479,7 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
       tc_fence_after();
       const int valid = nk - j * kAttnBN;           // keys of this tile (< 128 only in the last)
       const bool full = valid >= kAttnBN;           // uniform over the CTA
-      const float2 sc2 = make_float2(a.scale_log2, a.scale_log2);
+      const float2 sc2 = make_float2(sl2, sl2);
       float2 acc[4];
 #pragma unroll
       for (int i = 0; i < 4; ++i) acc[i] = make_float2(0.0f, 0.0f);
@@ -462,7 +508,7 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
         }
         const float mx = fmaxf(fmaxf(fmaxf(mxa[0], mxa[1]), fmaxf(mxa[2], mxa[3])),
                                fmaxf(fmaxf(mxa[4], mxa[5]), fmaxf(mxa[6], mxa[7])));
-        const float m_new = fmaxf(m, mx * a.scale_log2);
+        const float m_new = fmaxf(m, mx * sl2);
         if (__any_sync(0xffffffffu, m_new > m + kRescaleThreshold)) {   // warp-uniform
           const float alpha = fast_exp2(m - m_new);  // 0 when m = -inf
           l *= alpha;
@@ -508,8 +554,8 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
             const float x0 = c < valid ? __uint_as_float(sv[2 * q]) : -INFINITY;
             const float x1 = c + 1 < valid ? __uint_as_float(sv[2 * q + 1]) : -INFINITY;
             float2 e;
-            e.x = fast_exp2(fmaf(x0, a.scale_log2, -m));
-            e.y = fast_exp2(fmaf(x1, a.scale_log2, -m));
+            e.x = fast_exp2(fmaf(x0, sl2, -m));
+            e.y = fast_exp2(fmaf(x1, sl2, -m));
             acc[q & 3] = fadd2(acc[q & 3], e);
             pk[q] = pack_bf16(e.x, e.y);
           }
@@ -861,30 +907,36 @@ void launch_merge(int head_dim, const AttnArgs& a, cudaStream_t s) {
 }
 
 cudaError_t attention_prepare(int head_dim) {
+  const auto set = [](const void* fn, int smem) {
+    return cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  };
   cudaError_t e;
   if (head_dim == 128) {
-    e = cudaFuncSetAttribute(attn_kernel<128, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             Layout<128>::kSmem);
-    if (e != cudaSuccess) return e;
-    return cudaFuncSetAttribute(attn_kernel<128, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                Layout<128>::kSmem);
+    if ((e = set((const void*)attn_kernel<128, false, false>, Layout<128>::kSmem)) != cudaSuccess) return e;
+    if ((e = set((const void*)attn_kernel<128, true, false>, Layout<128>::kSmem)) != cudaSuccess) return e;
+    if ((e = set((const void*)attn_kernel<128, false, true>, Layout<128, true>::kSmem)) != cudaSuccess) return e;
+    return set((const void*)attn_kernel<128, true, true>, Layout<128, true>::kSmem);
   }
-  e = cudaFuncSetAttribute(attn_kernel<64, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           Layout<64>::kSmem);
-  if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(attn_kernel<64, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              Layout<64>::kSmem);
+  if ((e = set((const void*)attn_kernel<64, false, false>, Layout<64>::kSmem)) != cudaSuccess) return e;
+  return set((const void*)attn_kernel<64, true, false>, Layout<64>::kSmem);
 }
 
-void launch_attention(int head_dim, const CUtensorMap& tmQ, const CUtensorMap& tmK,
+void launch_attention(int head_dim, bool fp8, const CUtensorMap& tmQ, const CUtensorMap& tmK,
                       const CUtensorMap& tmV, const AttnArgs& a, cudaStream_t s) {
   const unsigned grid = (unsigned)(a.n_qtiles * a.H * a.kv_splits);
-  if (head_dim == 128) {
-    if (a.kv_splits > 1) attn_kernel<128, true><<<grid, kAttnThreads, Layout<128>::kSmem, s>>>(tmQ, tmK, tmV, a);
-    else attn_kernel<128, false><<<grid, kAttnThreads, Layout<128>::kSmem, s>>>(tmQ, tmK, tmV, a);
+  const bool split = a.kv_splits > 1;
+  if (head_dim == 128 && fp8) {
+    constexpr int sm = Layout<128, true>::kSmem;
+    if (split) attn_kernel<128, true, true><<<grid, kAttnThreads, sm, s>>>(tmQ, tmK, tmV, a);
+    else attn_kernel<128, false, true><<<grid, kAttnThreads, sm, s>>>(tmQ, tmK, tmV, a);
+  } else if (head_dim == 128) {
+    constexpr int sm = Layout<128>::kSmem;
+    if (split) attn_kernel<128, true, false><<<grid, kAttnThreads, sm, s>>>(tmQ, tmK, tmV, a);
+    else attn_kernel<128, false, false><<<grid, kAttnThreads, sm, s>>>(tmQ, tmK, tmV, a);
   } else {
-    if (a.kv_splits > 1) attn_kernel<64, true><<<grid, kAttnThreads, Layout<64>::kSmem, s>>>(tmQ, tmK, tmV, a);
-    else attn_kernel<64, false><<<grid, kAttnThreads, Layout<64>::kSmem, s>>>(tmQ, tmK, tmV, a);
+    constexpr int sm = Layout<64>::kSmem;
+    if (split) attn_kernel<64, true, false><<<grid, kAttnThreads, sm, s>>>(tmQ, tmK, tmV, a);
+    else attn_kernel<64, false, false><<<grid, kAttnThreads, sm, s>>>(tmQ, tmK, tmV, a);
   }
 }
 

@@ -16,6 +16,9 @@
 //                int64 scoring sums (scratch); status word;
 //                host staging (two slots of K, V and Q; O) and the attention key-split
 //                scratch (fp32 partial outputs and row statistics of two splits).
+//   FP8_QK only  the E4M3 copy of the K view arena ([rows][D] bytes, refreshed before an
+//                attention call for the rows changed since the last one) and the
+//                quantized queries of one call (codes [C*F][H][D], exponents [C*F][H]).
 #include <algorithm>
 #include <cmath>
 #include <cstdio>
@@ -59,6 +62,10 @@ struct LayerState {
   int ring_end = 0;
   int ring_head = 0;
   int sinks_done = 0;     // sink frames already in the dynamic views
+  // FP8_QK: the E4M3 copy of this layer's K views matches the current-chunk rows / the
+  // history rows (sink, anchor, kept segments)
+  bool k8_cur_ok = false;
+  bool k8_hist_ok = false;
 };
 
 struct Staging {
@@ -132,6 +139,7 @@ struct fk_handle {
   int selection = FK_SELECT_SIMILARITY;
   uint32_t select_seed = 0;
   bool drop_anchor = false;        // static heads keep sink + current chunk only
+  bool fp8 = false;                // FK_ATTN_FP8_QK
   std::vector<HeadBuf> heads;      // [L*H]
   std::vector<LayerState> layers;  // [L]
   // device memory
@@ -173,6 +181,10 @@ struct fk_handle {
   int max_run = 0;
   int score_ctas = 0;
   CUtensorMap tmK{}, tmV{};
+  uint8_t* viewK8 = nullptr;       // FP8_QK: E4M3 codes of the K view arena
+  uint8_t* q8 = nullptr;           // FP8_QK: E4M3 codes of one call's queries
+  int8_t* q_exp = nullptr;         //         and their row exponents [C*F][H]
+  CUtensorMap tmK8{}, tmQ8{};
   const void* q_cached[2] = {};   // two cached Q maps (the two Q staging slots alternate)
   CUtensorMap tmQ[2]{};
   int q_next = 0;
@@ -339,23 +351,29 @@ fk_status stage_inputs(fk_handle* h, Staging& sg, const void* a, const void* b, 
   return FK_OK;
 }
 
-fk_status encode_2d(CUtensorMap* m, void* base, int64_t rows, int D) {
+// 2D map over a [rows][D] arena, 128-row boxes of one 128-byte swizzle atom per row: 64 bf16
+// (bf16) or 128 E4M3 codes (e4m3, D = 128)
+fk_status encode_2d(CUtensorMap* m, void* base, int64_t rows, int D, bool e4m3 = false) {
   const cuuint64_t dims[2] = {(cuuint64_t)D, (cuuint64_t)rows};
-  const cuuint64_t strides[1] = {(cuuint64_t)D * 2};
-  const cuuint32_t box[2] = {64, (cuuint32_t)kAttnBN};
+  const cuuint64_t strides[1] = {(cuuint64_t)D * (e4m3 ? 1 : 2)};
+  const cuuint32_t box[2] = {e4m3 ? 128u : 64u, (cuuint32_t)kAttnBN};
   const cuuint32_t es[2] = {1, 1};
-  CUresult r = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, dims, strides, box, es,
+  CUresult r = g_encode(m, e4m3 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
+                        2, base, dims, strides, box, es,
                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS ? FK_OK : FK_ERR_CUDA;
 }
 
-fk_status encode_q(CUtensorMap* m, const void* q, int Nq, int H, int D) {
+// 3D map over token-major [Nq][H][D], boxes of 128 rows of one head (as encode_2d)
+fk_status encode_q(CUtensorMap* m, const void* q, int Nq, int H, int D, bool e4m3 = false) {
+  const int es_b = e4m3 ? 1 : 2;
   const cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)H, (cuuint64_t)Nq};
-  const cuuint64_t strides[2] = {(cuuint64_t)D * 2, (cuuint64_t)H * D * 2};
-  const cuuint32_t box[3] = {64, 1, (cuuint32_t)kAttnBM};
+  const cuuint64_t strides[2] = {(cuuint64_t)D * es_b, (cuuint64_t)H * D * es_b};
+  const cuuint32_t box[3] = {e4m3 ? 128u : 64u, 1, (cuuint32_t)kAttnBM};
   const cuuint32_t es[3] = {1, 1, 1};
-  CUresult r = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(q), dims,
+  CUresult r = g_encode(m, e4m3 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
+                        3, const_cast<void*>(q), dims,
                         strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
                         CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
@@ -408,6 +426,7 @@ fk_status push_history(fk_handle* h, int layer, const bf16* tokK, const bf16* to
   }
   ls.nh = nh1;
   ls.dirty = true;
+  ls.k8_hist_ok = false;
   update_lengths(h, layer);
   return FK_OK;
 }
@@ -454,7 +473,9 @@ fk_status update_current(fk_handle* h, int layer, bool retire, const void* K, co
   if (retire) {
     ls.nh += h->C;
     ls.dirty = true;
+    ls.k8_hist_ok = false;
   }
+  if (k) ls.k8_cur_ok = false;
   ls.has_current = k != nullptr || (ls.has_current && !retire);
   update_lengths(h, layer);
   return FK_OK;
@@ -501,6 +522,31 @@ fk_status fk_head_profile(const void* Q, const void* K, int n_queries, int n_key
              : FK_ERR_CUDA;
 }
 
+fk_status fk_quantize_e4m3(const void* X, int64_t rows, int dim, int row_scaled, void* q8,
+                           int8_t* exps, void* stream) {
+  if (!X || !q8 || !aligned16(X) || !aligned16(q8)) return FK_ERR_ARG;
+  if (row_scaled != 0 && row_scaled != 1) return FK_ERR_CONFIG;
+  if (rows < 0 || rows > ((int64_t)1 << 31)) return FK_ERR_CONFIG;
+  if (row_scaled ? (dim != 64 && dim != 128) : (dim < 8 || dim > 1024 || dim % 8)) return FK_ERR_CONFIG;
+  if (row_scaled && !exps) return FK_ERR_ARG;
+  if (rows == 0) return FK_OK;
+  if (!is_device_ptr(X) || !is_device_ptr(q8) || (row_scaled && !is_device_ptr(exps))) return FK_ERR_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (row_scaled) {
+    launch_quant_rows_scaled(static_cast<const bf16*>(X), rows, dim, static_cast<uint8_t*>(q8), exps, s);
+  } else {
+    QuantRanges qr{};
+    qr.src = static_cast<const bf16*>(X);
+    qr.dst = static_cast<uint8_t*>(q8);
+    qr.D = dim;
+    qr.n = 1;
+    qr.row0[0] = 0;
+    qr.rows[0] = rows;
+    launch_quant_ranges(qr, s);
+  }
+  return cudaGetLastError() == cudaSuccess ? FK_OK : FK_ERR_CUDA;
+}
+
 fk_status fk_classify_heads(const double* mass, int n_heads, int alpha_permille,
                             uint8_t* head_is_static) {
   if (!mass || !head_is_static || n_heads < 0) return FK_ERR_ARG;
@@ -540,7 +586,7 @@ fk_status fk_wait_outputs(fk_handle* h, void* stream) {
   return FK_OK;
 }
 
-int fk_abi_version(void) { return 2; }
+int fk_abi_version(void) { return 3; }
 
 const char* fk_status_str(fk_status s) {
   switch (s) {
@@ -574,6 +620,8 @@ fk_status fk_validate_config(const fk_config* c) {
   if (c->selection < FK_SELECT_SIMILARITY || c->selection > FK_SELECT_RANDOM) return FK_ERR_CONFIG;
   if (c->selection == FK_SELECT_UNIFORM && c->select_scope != FK_SCOPE_PER_FRAME) return FK_ERR_CONFIG;
   if (c->static_drop_anchor != 0 && c->static_drop_anchor != 1) return FK_ERR_CONFIG;
+  if (c->attn_precision != FK_ATTN_BF16 && c->attn_precision != FK_ATTN_FP8_QK) return FK_ERR_CONFIG;
+  if (c->attn_precision == FK_ATTN_FP8_QK && c->head_dim != 128) return FK_ERR_CONFIG;
   const int64_t cf = (int64_t)c->frames_per_chunk * c->tokens_per_frame;
   if (cf > (1 << 24) || (int64_t)c->tokens_per_frame * c->head_dim > (1 << 28)) return FK_ERR_CONFIG;
   // 16-byte granules of one chunk (all heads) are indexed with 32-bit integers
@@ -616,6 +664,7 @@ fk_status fk_create(const fk_config* cfg, fk_handle** out) {
   h->selection = cfg->selection;
   h->select_seed = cfg->select_seed;
   h->drop_anchor = cfg->static_drop_anchor != 0;
+  h->fp8 = cfg->attn_precision == FK_ATTN_FP8_QK;
   h->k_frame = h->selection == FK_SELECT_ALL ? h->n : (h->b * h->n) / 1000;
   h->kmax = std::max(1, keep_total(h, h->cap_nonsink - 1));
   h->chunks = (h->seg + kScoreTokensPerCta - 1) / kScoreTokensPerCta;
@@ -682,6 +731,14 @@ fk_status fk_create(const fk_config* cfg, fk_handle** out) {
   h->viewK = static_cast<bf16*>(p);
   if ((st = dev_alloc(h, view_bytes, &p)) != FK_OK) return fail(st);
   h->viewV = static_cast<bf16*>(p);
+  if (h->fp8) {
+    if ((st = dev_alloc(h, view_bytes / 2, &p)) != FK_OK) return fail(st);
+    h->viewK8 = static_cast<uint8_t*>(p);
+    if ((st = dev_alloc(h, (size_t)h->CF * h->H * h->D, &p)) != FK_OK) return fail(st);
+    h->q8 = static_cast<uint8_t*>(p);
+    if ((st = dev_alloc(h, (size_t)h->CF * h->H, &p)) != FK_OK) return fail(st);
+    h->q_exp = static_cast<int8_t*>(p);
+  }
   size_t n_ret = 0;
   for (auto& hb : h->heads) n_ret += hb.retains;
   const size_t ring_elems = (size_t)h->ring_slots * h->F * h->D;
@@ -790,6 +847,10 @@ fk_status fk_create(const fk_config* cfg, fk_handle** out) {
 
   if ((st = encode_2d(&h->tmK, h->viewK, h->view_rows_total, h->D)) != FK_OK) return fail(st);
   if ((st = encode_2d(&h->tmV, h->viewV, h->view_rows_total, h->D)) != FK_OK) return fail(st);
+  if (h->fp8) {
+    if ((st = encode_2d(&h->tmK8, h->viewK8, h->view_rows_total, h->D, true)) != FK_OK) return fail(st);
+    if ((st = encode_q(&h->tmQ8, h->q8, h->CF, h->H, h->D, true)) != FK_OK) return fail(st);
+  }
   if (cudaDeviceSynchronize() != cudaSuccess) return fail(FK_ERR_CUDA);
   for (int l = 0; l < h->L; ++l) update_lengths(h, l);
   *out = h;
@@ -886,6 +947,7 @@ fk_status fk_compress(fk_handle* h, void* stream) {
   bool any = false;
   for (auto& ls : h->layers) any |= ls.dirty;
   if (!any) return FK_OK;
+  for (auto& ls : h->layers) ls.k8_hist_ok = false;   // views are rebuilt or extended
   const bool pooled_src = h->source == FK_SCORE_LAYER0_POOLED;
   if (pooled_src) {
     for (int l = 1; l < h->L; ++l)
@@ -1032,7 +1094,7 @@ fk_status fk_attend(fk_handle* h, int layer, const void* Q, void* O, void* strea
   fk_status st = check_layer(h, layer);
   if (st != FK_OK) return st;
   if (!Q || !O || !aligned16(Q) || !aligned16(O)) return FK_ERR_ARG;
-  const LayerState& ls = h->layers[layer];
+  LayerState& ls = h->layers[layer];
   if (!ls.has_current || ls.dirty) return FK_ERR_STATE;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   FK_CUDA(cudaSetDevice(h->dev));
@@ -1052,7 +1114,7 @@ fk_status fk_attend(fk_handle* h, int layer, const void* Q, void* O, void* strea
     if (h->o_pending[osl]) FK_CUDA(cudaStreamWaitEvent(s, h->o_copied[osl], 0));
   }
   int qm = q == h->q_cached[0] ? 0 : q == h->q_cached[1] ? 1 : -1;
-  if (qm < 0) {
+  if (qm < 0 && !h->fp8) {
     qm = h->q_next;
     h->q_next ^= 1;
     if ((st = encode_q(&h->tmQ[qm], q, h->CF, h->H, h->D)) != FK_OK) return st;
@@ -1060,6 +1122,7 @@ fk_status fk_attend(fk_handle* h, int layer, const void* Q, void* O, void* strea
   }
   AttnArgs a{};
   a.O = o;
+  a.q_exp = h->q_exp;
   a.Nq = h->CF;
   a.H = h->H;
   a.n_qtiles = (h->CF + 2 * kAttnBM - 1) / (2 * kAttnBM);   // CTA = two 128-row query tiles
@@ -1084,8 +1147,33 @@ fk_status fk_attend(fk_handle* h, int layer, const void* Q, void* O, void* strea
   a.part_o = h->part_o;
   a.part_ml = h->part_ml;
   const int D = h->D;
+  if (h->fp8) {
+    // E4M3 queries of this call, and the key rows changed since the layer's last call:
+    // the current chunk [0, C*F) and / or the history rows [C*F, n_keys) of every head
+    QuantRanges qr{};
+    qr.src = h->viewK;
+    qr.dst = h->viewK8;
+    qr.D = D;
+    if (!ls.k8_cur_ok || !ls.k8_hist_ok)
+      for (int hd = 0; hd < h->H; ++hd) {
+        const int lo = ls.k8_cur_ok ? h->CF : 0, hi = ls.k8_hist_ok ? h->CF : a.n_keys[hd];
+        if (hi <= lo) continue;
+        qr.row0[qr.n] = a.row_base[hd] + lo;
+        qr.rows[qr.n] = hi - lo;
+        ++qr.n;
+      }
+    if ((st = launch(h, s, FK_KERNEL_QUANT, [&] {
+           launch_quant_rows_scaled(q, (int64_t)h->CF * h->H, D, h->q8, h->q_exp, s);
+           if (qr.n) launch_quant_ranges(qr, s);
+         })) != FK_OK)
+      return st;
+    if (qr.n) h->launches++;   // the key pass
+    ls.k8_cur_ok = ls.k8_hist_ok = true;
+  }
+  const CUtensorMap& tq = h->fp8 ? h->tmQ8 : h->tmQ[qm];
+  const CUtensorMap& tk = h->fp8 ? h->tmK8 : h->tmK;
   if ((st = launch(h, s, FK_KERNEL_ATTEND, [&] {
-         launch_attention(D, h->tmQ[qm], h->tmK, h->tmV, a, s);
+         launch_attention(D, h->fp8, tq, tk, h->tmV, a, s);
          if (a.kv_splits > 1) launch_merge(D, a, s);
        })) != FK_OK)
     return st;
@@ -1118,7 +1206,7 @@ size_t fk_cache_bytes(const fk_handle* h) {
       const HeadBuf& hb = h->heads[l * h->H + hd];
       if (hb.retains) bytes += (size_t)live_frames * frame_bytes;
       const int rows = hb.is_static ? ls.len_static : ls.len_dynamic;
-      bytes += (size_t)rows * h->D * 2 * 2;
+      bytes += (size_t)rows * h->D * (h->fp8 ? 5 : 4);   // K and V bf16 (+ E4M3 K)
     }
   }
   bytes += h->targets.size() * ((size_t)h->ring_slots * h->n * sizeof(float) + h->kmax * sizeof(int));

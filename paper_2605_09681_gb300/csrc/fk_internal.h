@@ -153,6 +153,7 @@ void launch_compact(const CompactArgs& a, cudaStream_t s);
 // ------------------------------------------------------------------ attention
 struct AttnArgs {
   bf16* O;                      // [Nq][H][D]
+  const int8_t* q_exp;          // FP8_QK: per (query row, head) exponent e, [Nq][H]; else null
   int Nq;
   int H;
   int n_qtiles;
@@ -166,12 +167,30 @@ struct AttnArgs {
   int n_keys[kMaxHeads];        // keys the head attends to
 };
 // tmQ: 3D map over Q [Nq][H][D]; tmK/tmV: 2D maps over the view arenas [rows][D].
-void launch_attention(int head_dim, const CUtensorMap& tmQ, const CUtensorMap& tmK,
+// fp8: Q K^T on E4M3 operands (head_dim 128): tmQ / tmK then map the quantized bytes
+// (box 128 x 128, one 128-byte swizzle atom per row) and a.q_exp holds the query exponents.
+void launch_attention(int head_dim, bool fp8, const CUtensorMap& tmQ, const CUtensorMap& tmK,
                       const CUtensorMap& tmV, const AttnArgs& a, cudaStream_t s);
-cudaError_t attention_prepare(int head_dim);   // sets the dynamic shared-memory limit
+cudaError_t attention_prepare(int head_dim);   // sets the dynamic shared-memory limits
 // combine the key splits of every (row, head) into O (bf16)
 void launch_merge(int head_dim, const AttnArgs& a, cudaStream_t s);
 constexpr int kMaxKvSplits = 2;
+
+// ------------------------------------------------------------------ FP8 (E4M3) quantization
+// Unscaled rounding of row ranges of a [rows][D] bf16 arena into the byte arena of the same
+// shape (keys): range i covers rows [row0[i], row0[i] + rows[i]).
+struct QuantRanges {
+  const bf16* src;
+  uint8_t* dst;
+  int D;                        // a multiple of 8
+  int n;                        // ranges, <= kMaxHeads
+  int64_t row0[kMaxHeads];
+  int64_t rows[kMaxHeads];
+};
+void launch_quant_ranges(const QuantRanges& a, cudaStream_t s);
+// Row-scaled rounding of [rows][D] bf16, D = 64 or 128 (queries): exps[r] = e_r.
+void launch_quant_rows_scaled(const bf16* x, int64_t rows, int D, uint8_t* q8, int8_t* exps,
+                              cudaStream_t s);
 
 // ------------------------------------------------------------------ head profiling (Eq. 1)
 struct ProfArgs {

@@ -90,3 +90,42 @@ def run_snapshot(w: W.Workload, rows=None, check_scores=True, inputs=None, head_
         orc.append_frames(0, hk, hv)
         orc.set_current(0, ck, cv)
         return compare_layer(cache, orc, 0, q, Od, rows=rows, check_scores=check_scores, label=w.name)
+
+
+def run_stream(w, track_layers=(0,), compare_every=1, step_filter=None, layer_data=None):
+    """Drive a streaming workload through the library and the oracle; compare tracked layers
+    (every `compare_every` chunks and the last; denoising steps in `step_filter`, or all)."""
+    import torch
+    from paper_2605_09681_gb300 import ForcingKVCache
+    hm = W.head_map(w)
+    orc = O.ForcingKVOracle.from_workload(w, hm, track_layers=list(track_layers))
+    streams = {l: W.FrameStream(w, l) for l in orc.layers}
+    n_cmp = 0
+    with ForcingKVCache.from_workload(w, hm) as cache:
+        for c in range(w.n_chunks):
+            clean = {l: streams[l].frames(w.frames_per_chunk) for l in orc.layers}
+            for d in range(w.denoise_steps):
+                kv = {l: W.step_kv(w, l, c, d, *clean[l]) for l in orc.layers}
+                dev = {l: (to_dev(kv[l][0]), to_dev(kv[l][1])) for l in orc.layers}
+                for l in range(w.n_layers):
+                    src = l if l in dev else orc.layers[0]
+                    if d == 0:
+                        cache.append_chunk(l, *dev[src])
+                    else:
+                        cache.set_current(l, *dev[src])
+                for l in orc.layers:
+                    (orc.append_chunk if d == 0 else orc.set_current)(l, *kv[l])
+                if d == 0:
+                    cache.compress()
+                check = (c % compare_every == 0 or c == w.n_chunks - 1) and (
+                    step_filter is None or d in step_filter)
+                for l in orc.layers:
+                    q = W.queries(w, l, c, d)
+                    Od = cache.attend(l, to_dev(q))
+                    if check:
+                        torch.cuda.synchronize()
+                        rows = sample_rows(q.shape[0], 48, seed=c) if q.shape[0] > 1024 else None
+                        compare_layer(cache, orc, l, q, Od, rows=rows, label="%s c%d d%d" % (w.name, c, d))
+                        n_cmp += 1
+        assert cache.sync_status() == 0
+    return n_cmp

@@ -48,11 +48,12 @@ def test_config_struct_layout():
     from paper_2605_09681_gb300._lib import FkConfig
     assert ctypes.sizeof(FkConfig) == 80
     assert FkConfig.head_is_static.offset == 56
-    assert (FkConfig.selection.offset, FkConfig.select_seed.offset, FkConfig.static_drop_anchor.offset) == (64, 68, 72)
+    assert (FkConfig.selection.offset, FkConfig.select_seed.offset, FkConfig.static_drop_anchor.offset,
+            FkConfig.attn_precision.offset) == (64, 68, 72, 76)
 
 
 def test_abi_version(lib):
-    assert lib.fk_abi_version() == 2
+    assert lib.fk_abi_version() == 3
 
 
 @pytest.mark.parametrize("bad", [
@@ -62,6 +63,7 @@ def test_abi_version(lib):
     dict(score_source=5), dict(incremental=2), dict(window_frames=-1), dict(n_sink_frames=-1),
     dict(window_frames=0, max_history_frames=0), dict(selection=4), dict(selection=-1),
     dict(selection=2, select_scope=1, n_segments=1), dict(static_drop_anchor=2),
+    dict(attn_precision=2), dict(attn_precision=-1), dict(attn_precision=1, head_dim=64),
 ])
 def test_validate_rejects_bad_configs(lib, bad):
     c, _keep = _cfg(**bad)
@@ -76,7 +78,8 @@ def test_validate_accepts_paper_configs(lib):
                dict(n_layers=30, n_heads=12, score_source=1, incremental=1, max_history_frames=21),
                dict(selection=1, n_sink_frames=3, window_frames=4),
                dict(selection=1, window_frames=2, static_drop_anchor=1),
-               dict(selection=2, n_segments=60), dict(selection=3, select_seed=7, n_segments=60)]:
+               dict(selection=2, n_segments=60), dict(selection=3, select_seed=7, n_segments=60),
+               dict(attn_precision=1, head_dim=128)]:
         c, _keep = _cfg(**kw)
         assert lib.fk_validate_config(ctypes.byref(c)) == 0, kw
 
@@ -85,7 +88,7 @@ def test_null_config_and_status_strings(lib):
     assert lib.fk_validate_config(None) == 2
     for s in range(9):
         assert lib.fk_status_str(s)
-    assert lib.fk_abi_version() == 2
+    assert lib.fk_abi_version() == 3
 
 
 @pytest.mark.skipif(os.path.exists("/dev/nvidia0"), reason="checks the no-GPU error path")
@@ -150,3 +153,31 @@ def test_head_profile_rejects_bad_arguments(lib):
     assert call(n_generate=200, n_sink=40, n_transition=40) == FK_ERR_CONFIG
     assert call(n_sink=-1) == FK_ERR_CONFIG
     assert call() == FK_ERR_ARG                                   # host pointers: not device memory
+
+
+def test_quantize_e4m3_rejects_bad_arguments(lib):
+    # argument checks run on the host before any device query
+    buf = np.zeros(4096, dtype=np.float64)
+    p = buf.ctypes.data
+    e = ctypes.cast(p, ctypes.c_void_p)
+    from paper_2605_09681_gb300._lib import FK_ERR_ARG, FK_ERR_CONFIG, FK_OK
+    q = lib.fk_quantize_e4m3
+    assert q(None, 4, 128, 1, p, e, None) == FK_ERR_ARG
+    assert q(p, 4, 128, 0, None, None, None) == FK_ERR_ARG
+    assert q(p + 8, 4, 128, 0, p, None, None) == FK_ERR_ARG            # not 16-byte aligned
+    assert q(p, 4, 128, 1, p, None, None) == FK_ERR_ARG                # exponents required
+    assert q(p, 4, 96, 1, p, e, None) == FK_ERR_CONFIG                 # scaled rows: 64 or 128
+    assert q(p, 4, 12, 0, p, None, None) == FK_ERR_CONFIG              # a multiple of 8
+    assert q(p, 4, 1032, 0, p, None, None) == FK_ERR_CONFIG
+    assert q(p, -1, 128, 0, p, None, None) == FK_ERR_CONFIG
+    assert q(p, 4, 128, 2, p, e, None) == FK_ERR_CONFIG
+    assert q(p, 0, 128, 0, p, None, None) == FK_OK                     # nothing to do
+    assert q(p, 4, 128, 0, p, None, None) == FK_ERR_ARG                # host pointers
+
+
+def test_kernel_kinds_match_header():
+    from paper_2605_09681_gb300 import KERNEL_KINDS
+    text = open(os.path.join(ROOT, "include", "fk.h")).read()
+    for name, v in KERNEL_KINDS.items():
+        assert re.search(r"FK_KERNEL_%s = %d\b" % (name.upper(), v), text), name
+    assert "FK_KERNEL_KINDS = %d" % len(KERNEL_KINDS) in text

@@ -1,0 +1,155 @@
+"""GPU parity of the FP8_QK attention path (Q K^T on E4M3 operands, the paper's quantization
+appendix) through the C ABI: the E4M3 codes and query exponents bit-exact against the
+oracle's rounding, attention within the standard tolerance of the oracle's FP8 attention
+(same quantization, fp64 arithmetic), and within a documented bound of exact attention."""
+import numpy as np
+import pytest
+
+import oracle as O
+import workloads as W
+from fkharness import (compare_layer, run_snapshot, run_stream, sample_rows, snapshot, to_dev,
+                       to_f64)
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+
+# FP8 attention against exact (bf16-input, fp64) attention on the synthetic workloads: the
+# E4M3 rounding of Q and K (relative 2^-4 per element) moves the sharpest heads' outputs by
+# up to ~0.064 (max) / 1.2e-3 (mean) in the oracle's own comparison at 480P
+FP8_VS_EXACT_MAX = 0.15
+FP8_VS_EXACT_MEAN = 4e-3
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _library():
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    from paper_2605_09681_gb300 import build, load_library
+    build.build()
+    load_library()
+
+
+def _decode(codes: np.ndarray) -> np.ndarray:
+    """E4M3 code -> value, from the format's bit fields (sign, 4-bit exponent with bias 7,
+    3-bit mantissa; exponent 0 = subnormal m 2^-9)."""
+    c = codes.astype(np.int64)
+    s, e, m = c >> 7, (c >> 3) & 15, c & 7
+    v = np.where(e == 0, m * 2.0 ** -9, (1 + m / 8) * np.ldexp(1.0, e - 7))
+    assert not np.any((e == 15) & (m == 7)), "NaN code"
+    return np.where(s == 1, -v, v)
+
+
+def _bf16_bits(x: np.ndarray) -> np.ndarray:
+    """Round-to-nearest-even fp32 -> bf16 bit patterns (uint16)."""
+    u = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32).astype(np.uint64)
+    u = (u + 0x7FFF + ((u >> 16) & 1)) >> 16
+    return u.astype(np.uint16)
+
+
+def _bits_to_f64(b: np.ndarray) -> np.ndarray:
+    return (b.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+
+
+def _query_rows(D: int) -> np.ndarray:
+    rng = np.random.default_rng(21 + D)
+    rows = [rng.standard_normal(D) * 2.0 ** k for k in range(-30, 31, 3)]
+    rows.append(np.zeros(D))                                         # e = 0
+    for k in (-3, 0, 5):                                             # amax exactly 448 * 2^k
+        r = rng.uniform(-1, 1, D) * 448.0 * 2.0 ** k
+        r[3] = 448.0 * 2.0 ** k
+        rows.append(r)
+    r = rng.uniform(-1, 1, D) * 450.0                                # just above 448 (e = 1)
+    r[0] = 450.0
+    rows.append(r)
+    grid = np.array([1.0, 1.125, 1.25, 1.375])                       # midpoints of the grid
+    rows.append(np.resize(np.concatenate([grid + 0.0625, -(grid + 0.0625), [448.0]]), D))
+    rows.append(rng.standard_normal(D) * 2.0 ** -128)                # bf16 subnormals
+    rows += [rng.standard_normal(D) for _ in range(200)]
+    return _bf16_bits(np.stack(rows))
+
+
+@pytest.mark.parametrize("D", [64, 128])
+def test_quantize_query_rows_bit_exact(D):
+    from paper_2605_09681_gb300 import quantize_e4m3
+    bits = _query_rows(D)
+    q8, e = quantize_e4m3(to_dev(bits), row_scaled=True)
+    torch.cuda.synchronize()
+    ref_v, ref_e = O.quantize_q_rows(_bits_to_f64(bits))
+    assert np.array_equal(e.cpu().numpy().astype(np.int64), ref_e)
+    assert np.array_equal(_decode(q8.cpu().numpy()), ref_v)
+
+
+@pytest.mark.parametrize("dim", [128, 72])
+def test_quantize_keys_unscaled_bit_exact(dim):
+    from paper_2605_09681_gb300 import quantize_e4m3
+    rng = np.random.default_rng(dim)
+    x = rng.standard_normal((777, dim)) * rng.uniform(0.01, 300.0, size=(777, 1))
+    x[0, :8] = [448.0, 449.0, 464.0, 500.0, -1e4, 2.0 ** -10, 3 * 2.0 ** -10, -2.0 ** -11]
+    bits = _bf16_bits(x)
+    q8, e = quantize_e4m3(to_dev(bits), row_scaled=False)
+    torch.cuda.synchronize()
+    assert e is None
+    assert np.array_equal(_decode(q8.cpu().numpy()), O.e4m3_round(_bits_to_f64(bits)))
+
+
+def _small128(**kw):
+    base = dict(name="small128", n_layers=1, n_heads=4, head_dim=128, tokens_per_frame=200,
+                frames_per_chunk=3, n_sink_frames=1, window_frames=0, n_segments=4,
+                keep_budget_permille=750, schedule="snapshot", n_history_frames=9,
+                static_heads=(0, 2), seed=5, attn_precision="fp8_qk")
+    base.update(kw)
+    return W.Workload(**base)
+
+
+def test_fp8_small_every_row():
+    # 600 queries (4 full query tiles + 88), ragged key tiles, every output row compared
+    st = run_snapshot(_small128())
+    print("fp8 small", st)
+
+
+@pytest.mark.parametrize("budget", [0, 1000])
+def test_fp8_budget_extremes(budget):
+    run_snapshot(_small128(keep_budget_permille=budget, seed=budget + 1))
+
+
+def test_fp8_stream_requantizes_changed_rows():
+    # appends, compressions and denoising steps (fk_set_current) between attention calls: the
+    # E4M3 key copy is refreshed for the current chunk alone after fk_set_current and for
+    # every row after an append; a stale row would show in the next comparison
+    w = W.ROLLING.with_(name="rolling_fp8_small", head_dim=128, tokens_per_frame=64, n_segments=4,
+                        n_heads=4, window_frames=5, n_chunks=8, denoise_steps=3, scene_cut_every_chunks=3,
+                        attn_precision="fp8_qk")
+    assert run_stream(w) == 8 * 3
+
+
+def _layer_fp8_vs_both(w, n_rows):
+    from paper_2605_09681_gb300 import ForcingKVCache
+    hk, hv, ck, cv, q = snapshot(w.with_(attn_precision="bf16"))
+    hm = W.head_map(w)
+    rows = sample_rows(w.n_queries, n_rows)
+    with ForcingKVCache.from_workload(w, hm) as cache:
+        cache.append_frames(0, to_dev(hk), to_dev(hv))
+        cache.set_current(0, to_dev(ck), to_dev(cv))
+        cache.compress()
+        Od = cache.attend(0, to_dev(q))
+        torch.cuda.synchronize()
+        assert cache.sync_status() == 0
+        orc = O.ForcingKVOracle.from_workload(w, hm)
+        orc.append_frames(0, hk, hv)
+        orc.set_current(0, ck, cv)
+        st = compare_layer(cache, orc, 0, q, Od, rows=rows, label=w.name)
+        exact = O.ForcingKVOracle.from_workload(w.with_(attn_precision="bf16"), hm)
+        exact.append_frames(0, hk, hv)
+        exact.set_current(0, ck, cv)
+        err = np.abs(to_f64(Od)[rows] - exact.attend(0, q, rows=rows))
+        st["vs_exact_max"], st["vs_exact_mean"] = float(err.max()), float(err.mean())
+        assert st["vs_exact_max"] <= FP8_VS_EXACT_MAX and st["vs_exact_mean"] <= FP8_VS_EXACT_MEAN, st
+    return st
+
+
+def test_fp8_480p_layer():
+    print("fp8 480p", _layer_fp8_vs_both(W.P480_LAYER_FP8, 96))
+
+
+def test_fp8_1080p_layer():
+    print("fp8 1080p", _layer_fp8_vs_both(W.P1080_LAYER_FP8, 48))

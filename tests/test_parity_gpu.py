@@ -5,8 +5,8 @@ import pytest
 
 import oracle as O
 import workloads as W
-from fkharness import (ATOL_MAX, ATOL_MEAN, compare_layer, run_snapshot, sample_rows, snapshot,
-                       to_dev, to_f64)
+from fkharness import (ATOL_MAX, ATOL_MEAN, compare_layer, run_snapshot, run_stream, sample_rows,
+                       snapshot, to_dev, to_f64)
 
 pytestmark = pytest.mark.gpu
 
@@ -96,47 +96,10 @@ def test_host_pointers_match_device():
 
 
 # ------------------------------------------------------------------ streaming (window, incremental)
-def _stream(w, track_layers=(0,), compare_every=1, step_filter=None, layer_data=None):
-    """Drive a streaming workload through the library and the oracle; compare tracked layers."""
-    from paper_2605_09681_gb300 import ForcingKVCache
-    hm = W.head_map(w)
-    orc = O.ForcingKVOracle.from_workload(w, hm, track_layers=list(track_layers))
-    streams = {l: W.FrameStream(w, l) for l in orc.layers}
-    n_cmp = 0
-    with ForcingKVCache.from_workload(w, hm) as cache:
-        for c in range(w.n_chunks):
-            clean = {l: streams[l].frames(w.frames_per_chunk) for l in orc.layers}
-            for d in range(w.denoise_steps):
-                kv = {l: W.step_kv(w, l, c, d, *clean[l]) for l in orc.layers}
-                dev = {l: (to_dev(kv[l][0]), to_dev(kv[l][1])) for l in orc.layers}
-                for l in range(w.n_layers):
-                    src = l if l in dev else orc.layers[0]
-                    if d == 0:
-                        cache.append_chunk(l, *dev[src])
-                    else:
-                        cache.set_current(l, *dev[src])
-                for l in orc.layers:
-                    (orc.append_chunk if d == 0 else orc.set_current)(l, *kv[l])
-                if d == 0:
-                    cache.compress()
-                check = (c % compare_every == 0 or c == w.n_chunks - 1) and (
-                    step_filter is None or d in step_filter)
-                for l in orc.layers:
-                    q = W.queries(w, l, c, d)
-                    Od = cache.attend(l, to_dev(q))
-                    if check:
-                        torch.cuda.synchronize()
-                        rows = sample_rows(q.shape[0], 48, seed=c) if q.shape[0] > 1024 else None
-                        compare_layer(cache, orc, l, q, Od, rows=rows, label="%s c%d d%d" % (w.name, c, d))
-                        n_cmp += 1
-        assert cache.sync_status() == 0
-    return n_cmp
-
-
 def test_stream_window_small():
     w = W.ROLLING.with_(name="rolling_small", head_dim=64, tokens_per_frame=48, n_heads=4,
                         window_frames=5, n_chunks=12, scene_cut_every_chunks=4)
-    assert _stream(w) == 12
+    assert run_stream(w) == 12
 
 
 def test_incremental_compaction_matches_rebuild():
@@ -190,7 +153,7 @@ def test_stream_incremental_matches_rescore():
 def test_stream_layer0_pooled_small():
     w = W.P480_STACK.with_(name="stack_small", n_layers=3, n_heads=4, head_dim=64,
                            tokens_per_frame=60, n_chunks=5, denoise_steps=2)
-    assert _stream(w, track_layers=(0, 1, 2)) == 5 * 2 * 3
+    assert run_stream(w, track_layers=(0, 1, 2)) == 5 * 2 * 3
 
 
 # ------------------------------------------------------------------ error paths (host-side)
@@ -246,14 +209,14 @@ def test_1080p_layer():
 
 def test_rolling_full():
     w = W.ROLLING
-    assert _stream(w, compare_every=10) >= 6
+    assert run_stream(w, compare_every=10) >= 6
 
 
 def test_480p_stack_full():
     # all 30 layers are appended and compressed; layers 0, 13, 29 carry their own seeded
     # data and are attended and compared (the other layers replay layer 0's inputs)
     w = W.P480_STACK
-    assert _stream(w, track_layers=(0, 13, 29), compare_every=3, step_filter=(0, 3)) > 0
+    assert run_stream(w, track_layers=(0, 13, 29), compare_every=3, step_filter=(0, 3)) > 0
 
 
 @pytest.mark.parametrize("head_dim,F,hist", [(128, 260, 8), (64, 100, 5)])
