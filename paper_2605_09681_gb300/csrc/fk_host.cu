@@ -531,19 +531,21 @@ fk_status fk_quantize_e4m3(const void* X, int64_t rows, int dim, int row_scaled,
   if (row_scaled && !exps) return FK_ERR_ARG;
   if (rows == 0) return FK_OK;
   if (!is_device_ptr(X) || !is_device_ptr(q8) || (row_scaled && !is_device_ptr(exps))) return FK_ERR_ARG;
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  QuantArgs qa{};
   if (row_scaled) {
-    launch_quant_rows_scaled(static_cast<const bf16*>(X), rows, dim, static_cast<uint8_t*>(q8), exps, s);
+    qa.q_src = static_cast<const bf16*>(X);
+    qa.q_dst = static_cast<uint8_t*>(q8);
+    qa.q_exp = exps;
+    qa.q_rows = rows;
+    qa.q_dim = dim;
   } else {
-    QuantRanges qr{};
-    qr.src = static_cast<const bf16*>(X);
-    qr.dst = static_cast<uint8_t*>(q8);
-    qr.D = dim;
-    qr.n = 1;
-    qr.row0[0] = 0;
-    qr.rows[0] = rows;
-    launch_quant_ranges(qr, s);
+    qa.k_src = static_cast<const bf16*>(X);
+    qa.k_dst = static_cast<uint8_t*>(q8);
+    qa.k_dim = dim;
+    qa.n = 1;
+    qa.rows[0] = rows;
   }
+  launch_quant(qa, static_cast<cudaStream_t>(stream));
   return cudaGetLastError() == cudaSuccess ? FK_OK : FK_ERR_CUDA;
 }
 
@@ -1150,24 +1152,24 @@ fk_status fk_attend(fk_handle* h, int layer, const void* Q, void* O, void* strea
   if (h->fp8) {
     // E4M3 queries of this call, and the key rows changed since the layer's last call:
     // the current chunk [0, C*F) and / or the history rows [C*F, n_keys) of every head
-    QuantRanges qr{};
-    qr.src = h->viewK;
-    qr.dst = h->viewK8;
-    qr.D = D;
+    QuantArgs qa{};
+    qa.q_src = q;
+    qa.q_dst = h->q8;
+    qa.q_exp = h->q_exp;
+    qa.q_rows = (int64_t)h->CF * h->H;
+    qa.q_dim = D;
+    qa.k_src = h->viewK;
+    qa.k_dst = h->viewK8;
+    qa.k_dim = D;
     if (!ls.k8_cur_ok || !ls.k8_hist_ok)
       for (int hd = 0; hd < h->H; ++hd) {
         const int lo = ls.k8_cur_ok ? h->CF : 0, hi = ls.k8_hist_ok ? h->CF : a.n_keys[hd];
         if (hi <= lo) continue;
-        qr.row0[qr.n] = a.row_base[hd] + lo;
-        qr.rows[qr.n] = hi - lo;
-        ++qr.n;
+        qa.row0[qa.n] = a.row_base[hd] + lo;
+        qa.rows[qa.n] = hi - lo;
+        ++qa.n;
       }
-    if ((st = launch(h, s, FK_KERNEL_QUANT, [&] {
-           launch_quant_rows_scaled(q, (int64_t)h->CF * h->H, D, h->q8, h->q_exp, s);
-           if (qr.n) launch_quant_ranges(qr, s);
-         })) != FK_OK)
-      return st;
-    if (qr.n) h->launches++;   // the key pass
+    if ((st = launch(h, s, FK_KERNEL_QUANT, [&] { launch_quant(qa, s); })) != FK_OK) return st;
     ls.k8_cur_ok = ls.k8_hist_ok = true;
   }
   const CUtensorMap& tq = h->fp8 ? h->tmQ8 : h->tmQ[qm];

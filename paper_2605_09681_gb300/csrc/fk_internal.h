@@ -177,20 +177,23 @@ void launch_merge(int head_dim, const AttnArgs& a, cudaStream_t s);
 constexpr int kMaxKvSplits = 2;
 
 // ------------------------------------------------------------------ FP8 (E4M3) quantization
-// Unscaled rounding of row ranges of a [rows][D] bf16 arena into the byte arena of the same
-// shape (keys): range i covers rows [row0[i], row0[i] + rows[i]).
-struct QuantRanges {
-  const bf16* src;
-  uint8_t* dst;
-  int D;                        // a multiple of 8
-  int n;                        // ranges, <= kMaxHeads
-  int64_t row0[kMaxHeads];
+// One launch: the query rows (part 0, row-scaled) and key row ranges of a [rows][k_dim] bf16
+// arena (parts 1..n, unscaled) into byte arrays of the same shapes.
+struct QuantArgs {
+  const bf16* q_src;            // [q_rows][q_dim] bf16 (q_rows = 0: no query part)
+  uint8_t* q_dst;               // [q_rows][q_dim] E4M3 codes
+  int8_t* q_exp;                // [q_rows] row exponents
+  int64_t q_rows;
+  int q_dim;                    // 64 or 128
+  const bf16* k_src;            // key arena [rows][k_dim] bf16
+  uint8_t* k_dst;               // its E4M3 copy [rows][k_dim]
+  int k_dim;                    // a multiple of 8
+  int n;                        // key ranges, <= kMaxHeads
+  int64_t row0[kMaxHeads];      // range i: rows [row0[i], row0[i] + rows[i])
   int64_t rows[kMaxHeads];
+  int64_t blk[kMaxHeads + 2];   // first block of each part, set by launch_quant
 };
-void launch_quant_ranges(const QuantRanges& a, cudaStream_t s);
-// Row-scaled rounding of [rows][D] bf16, D = 64 or 128 (queries): exps[r] = e_r.
-void launch_quant_rows_scaled(const bf16* x, int64_t rows, int D, uint8_t* q8, int8_t* exps,
-                              cudaStream_t s);
+void launch_quant(QuantArgs& a, cudaStream_t s);
 
 // ------------------------------------------------------------------ head profiling (Eq. 1)
 struct ProfArgs {
