@@ -503,6 +503,7 @@ def run_fp8(args, w, hm, local_rank, hk, hv, dK, dV, dQ, dO, flush, stream, worl
     quant_bytes = (sum(keys) + nq * w.n_heads) * D * 3 + nq * w.n_heads
     quant_ms = prof["quant"][0] / args.steps
     quant_gbs = quant_bytes / (quant_ms * 1e-3) / 1e9
+    traffic = _traffic("480p_layer") if w.name == "480p_layer" else {}
     return {
         "workload": wf.name if wf.name.endswith("fp8") else wf.name + " (fp8_qk)",
         "ms_per_step": round(total_ms / args.steps, 4),
@@ -512,10 +513,11 @@ def run_fp8(args, w, hm, local_rank, hk, hv, dK, dV, dQ, dO, flush, stream, worl
         "attention": {"us": round(attn_ms * 1e3, 2), "achieved": round(attn_tflops, 1),
                       "unit": "TFLOP/s", "peak": round(mixed_peak, 1),
                       "frac": round(attn_tflops / mixed_peak, 4),
-                      "speedup_vs_bf16_kernel": round(bf16_attn_ms / attn_ms, 3)},
+                      "speedup_vs_bf16_kernel": round(bf16_attn_ms / attn_ms, 3),
+                      "traffic": traffic.get("attend_fp8")},
         "quant": {"bytes": quant_bytes, "us": round(quant_ms * 1e3, 2), "achieved": round(quant_gbs, 1),
                   "unit": "GB/s", "frac": round(quant_gbs / peaks["hbm_gbs"], 4),
-                  "launches_per_step": prof["quant"][1] / args.steps},
+                  "launches_per_step": prof["quant"][1] / args.steps, "traffic": traffic.get("quant")},
         "note": "same algorithmic FLOPs as the bf16 step; Q K^T on E4M3 (kind::f8f6f4), P V bf16; "
                 "the attention is compared with the 4/3 x bf16 mixed peak",
     }
@@ -625,7 +627,9 @@ def run_stack(local_rank):
 # is reported only while that source is unchanged.
 NCU_TRAFFIC = {
     "480p_layer": {
-        "attend": ("fk_attn.cu", "ab1645e4ffd2", 121940224),
+        "attend": ("fk_attn.cu", "165cd65ac773", 118925173),
+        "attend_fp8": ("fk_attn.cu", "165cd65ac773", 84879331),
+        "quant": ("fk_quant.cu", "f49ae0710413", 67233962),
         "compact": ("fk_copy.cu", "b4908ca5adab", 76899072),
         "score": ("fk_score.cu", "b939942305b6", 43160576),
     },

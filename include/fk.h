@@ -9,8 +9,8 @@
  *     with a cosine similarity, keep the floor(b*n) lowest-similarity segments of the
  *     n equal segments of each frame (BottomK, Sec. 4.3, Eq. 3; b = 1 - r, the keep
  *     budget, App. H) and attend to [sink, kept segments, anchor frame, current chunk]
- *     (Sec. 4.3, Eq. 4; the anchor is kept because the dynamic-head cache subsumes the
- *     static portion, Sec. 5.3);
+ *     (Sec. 4.3, Eq. 4; the anchor is kept because a dynamic head's cache holds
+ *     everything a static head keeps, Sec. 5.3);
  *   - compression starts once adjacent history frames exist (App. H); sink frames are
  *     never scored or evicted.
  *
@@ -73,8 +73,9 @@ enum {
 enum {
   FK_SCORE_PER_HEAD = 0,      /* each dynamic head scores its own keys                     */
   FK_SCORE_LAYER0_POOLED = 1  /* keys of every head of layer 0, pooled, score every dynamic
-                                 head of every layer ("the first block ... as a proxy",
-                                 Sec. 4.3); one kept set is shared by all dynamic heads     */
+                                 head of every layer (the first block's keys stand in
+                                 for every layer, Sec. 4.3); one kept set is shared by all
+                                 dynamic heads                                              */
 };
 
 /* Which segments of a scoreable frame dynamic heads keep.  SIMILARITY is the method (Eq. 3);

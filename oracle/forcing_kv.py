@@ -193,8 +193,8 @@ def dynamic_key_tokens(roles: FrameRoles, F: int, n_segments: int, kept: list,
                        current_frames) -> list:
     """Eq. 4 plus the anchor frame: [sink, kept segments (t, j ascending), anchor, current].
 
-    `kept` holds segment ids t*n + j.  The anchor is kept whole: the dynamic cache
-    subsumes the static portion (Sec. 5.3, head-profiling ablation)."""
+    `kept` holds segment ids t*n + j.  The anchor is kept whole: a dynamic head's cache
+    holds everything a static head keeps (Sec. 5.3, head-profiling ablation)."""
     ids = []
     for f in roles.sink:
         ids += frame_tokens(f, F)
