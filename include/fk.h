@@ -208,9 +208,7 @@ FK_API fk_status fk_sync_status(fk_handle* h, void* stream);
  * stream.  fk_profile_read synchronizes and returns, per kernel kind, the total device
  * milliseconds and the number of launches since the last reset. */
 enum { FK_KERNEL_APPEND = 0, FK_KERNEL_SCORE = 1, FK_KERNEL_SELECT = 2, FK_KERNEL_COMPACT = 3,
-       FK_KERNEL_ATTEND = 4, FK_KERNEL_QUANT = 5, FK_KERNEL_KINDS = 6 };
-/* FK_KERNEL_QUANT: the E4M3 quantization of queries and of changed key rows that precedes
- * the attention kernel under FK_ATTN_FP8_QK. */
+       FK_KERNEL_ATTEND = 4, FK_KERNEL_KINDS = 5 };
 FK_API fk_status fk_profile_enable(fk_handle* h, int on);
 FK_API fk_status fk_profile_read(fk_handle* h, int kind, double* total_ms, int64_t* launches);
 FK_API fk_status fk_profile_reset(fk_handle* h);
@@ -306,8 +304,7 @@ FK_API fk_status fk_quantize_e4m3(const void* X, int64_t rows, int dim, int row_
 FK_API const char* fk_status_str(fk_status s);
 
 /* ABI version of this header: 3 (fk_config gained selection, select_seed and
- * static_drop_anchor after head_is_static in version 2, attn_precision in version 3;
- * FK_KERNEL_QUANT was added in version 3). */
+ * static_drop_anchor after head_is_static in version 2, attn_precision in version 3). */
 FK_API int fk_abi_version(void);
 
 #ifdef __cplusplus

@@ -17,7 +17,7 @@ FK_SCOPE_PER_FRAME, FK_SCOPE_POOLED = 0, 1
 FK_SCORE_PER_HEAD, FK_SCORE_LAYER0_POOLED = 0, 1
 FK_SELECT = {"similarity": 0, "all": 1, "uniform": 2, "random": 3}
 FK_ATTN = {"bf16": 0, "fp8_qk": 1}
-KERNEL_KINDS = {"append": 0, "score": 1, "select": 2, "compact": 3, "attend": 4, "quant": 5}
+KERNEL_KINDS = {"append": 0, "score": 1, "select": 2, "compact": 3, "attend": 4}
 
 EXPORTS = [
     "fk_validate_config", "fk_create", "fk_destroy", "fk_append_frames", "fk_append_chunk",

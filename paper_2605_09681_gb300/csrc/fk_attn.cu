@@ -13,10 +13,12 @@
 //                      lazily rescaled running max, writes P as bf16 pairs over S's first
 //                      64 columns with tcgen05.st, and finally normalises O and stores it.
 // TMEM columns: S0 0-127, S1 128-255, O0 256.., O1 256+D.. (512 allocated).
-// FP8_QK variant (D = 128): Q and K tiles hold E4M3 codes (one 128-byte swizzle atom per
-// row), S = Q K^T runs as tcgen05.mma kind::f8f6f4 (K = 32 per instruction), and each
-// softmax thread scales its row's logits by 2^e_row (the query row's quantization exponent)
-// along with 1/sqrt(D); P V is unchanged (bf16).
+// FP8_QK variant (D = 128): the K tiles hold E4M3 codes (one 128-byte swizzle atom per row,
+// from the view arena's E4M3 copy); the bf16 Q tiles are loaded as usual and each softmax
+// thread quantizes its own row into an E4M3 tile (row exponent e_row, codes of the row times
+// 2^-e_row, written in the 128-byte swizzle pattern) before the first MMA; S = Q K^T runs as
+// tcgen05.mma kind::f8f6f4 (K = 32 per instruction) and the thread scales its row's logits by
+// 2^e_row along with 1/sqrt(D); P V is unchanged (bf16).
 // Every mbarrier wait is bounded (%globaltimer); on expiry the CTA records
 // FK_ERR_TIMEOUT in the status word, drains its own TMA loads and MMAs and frees TMEM.
 #include "fk_internal.h"
@@ -37,19 +39,22 @@ struct AttnBarriers {
   uint64_t v_full[2], v_empty[2];
   uint64_t s_full[2], p_full[2];
   uint64_t o_done, fin;
+  uint64_t q8_ready;            // FP8_QK: the 256 softmax threads have written the E4M3 Q rows
   uint32_t tmem_base;
   volatile int abort;
 };
 
 template <int D, bool kFp8 = false>
 struct Layout {
-  static constexpr int kQ = kAttnBM * D * (kFp8 ? 1 : 2);   // one 128-row query tile
+  static constexpr int kQ = kAttnBM * D * (kFp8 ? 1 : 2);   // one 128-row query tile (MMA operand)
   static constexpr int kK = kAttnBN * D * (kFp8 ? 1 : 2);   // one 128-key K tile
   static constexpr int kKV = kAttnBN * D * 2;               // one 128-key V tile (bf16)
+  static constexpr int kQ16 = kFp8 ? kAttnBM * D * 2 : 0;   // FP8: one bf16 query tile as loaded
   static constexpr int kOffQ = 0;                 // two query tiles
   static constexpr int kOffK = kOffQ + 2 * kQ;    // two K stages
   static constexpr int kOffV = kOffK + 2 * kK;    // two V stages
-  static constexpr int kOffBar = kOffV + 2 * kKV;
+  static constexpr int kOffQ16 = kOffV + 2 * kKV; // FP8: two bf16 query tiles
+  static constexpr int kOffBar = kOffQ16 + 2 * kQ16;
   static constexpr int kUsed = kOffBar + 256;
   // at least ~116 KB so that one CTA occupies an SM (its 512 TMEM columns are then free)
   static constexpr int kSmem = (kUsed + 1024) > 118 * 1024 ? (kUsed + 1024) : 118 * 1024;
@@ -295,6 +300,7 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
   uint8_t* sQ = smem + Lay::kOffQ;
   uint8_t* sK = smem + Lay::kOffK;
   uint8_t* sV = smem + Lay::kOffV;
+  uint8_t* sQ16 = smem + Lay::kOffQ16;            // FP8: bf16 query tiles (TMA destination)
   AttnBarriers* bar = reinterpret_cast<AttnBarriers*>(smem + Lay::kOffBar);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -327,6 +333,7 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
     }
     mbar_init(&bar->o_done, 1);
     mbar_init(&bar->fin, 1);
+    if (kFp8) mbar_init(&bar->q8_ready, 2 * kAttnBM);
     bar->abort = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -345,16 +352,14 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
     if (lane == 0) {
       int lastK[2] = {-1, -1}, lastV[2] = {-1, -1};
       bool ok = true;
-      mbar_expect_tx(&bar->q_full, 2 * Lay::kQ);
-      for (int t = 0; t < 2; ++t) {
-        if constexpr (kFp8) {
-          tma_load_3d(sQ + t * Lay::kQ, &tmQ, &bar->q_full, 0, head, q0 + t * kAttnBM);
-        } else {
-          for (int h = 0; h < kHalves; ++h)
-            tma_load_3d(sQ + t * Lay::kQ + h * 16384, &tmQ, &bar->q_full, h * 64, head,
-                        q0 + t * kAttnBM);
-        }
-      }
+      // bf16 query tiles: the MMA operand, or (FP8) the softmax threads' quantization input
+      uint8_t* q_dst = kFp8 ? sQ16 : sQ;
+      constexpr int kQBytes = kAttnBM * D * 2;
+      mbar_expect_tx(&bar->q_full, 2 * kQBytes);
+      for (int t = 0; t < 2; ++t)
+        for (int h = 0; h < kHalves; ++h)
+          tma_load_3d(q_dst + t * kQBytes + h * 16384, &tmQ, &bar->q_full, h * 64, head,
+                      q0 + t * kAttnBM);
       for (int j = 0; j < nt && ok; ++j) {
         const int st = j & 1, u = j >> 1;
         if (j >= 2 && !wait_phase(&bar->k_empty[st], (u - 1) & 1, bar, a.status)) { ok = false; break; }
@@ -422,7 +427,7 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
                   kIdPV, (j > 0 || kk > 0) ? 1u : 0u);
         }
       };
-      bool ok = wait_phase(&bar->q_full, 0, bar, a.status) &&
+      bool ok = wait_phase(kFp8 ? &bar->q8_ready : &bar->q_full, 0, bar, a.status) &&
                 wait_phase(&bar->k_full[0], 0, bar, a.status);
       if (ok) {
         tc_fence_after();
@@ -467,14 +472,38 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
     // logit scale of this row in the log2 domain: log2(e) / sqrt(D), times 2^e_row for E4M3
     // queries (e_row in [-120, 120]: the product is exact)
     float sl2 = a.scale_log2;
+    bool ok = true;
     if constexpr (kFp8) {
-      const int qr = q0 + t * kAttnBM + row;
-      const int e = qr < a.Nq ? (int)a.q_exp[(int64_t)qr * a.H + head] : 0;
-      sl2 *= __uint_as_float((uint32_t)(127 + e) << 23);
+      // quantize this thread's query row: the bf16 row (two 64-element swizzle atoms, 16-byte
+      // chunk j of row r at chunk j ^ (r & 7)) -> max |q| -> e -> E4M3 codes of q 2^-e, 128 bytes
+      // in the same swizzle pattern (rows past Nq were zero-filled: e = 0, codes 0)
+      if (warp_wait(&bar->q_full, 0, bar, a.status)) {
+        const uint8_t* src = sQ16 + t * (kAttnBM * D * 2) + row * 128;
+        uint4 v[16];
+#pragma unroll
+        for (int j = 0; j < 16; ++j)
+          v[j] = *reinterpret_cast<const uint4*>(src + (j >> 3) * 16384 + (((j & 7) ^ (row & 7)) << 4));
+        float amax = 0.0f;
+#pragma unroll
+        for (int j = 0; j < 16; ++j) amax = fmaxf(amax, absmax8(v[j]));
+        const int e = e4m3_row_exponent(amax);
+        const float inv = pow2f(-e);
+        uint8_t* dst = sQ + t * Lay::kQ + row * 128;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const uint2 lo = e4m3x8(v[2 * j], inv), hi = e4m3x8(v[2 * j + 1], inv);
+          *reinterpret_cast<uint4*>(dst + ((j ^ (row & 7)) << 4)) = make_uint4(lo.x, lo.y, hi.x, hi.y);
+        }
+        sl2 *= pow2f(e);
+        // the tensor core reads shared memory through the async proxy
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      } else {
+        ok = false;
+      }
+      mbar_arrive(&bar->q8_ready);
     }
     float m = -INFINITY, l = 0.0f;
-    bool ok = true;
-    for (int j = 0; j < nt; ++j) {
+    for (int j = 0; j < nt && ok; ++j) {
       if (!warp_wait(&bar->s_full[t], j & 1, bar, a.status)) { ok = false; break; }
       tc_fence_after();
       const int valid = nk - j * kAttnBN;           // keys of this tile (< 128 only in the last)

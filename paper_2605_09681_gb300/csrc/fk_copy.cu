@@ -6,6 +6,8 @@
 // anchor frame; attention does not depend on the order of the keys, so a view holds them as
 // [sinks | anchor | kept-segment ring] and incremental compaction only appends).
 // All of them are HBM-bound: every byte is read once and written once in 16-byte accesses.
+// Under FP8_QK attention each of them also writes the E4M3 codes of every view K row it writes
+// (8 bytes per 16-byte granule), so the attention's key operand is ready without another pass.
 #include "fk_internal.h"
 
 namespace fk {
@@ -84,10 +86,12 @@ __global__ void __launch_bounds__(256) current_kernel(const CurrentArgs a) {
     if (to_slot) {
       st_v4(a.viewK[h] + so, ko);
       st_v4(a.viewV[h] + so, vo4);
+      if (a.viewK8[h]) *reinterpret_cast<uint2*>(a.viewK8[h] + so) = e4m3x8(ko, 1.0f);
     }
     if (a.srcK) {
       st_v4(a.viewK[h] + vo, kn);
       st_v4(a.viewV[h] + vo, vn);
+      if (a.viewK8[h]) *reinterpret_cast<uint2*>(a.viewK8[h] + vo) = e4m3x8(kn, 1.0f);
     }
   }
 }
@@ -104,7 +108,11 @@ __global__ void __launch_bounds__(256) scatter_kernel(const ScatterArgs a) {
     const int h = rem / gpr;
     const int c = rem - h * gpr;
     const int64_t dst_off = (int64_t)row * a.head_dim + c * 8;
-    if (a.dstK[h]) st_v4(a.dstK[h] + dst_off, ld_stream(a.srcK + (size_t)g * 8));
+    if (a.dstK[h]) {
+      const uint4 k = ld_stream(a.srcK + (size_t)g * 8);
+      st_v4(a.dstK[h] + dst_off, k);
+      if (a.dstK8[h]) *reinterpret_cast<uint2*>(a.dstK8[h] + dst_off) = e4m3x8(k, 1.0f);
+    }
     if (a.dstV[h]) st_v4(a.dstV[h] + dst_off, ld_stream(a.srcV + (size_t)g * 8));
   }
 }
@@ -166,6 +174,7 @@ __global__ void __launch_bounds__(256) compact_kernel(const CompactArgs a) {
     const uint4* sV = reinterpret_cast<const uint4*>(it.pagesV + src_off);
     uint4* dK = reinterpret_cast<uint4*>(it.viewK + dst_off);
     uint4* dV = reinterpret_cast<uint4*>(it.viewV + dst_off);
+    uint2* dK8 = it.viewK8 ? reinterpret_cast<uint2*>(it.viewK8 + dst_off) : nullptr;
 #pragma unroll
     for (int r = 0; r < kPer; ++r) {
       const int64_t i = g0 + threadIdx.x + r * 256;
@@ -180,16 +189,19 @@ __global__ void __launch_bounds__(256) compact_kernel(const CompactArgs a) {
       if (i < n) {
         st_v4(dK + i, k[r]);
         st_v4(dV + i, v[r]);
+        if (dK8) dK8[i] = e4m3x8(k[r], 1.0f);
       }
     }
     return;
   }
   uint4* dK[kPer];
   uint4* dV[kPer];
+  int64_t e8[kPer];                                      // element offset of the E4M3 copy
 #pragma unroll
   for (int r = 0; r < kPer; ++r) {
     const int64_t gi = threadIdx.x + r * 256;            // granule of this CTA's G units
     dK[r] = nullptr;
+    e8[r] = 0;
     int64_t src_off, dst_off;
     if (gi < G * n && unit_offsets(a, it, blk * G + (int)(gi / n), src_off, dst_off)) {
       const int64_t i = gi - (gi / n) * n;
@@ -197,6 +209,7 @@ __global__ void __launch_bounds__(256) compact_kernel(const CompactArgs a) {
       v[r] = ld_stream(reinterpret_cast<const uint4*>(it.pagesV + src_off) + i);
       dK[r] = reinterpret_cast<uint4*>(it.viewK + dst_off) + i;
       dV[r] = reinterpret_cast<uint4*>(it.viewV + dst_off) + i;
+      e8[r] = dst_off + i * 8;
     }
   }
 #pragma unroll
@@ -204,6 +217,7 @@ __global__ void __launch_bounds__(256) compact_kernel(const CompactArgs a) {
     if (dK[r]) {
       st_v4(dK[r], k[r]);
       st_v4(dV[r], v[r]);
+      if (it.viewK8) *reinterpret_cast<uint2*>(it.viewK8 + e8[r]) = e4m3x8(k[r], 1.0f);
     }
   }
 }

@@ -16,9 +16,9 @@
 //                int64 scoring sums (scratch); status word;
 //                host staging (two slots of K, V and Q; O) and the attention key-split
 //                scratch (fp32 partial outputs and row statistics of two splits).
-//   FP8_QK only  the E4M3 copy of the K view arena ([rows][D] bytes, refreshed before an
-//                attention call for the rows changed since the last one) and the
-//                quantized queries of one call (codes [C*F][H][D], exponents [C*F][H]).
+//   FP8_QK only  the E4M3 copy of the K view arena ([rows][D] bytes, written by the copy
+//                kernels together with every bf16 view K row; the attention kernel
+//                quantizes its query tiles itself).
 #include <algorithm>
 #include <cmath>
 #include <cstdio>
@@ -62,10 +62,6 @@ struct LayerState {
   int ring_end = 0;
   int ring_head = 0;
   int sinks_done = 0;     // sink frames already in the dynamic views
-  // FP8_QK: the E4M3 copy of this layer's K views matches the current-chunk rows / the
-  // history rows (sink, anchor, kept segments)
-  bool k8_cur_ok = false;
-  bool k8_hist_ok = false;
 };
 
 struct Staging {
@@ -182,9 +178,7 @@ struct fk_handle {
   int score_ctas = 0;
   CUtensorMap tmK{}, tmV{};
   uint8_t* viewK8 = nullptr;       // FP8_QK: E4M3 codes of the K view arena
-  uint8_t* q8 = nullptr;           // FP8_QK: E4M3 codes of one call's queries
-  int8_t* q_exp = nullptr;         //         and their row exponents [C*F][H]
-  CUtensorMap tmK8{}, tmQ8{};
+  CUtensorMap tmK8{};
   const void* q_cached[2] = {};   // two cached Q maps (the two Q staging slots alternate)
   CUtensorMap tmQ[2]{};
   int q_next = 0;
@@ -365,15 +359,12 @@ fk_status encode_2d(CUtensorMap* m, void* base, int64_t rows, int D, bool e4m3 =
   return r == CUDA_SUCCESS ? FK_OK : FK_ERR_CUDA;
 }
 
-// 3D map over token-major [Nq][H][D], boxes of 128 rows of one head (as encode_2d)
-fk_status encode_q(CUtensorMap* m, const void* q, int Nq, int H, int D, bool e4m3 = false) {
-  const int es_b = e4m3 ? 1 : 2;
+fk_status encode_q(CUtensorMap* m, const void* q, int Nq, int H, int D) {
   const cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)H, (cuuint64_t)Nq};
-  const cuuint64_t strides[2] = {(cuuint64_t)D * es_b, (cuuint64_t)H * D * es_b};
-  const cuuint32_t box[3] = {e4m3 ? 128u : 64u, 1, (cuuint32_t)kAttnBM};
+  const cuuint64_t strides[2] = {(cuuint64_t)D * 2, (cuuint64_t)H * D * 2};
+  const cuuint32_t box[3] = {64, 1, (cuuint32_t)kAttnBM};
   const cuuint32_t es[3] = {1, 1, 1};
-  CUresult r = g_encode(m, e4m3 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
-                        3, const_cast<void*>(q), dims,
+  CUresult r = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(q), dims,
                         strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
                         CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
@@ -412,6 +403,7 @@ fk_status push_history(fk_handle* h, int layer, const bf16* tokK, const bf16* to
         const int64_t row = h->CF + (int64_t)(sink ? f : h->S) * h->F;
         va.dstK[hd] = hb.viewK + row * h->D;
         va.dstV[hd] = hb.viewV + row * h->D;
+        if (h->fp8) va.dstK8[hd] = h->viewK8 + (hb.row_base + row) * h->D;
         any_v = true;
       }
     }
@@ -426,7 +418,6 @@ fk_status push_history(fk_handle* h, int layer, const bf16* tokK, const bf16* to
   }
   ls.nh = nh1;
   ls.dirty = true;
-  ls.k8_hist_ok = false;
   update_lengths(h, layer);
   return FK_OK;
 }
@@ -465,6 +456,7 @@ fk_status update_current(fk_handle* h, int layer, bool retire, const void* K, co
     a.viewV[hd] = hb.viewV;
     a.pageK[hd] = hb.retains ? hb.pageK : nullptr;
     a.pageV[hd] = hb.retains ? hb.pageV : nullptr;
+    a.viewK8[hd] = h->fp8 ? h->viewK8 + hb.row_base * h->D : nullptr;
     a.is_static[hd] = hb.is_static ? 1 : 0;
   }
   fk_status st = launch(h, s, FK_KERNEL_APPEND, [&] { launch_current(a, s); });
@@ -473,9 +465,7 @@ fk_status update_current(fk_handle* h, int layer, bool retire, const void* K, co
   if (retire) {
     ls.nh += h->C;
     ls.dirty = true;
-    ls.k8_hist_ok = false;
   }
-  if (k) ls.k8_cur_ok = false;
   ls.has_current = k != nullptr || (ls.has_current && !retire);
   update_lengths(h, layer);
   return FK_OK;
@@ -736,10 +726,6 @@ fk_status fk_create(const fk_config* cfg, fk_handle** out) {
   if (h->fp8) {
     if ((st = dev_alloc(h, view_bytes / 2, &p)) != FK_OK) return fail(st);
     h->viewK8 = static_cast<uint8_t*>(p);
-    if ((st = dev_alloc(h, (size_t)h->CF * h->H * h->D, &p)) != FK_OK) return fail(st);
-    h->q8 = static_cast<uint8_t*>(p);
-    if ((st = dev_alloc(h, (size_t)h->CF * h->H, &p)) != FK_OK) return fail(st);
-    h->q_exp = static_cast<int8_t*>(p);
   }
   size_t n_ret = 0;
   for (auto& hb : h->heads) n_ret += hb.retains;
@@ -829,7 +815,8 @@ fk_status fk_create(const fk_config* cfg, fk_handle** out) {
     for (int hd = 0; hd < h->H; ++hd) {
       const HeadBuf& hb = h->heads[l * h->H + hd];
       if (hb.is_static) continue;
-      h->compact_items.push_back({hb.pageK, hb.pageV, hb.viewK, hb.viewV, l, hb.target});
+      h->compact_items.push_back({hb.pageK, hb.pageV, hb.viewK, hb.viewV, l, hb.target,
+                                  h->fp8 ? h->viewK8 + hb.row_base * h->D : nullptr});
     }
   auto upload = [&](const void* src, size_t bytes, void** dst) -> fk_status {
     fk_status s2 = dev_alloc(h, std::max<size_t>(bytes, 16), dst);
@@ -849,10 +836,8 @@ fk_status fk_create(const fk_config* cfg, fk_handle** out) {
 
   if ((st = encode_2d(&h->tmK, h->viewK, h->view_rows_total, h->D)) != FK_OK) return fail(st);
   if ((st = encode_2d(&h->tmV, h->viewV, h->view_rows_total, h->D)) != FK_OK) return fail(st);
-  if (h->fp8) {
-    if ((st = encode_2d(&h->tmK8, h->viewK8, h->view_rows_total, h->D, true)) != FK_OK) return fail(st);
-    if ((st = encode_q(&h->tmQ8, h->q8, h->CF, h->H, h->D, true)) != FK_OK) return fail(st);
-  }
+  if (h->fp8 && (st = encode_2d(&h->tmK8, h->viewK8, h->view_rows_total, h->D, true)) != FK_OK)
+    return fail(st);
   if (cudaDeviceSynchronize() != cudaSuccess) return fail(FK_ERR_CUDA);
   for (int l = 0; l < h->L; ++l) update_lengths(h, l);
   *out = h;
@@ -949,7 +934,6 @@ fk_status fk_compress(fk_handle* h, void* stream) {
   bool any = false;
   for (auto& ls : h->layers) any |= ls.dirty;
   if (!any) return FK_OK;
-  for (auto& ls : h->layers) ls.k8_hist_ok = false;   // views are rebuilt or extended
   const bool pooled_src = h->source == FK_SCORE_LAYER0_POOLED;
   if (pooled_src) {
     for (int l = 1; l < h->L; ++l)
@@ -1096,7 +1080,7 @@ fk_status fk_attend(fk_handle* h, int layer, const void* Q, void* O, void* strea
   fk_status st = check_layer(h, layer);
   if (st != FK_OK) return st;
   if (!Q || !O || !aligned16(Q) || !aligned16(O)) return FK_ERR_ARG;
-  LayerState& ls = h->layers[layer];
+  const LayerState& ls = h->layers[layer];
   if (!ls.has_current || ls.dirty) return FK_ERR_STATE;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   FK_CUDA(cudaSetDevice(h->dev));
@@ -1116,7 +1100,7 @@ fk_status fk_attend(fk_handle* h, int layer, const void* Q, void* O, void* strea
     if (h->o_pending[osl]) FK_CUDA(cudaStreamWaitEvent(s, h->o_copied[osl], 0));
   }
   int qm = q == h->q_cached[0] ? 0 : q == h->q_cached[1] ? 1 : -1;
-  if (qm < 0 && !h->fp8) {
+  if (qm < 0) {
     qm = h->q_next;
     h->q_next ^= 1;
     if ((st = encode_q(&h->tmQ[qm], q, h->CF, h->H, h->D)) != FK_OK) return st;
@@ -1124,7 +1108,6 @@ fk_status fk_attend(fk_handle* h, int layer, const void* Q, void* O, void* strea
   }
   AttnArgs a{};
   a.O = o;
-  a.q_exp = h->q_exp;
   a.Nq = h->CF;
   a.H = h->H;
   a.n_qtiles = (h->CF + 2 * kAttnBM - 1) / (2 * kAttnBM);   // CTA = two 128-row query tiles
@@ -1149,33 +1132,10 @@ fk_status fk_attend(fk_handle* h, int layer, const void* Q, void* O, void* strea
   a.part_o = h->part_o;
   a.part_ml = h->part_ml;
   const int D = h->D;
-  if (h->fp8) {
-    // E4M3 queries of this call, and the key rows changed since the layer's last call:
-    // the current chunk [0, C*F) and / or the history rows [C*F, n_keys) of every head
-    QuantArgs qa{};
-    qa.q_src = q;
-    qa.q_dst = h->q8;
-    qa.q_exp = h->q_exp;
-    qa.q_rows = (int64_t)h->CF * h->H;
-    qa.q_dim = D;
-    qa.k_src = h->viewK;
-    qa.k_dst = h->viewK8;
-    qa.k_dim = D;
-    if (!ls.k8_cur_ok || !ls.k8_hist_ok)
-      for (int hd = 0; hd < h->H; ++hd) {
-        const int lo = ls.k8_cur_ok ? h->CF : 0, hi = ls.k8_hist_ok ? h->CF : a.n_keys[hd];
-        if (hi <= lo) continue;
-        qa.row0[qa.n] = a.row_base[hd] + lo;
-        qa.rows[qa.n] = hi - lo;
-        ++qa.n;
-      }
-    if ((st = launch(h, s, FK_KERNEL_QUANT, [&] { launch_quant(qa, s); })) != FK_OK) return st;
-    ls.k8_cur_ok = ls.k8_hist_ok = true;
-  }
-  const CUtensorMap& tq = h->fp8 ? h->tmQ8 : h->tmQ[qm];
+  // FP8_QK: the E4M3 keys come from the view arena's E4M3 copy; the kernel quantizes Q
   const CUtensorMap& tk = h->fp8 ? h->tmK8 : h->tmK;
   if ((st = launch(h, s, FK_KERNEL_ATTEND, [&] {
-         launch_attention(D, h->fp8, tq, tk, h->tmV, a, s);
+         launch_attention(D, h->fp8, h->tmQ[qm], tk, h->tmV, a, s);
          if (a.kv_splits > 1) launch_merge(D, a, s);
        })) != FK_OK)
     return st;

@@ -29,6 +29,51 @@ constexpr int kScoreTokensPerCta = (kScoreThreads / 32) * 8;
 constexpr int kStatusRange = 1;
 constexpr int kStatusTimeout = 2;
 
+#ifdef __CUDACC__
+// OCP FP8 E4M3 rounding of the FP8_QK attention (hardware cvt.rn.satfinite: to nearest, ties
+// to even, saturating at +-448): two floats -> two codes, `lo` in the low byte
+__device__ __forceinline__ uint32_t e4m3x2(float lo, float hi) {
+  uint16_t r;
+  asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(r) : "f"(hi), "f"(lo));
+  return r;
+}
+// eight bf16 (one 16-byte granule) times `scale` -> eight codes (8 bytes, element order)
+__device__ __forceinline__ uint2 e4m3x8(uint4 v, float scale) {
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+  uint32_t c[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float lo = __uint_as_float(w[i] << 16) * scale;
+    const float hi = __uint_as_float(w[i] & 0xFFFF0000u) * scale;
+    c[i] = e4m3x2(lo, hi);
+  }
+  return make_uint2(c[0] | (c[1] << 16), c[2] | (c[3] << 16));
+}
+// max |x| of eight bf16 (one granule), exact in fp32
+__device__ __forceinline__ float absmax8(uint4 v) {
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+  float m = 0.0f;
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+    m = fmaxf(m, fmaxf(fabsf(__uint_as_float(w[i] << 16)), fabsf(__uint_as_float(w[i] & 0xFFFF0000u))));
+  return m;
+}
+// Query row exponent: the smallest e with amax <= 448 * 2^e, from the bit fields of amax
+// (>= 0).  With amax = 1.f 2^E, i.e. m 2^(E+1) for m = 1.f / 2 in [0.5, 1), and 448 = 0.875 *
+// 2^9: e = E - 8 when m <= 0.875 (1.f <= 1.75: mantissa field <= 0x600000), else E - 7.  Zero
+// gives 0; subnormal amax (below 2^-126) and anything beyond [-120, 120] is clamped.
+__device__ __forceinline__ int e4m3_row_exponent(float amax) {
+  const uint32_t b = __float_as_uint(amax);
+  if (b == 0) return 0;
+  if ((b >> 23) == 0) return -120;
+  const int E = (int)(b >> 23) - 127;
+  const int e = (b & 0x7FFFFFu) <= 0x600000u ? E - 8 : E - 7;
+  return max(-120, min(120, e));
+}
+// 2^k as a float for k in [-126, 127] (exact)
+__device__ __forceinline__ float pow2f(int k) { return __uint_as_float((uint32_t)(127 + k) << 23); }
+#endif
+
 // ------------------------------------------------------------------ copy kernels
 // Current chunk update in one pass: each 16-byte granule of the previous current chunk (in
 // the view fronts) is first copied to its history location, then overwritten by the new
@@ -47,6 +92,7 @@ struct CurrentArgs {
   bf16* viewV[kMaxHeads];
   bf16* pageK[kMaxHeads];       // page rings (nullptr: head keeps no history pages)
   bf16* pageV[kMaxHeads];
+  uint8_t* viewK8[kMaxHeads];   // FP8_QK: E4M3 copies of the K views, same rows (else nullptr)
   unsigned char is_static[kMaxHeads];   // static: sink / anchor slots live in the view
 };
 void launch_current(const CurrentArgs& a, cudaStream_t s);
@@ -59,6 +105,7 @@ struct ScatterArgs {            // token-major [rows][H][D] -> per-head row-majo
   int head_dim;
   bf16* dstK[kMaxHeads];        // nullptr = skip this head
   bf16* dstV[kMaxHeads];
+  uint8_t* dstK8[kMaxHeads];    // FP8_QK view rows: E4M3 copy of dstK (else nullptr)
 };
 void launch_scatter(const ScatterArgs& a, cudaStream_t s);
 
@@ -126,6 +173,7 @@ struct CompactItem {            // one dynamic (layer, head)
   bf16* viewV;
   int layer;
   int target;                   // kept list
+  uint8_t* viewK8;              // FP8_QK: E4M3 copy of the K view, same rows (else nullptr)
 };
 
 struct CompactArgs {
@@ -153,7 +201,6 @@ void launch_compact(const CompactArgs& a, cudaStream_t s);
 // ------------------------------------------------------------------ attention
 struct AttnArgs {
   bf16* O;                      // [Nq][H][D]
-  const int8_t* q_exp;          // FP8_QK: per (query row, head) exponent e, [Nq][H]; else null
   int Nq;
   int H;
   int n_qtiles;
@@ -167,8 +214,9 @@ struct AttnArgs {
   int n_keys[kMaxHeads];        // keys the head attends to
 };
 // tmQ: 3D map over Q [Nq][H][D]; tmK/tmV: 2D maps over the view arenas [rows][D].
-// fp8: Q K^T on E4M3 operands (head_dim 128): tmQ / tmK then map the quantized bytes
-// (box 128 x 128, one 128-byte swizzle atom per row) and a.q_exp holds the query exponents.
+// fp8: Q K^T on E4M3 operands (head_dim 128): tmK then maps the E4M3 key arena (box 128 x 128,
+// one 128-byte swizzle atom per row); tmQ still maps the bf16 queries, which the kernel
+// quantizes itself.
 void launch_attention(int head_dim, bool fp8, const CUtensorMap& tmQ, const CUtensorMap& tmK,
                       const CUtensorMap& tmV, const AttnArgs& a, cudaStream_t s);
 cudaError_t attention_prepare(int head_dim);   // sets the dynamic shared-memory limits

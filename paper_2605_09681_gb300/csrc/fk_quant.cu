@@ -1,12 +1,15 @@
 // FP8 (OCP E4M3) quantization for the FP8_QK attention (the paper's quantization appendix:
-// FP8 attention on the compressed cache).  One HBM-bound streaming launch per attention call
-// covers the query rows and the changed key rows:
+// FP8 attention on the compressed cache): one HBM-bound streaming launch over query rows and /
+// or key row ranges:
 //   queries  row r scaled by 2^-e_r, e_r the smallest integer with max |x_r| <= 448 * 2^e_r,
 //            so the scaling is exact and the E4M3 rounding is the only inexact step;
 //   keys     rounded unscaled (the scoring precondition |K| <= 256 keeps them inside the
 //            E4M3 range; larger magnitudes saturate at 448).
 // The rounding is the hardware conversion cvt.rn.satfinite.e4m3x2.f32 (to nearest, ties to
-// even, saturating to the largest finite value).
+// even, saturating to the largest finite value) and the exponent rule is e4m3_row_exponent,
+// both in fk_internal.h and shared with the attention kernel, which quantizes its own query
+// tiles; the views' E4M3 keys are written by the copy kernels (fk_copy.cu).  This launch
+// serves fk_quantize_e4m3.
 // Work split: every part (the queries, each key range) is cut into chunks of kQuantChunk
 // 16-byte granules of bf16, one chunk per block; thread t converts granules t, t + 256,
 // t + 512 and t + 768 of its chunk, with all four loads issued before the first conversion
@@ -20,48 +23,6 @@ namespace {
 constexpr int kQuantThreads = 256;
 constexpr int kQuantUnroll = 4;
 constexpr int kQuantChunk = kQuantThreads * kQuantUnroll;
-
-// two floats -> two E4M3 codes, `lo` in the low byte
-__device__ __forceinline__ uint32_t e4m3x2(float lo, float hi) {
-  uint16_t r;
-  asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(r) : "f"(hi), "f"(lo));
-  return r;
-}
-
-// eight bf16 (one 16-byte granule) times `scale` -> eight codes (8 bytes, element order)
-__device__ __forceinline__ uint2 e4m3x8(uint4 v, float scale) {
-  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-  uint32_t c[4];
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const float lo = __uint_as_float(w[i] << 16) * scale;
-    const float hi = __uint_as_float(w[i] & 0xFFFF0000u) * scale;
-    c[i] = e4m3x2(lo, hi);
-  }
-  return make_uint2(c[0] | (c[1] << 16), c[2] | (c[3] << 16));
-}
-
-__device__ __forceinline__ float absmax8(uint4 v) {
-  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-  float m = 0.0f;
-#pragma unroll
-  for (int i = 0; i < 4; ++i)
-    m = fmaxf(m, fmaxf(fabsf(__uint_as_float(w[i] << 16)), fabsf(__uint_as_float(w[i] & 0xFFFF0000u))));
-  return m;
-}
-
-// smallest e with amax <= 448 * 2^e, from the bit fields of amax (>= 0): with amax = 1.f 2^E,
-// i.e. m 2^(E+1) for m = 1.f / 2 in [0.5, 1), and 448 = 0.875 * 2^9, e = E - 8 when
-// m <= 0.875 (1.f <= 1.75: mantissa field <= 0x600000), else E - 7.  Subnormal amax (below
-// 2^-126) and zero take the clamp / zero rule.
-__device__ __forceinline__ int row_exponent(float amax) {
-  const uint32_t b = __float_as_uint(amax);
-  if (b == 0) return 0;
-  if ((b >> 23) == 0) return -120;
-  const int E = (int)(b >> 23) - 127;
-  const int e = (b & 0x7FFFFFu) <= 0x600000u ? E - 8 : E - 7;
-  return max(-120, min(120, e));
-}
 
 template <int LANES>   // lanes per query row: D / 8
 __device__ __forceinline__ void quant_query_chunk(const QuantArgs& a, int64_t c0) {
@@ -80,9 +41,9 @@ __device__ __forceinline__ void quant_query_chunk(const QuantArgs& a, int64_t c0
     float m = absmax8(v[k]);
 #pragma unroll
     for (int off = LANES / 2; off >= 1; off >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, off));
-    const int e = row_exponent(m);
+    const int e = e4m3_row_exponent(m);
     if (g < ng) {
-      dst[g] = e4m3x8(v[k], __uint_as_float((uint32_t)(127 - e) << 23));
+      dst[g] = e4m3x8(v[k], pow2f(-e));
       if ((threadIdx.x & (LANES - 1)) == 0) a.q_exp[g / LANES] = (int8_t)e;
     }
   }

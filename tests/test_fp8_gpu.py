@@ -113,9 +113,10 @@ def test_fp8_budget_extremes(budget):
 
 
 def test_fp8_stream_requantizes_changed_rows():
-    # appends, compressions and denoising steps (fk_set_current) between attention calls: the
-    # E4M3 key copy is refreshed for the current chunk alone after fk_set_current and for
-    # every row after an append; a stale row would show in the next comparison
+    # appends, compressions and denoising steps (fk_set_current) between attention calls: every
+    # kernel that writes view K rows (current chunk, retired anchor slot, prefill scatter,
+    # compaction of sinks / anchor / kept segments into the ring) writes their E4M3 copy too;
+    # a stale row would show in the next comparison
     w = W.ROLLING.with_(name="rolling_fp8_small", head_dim=128, tokens_per_frame=64, n_segments=4,
                         n_heads=4, window_frames=5, n_chunks=8, denoise_steps=3, scene_cut_every_chunks=3,
                         attn_precision="fp8_qk")
