@@ -631,9 +631,9 @@ def run_stack(local_rank, attn_precision="bf16"):
 # is reported only while that source is unchanged.
 NCU_TRAFFIC = {
     "480p_layer": {
-        "attend": ("fk_attn.cu", "165cd65ac773", 118925173),
-        "attend_fp8": ("fk_attn.cu", "165cd65ac773", 84879331),
-        "compact": ("fk_copy.cu", "b4908ca5adab", 76899072),
+        "attend": ("fk_attn.cu", "2e17c482d9aa", 118953834),
+        "attend_fp8": ("fk_attn.cu", "2e17c482d9aa", 92209607),
+        "compact": ("fk_copy.cu", "e373e101c0f6", 73879072),
         "score": ("fk_score.cu", "b939942305b6", 43160576),
     },
 }
