@@ -154,3 +154,11 @@ def test_fp8_480p_layer():
 
 def test_fp8_1080p_layer():
     print("fp8 1080p", _layer_fp8_vs_both(W.P1080_LAYER_FP8, 48))
+
+
+def test_fp8_full_kv_key_splits():
+    # equal-length heads (every head keeps the whole window): fk_attend splits each CTA's keys
+    # in two and merges them, so the FP8 instantiation with key splits runs at full size
+    w = W.FULL_KV_480P.with_(name="full_kv_480p_fp8", attn_precision="fp8_qk")
+    st = run_snapshot(w, rows=sample_rows(w.n_queries, 64))
+    print("fp8 full kv", st)
