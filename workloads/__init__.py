@@ -232,11 +232,14 @@ P480_LAYER_FP8 = P480_LAYER.with_(
 P1080_LAYER_FP8 = P1080_LAYER.with_(
     name="1080p_layer_fp8", attn_precision="fp8_qk",
     description="the 1080P layer with Q K^T on FP8 E4M3 operands, P V in bf16")
+TINY_FP8 = TINY_PER_FRAME.with_(
+    name="tiny_fp8", head_dim=128, attn_precision="fp8_qk",
+    description="tiny per-frame case at head_dim 128 with Q K^T on FP8 E4M3 operands")
 
 WORKLOADS = {w.name: w for w in (TINY, TINY_PER_FRAME, P480_LAYER, P480_STACK, ROLLING, P1080_LAYER,
                                  FULL_KV_480P, STREAMINGLLM_480P, DUMMY_FORCING_480P,
                                  UNIFORM_TOKENS_480P, RANDOM_TOKENS_480P, P480_LAYER_FP8,
-                                 P1080_LAYER_FP8)}
+                                 P1080_LAYER_FP8, TINY_FP8)}
 
 
 def head_map(w: Workload) -> np.ndarray:
