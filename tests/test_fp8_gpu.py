@@ -162,3 +162,17 @@ def test_fp8_full_kv_key_splits():
     w = W.FULL_KV_480P.with_(name="full_kv_480p_fp8", attn_precision="fp8_qk")
     st = run_snapshot(w, rows=sample_rows(w.n_queries, 64))
     print("fp8 full kv", st)
+
+
+def test_fp8_stream_layer0_pooled_layers():
+    # three layers with their own seeded data, layer-0 pooled selection, incremental ring views
+    # and 2 denoising steps: every layer's E4M3 key rows sit at that layer's view rows
+    w = W.P480_STACK.with_(name="stack_small_fp8", n_layers=3, n_heads=4, head_dim=128,
+                           tokens_per_frame=60, n_chunks=5, denoise_steps=2, attn_precision="fp8_qk")
+    assert run_stream(w, track_layers=(0, 1, 2)) == 5 * 2 * 3
+
+
+def test_fp8_prefill_sinks_and_window():
+    # two sink frames and a 4-frame window loaded by the prefill (the scatter writes the static
+    # views' sinks and anchor, with their E4M3 copies)
+    run_snapshot(_small128(n_sink_frames=2, window_frames=4, n_history_frames=9, seed=9))
