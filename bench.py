@@ -631,8 +631,8 @@ def run_stack(local_rank, attn_precision="bf16"):
 # is reported only while that source is unchanged.
 NCU_TRAFFIC = {
     "480p_layer": {
-        "attend": ("fk_attn.cu", "2e17c482d9aa", 118953834),
-        "attend_fp8": ("fk_attn.cu", "2e17c482d9aa", 92209607),
+        "attend": ("fk_attn.cu", "06886eb57167", 119274474),
+        "attend_fp8": ("fk_attn.cu", "06886eb57167", 92321365),
         "compact": ("fk_copy.cu", "e373e101c0f6", 73879072),
         "score": ("fk_score.cu", "b939942305b6", 43160576),
     },

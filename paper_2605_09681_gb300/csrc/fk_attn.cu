@@ -21,6 +21,11 @@
 // 2^e_row along with 1/sqrt(D); P V is unchanged (bf16).
 // Every mbarrier wait is bounded (%globaltimer); on expiry the CTA records
 // FK_ERR_TIMEOUT in the status word, drains its own TMA loads and MMAs and frees TMEM.
+// The kernel is launched with programmatic dependent launch: its setup and query loads may
+// overlap the tail of the kernel before it in the stream (the compaction or current-chunk
+// kernel, which write the K/V views), and the TMA thread waits for that kernel
+// (griddepcontrol.wait) before its first K/V load; every global write of this kernel follows
+// MMAs that consume those loads.  It never triggers its own dependents early.
 #include "fk_internal.h"
 
 namespace fk {
@@ -360,6 +365,8 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
         for (int h = 0; h < kHalves; ++h)
           tma_load_3d(q_dst + t * kQBytes + h * 16384, &tmQ, &bar->q_full, h * 64, head,
                       q0 + t * kAttnBM);
+      // the K/V views were written by the previous kernel of the stream
+      asm volatile("griddepcontrol.wait;" ::: "memory");
       for (int j = 0; j < nt && ok; ++j) {
         const int st = j & 1, u = j >> 1;
         if (j >= 2 && !wait_phase(&bar->k_empty[st], (u - 1) & 1, bar, a.status)) { ok = false; break; }
@@ -952,21 +959,31 @@ cudaError_t attention_prepare(int head_dim) {
 
 void launch_attention(int head_dim, bool fp8, const CUtensorMap& tmQ, const CUtensorMap& tmK,
                       const CUtensorMap& tmV, const AttnArgs& a, cudaStream_t s) {
-  const unsigned grid = (unsigned)(a.n_qtiles * a.H * a.kv_splits);
+  using Kern = void (*)(const CUtensorMap, const CUtensorMap, const CUtensorMap, const AttnArgs);
   const bool split = a.kv_splits > 1;
+  Kern kern;
+  int smem;
   if (head_dim == 128 && fp8) {
-    constexpr int sm = Layout<128, true>::kSmem;
-    if (split) attn_kernel<128, true, true><<<grid, kAttnThreads, sm, s>>>(tmQ, tmK, tmV, a);
-    else attn_kernel<128, false, true><<<grid, kAttnThreads, sm, s>>>(tmQ, tmK, tmV, a);
+    kern = split ? attn_kernel<128, true, true> : attn_kernel<128, false, true>;
+    smem = Layout<128, true>::kSmem;
   } else if (head_dim == 128) {
-    constexpr int sm = Layout<128>::kSmem;
-    if (split) attn_kernel<128, true, false><<<grid, kAttnThreads, sm, s>>>(tmQ, tmK, tmV, a);
-    else attn_kernel<128, false, false><<<grid, kAttnThreads, sm, s>>>(tmQ, tmK, tmV, a);
+    kern = split ? attn_kernel<128, true, false> : attn_kernel<128, false, false>;
+    smem = Layout<128>::kSmem;
   } else {
-    constexpr int sm = Layout<64>::kSmem;
-    if (split) attn_kernel<64, true, false><<<grid, kAttnThreads, sm, s>>>(tmQ, tmK, tmV, a);
-    else attn_kernel<64, false, false><<<grid, kAttnThreads, sm, s>>>(tmQ, tmK, tmV, a);
+    kern = split ? attn_kernel<64, true, false> : attn_kernel<64, false, false>;
+    smem = Layout<64>::kSmem;
   }
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3((unsigned)(a.n_qtiles * a.H * a.kv_splits));
+  cfg.blockDim = dim3(kAttnThreads);
+  cfg.dynamicSmemBytes = (size_t)smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cudaLaunchKernelEx(&cfg, kern, tmQ, tmK, tmV, a);
 }
 
 }  // namespace fk
