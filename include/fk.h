@@ -167,14 +167,16 @@ FK_API fk_status fk_set_current(fk_handle* h, int layer, const void* K, const vo
 /* Compress every layer marked by an append: score the new (or, with incremental = 0,
  * all) adjacent frame pairs of the window segment by segment (Eq. 3), select the kept
  * segments (BottomK, ties to the lower segment id) and compact each dynamic head's
- * keys and values into its packed view [current chunk | sink | kept segments | anchor].
+ * keys and values into its packed view [current chunk | sinks | anchor | kept segments]
+ * (attention does not depend on the order of the keys).
  * With no scoreable frame it only rebuilds the views.  Asynchronous on `stream`;
  * FK_ERR_STATE when layer-0 pooled scoring finds layers with different histories. */
 FK_API fk_status fk_compress(fk_handle* h, void* stream);
 
 /* O [C*F][H][D] = per head softmax(Q K^T / sqrt(D)) V over the head's key set: Eq. 2
  * for static heads, Eq. 4 plus the anchor frame for dynamic heads.  Q: [C*F][H][D].
- * FK_ERR_STATE if `layer` has no current chunk or was appended to since the last
+ * Under FK_ATTN_FP8_QK, Q K^T runs on E4M3 operands (the rounding described there; P V in
+ * bf16).  FK_ERR_STATE if `layer` has no current chunk or was appended to since the last
  * fk_compress. */
 FK_API fk_status fk_attend(fk_handle* h, int layer, const void* Q, void* O, void* stream);
 
