@@ -96,11 +96,12 @@ enum {
 /* Operand precision of the chunk attention's Q K^T product (the paper's quantization
  * appendix: FP8 attention on the compressed cache).  BF16: Q, K, V in bf16 (the method).
  * FP8_QK: Q K^T on OCP FP8 E4M3 operands with f32 accumulation; P V stays bf16.  Keys are
- * rounded to E4M3 unscaled (the scoring precondition |K| <= 256 keeps them inside the E4M3
- * range, largest finite 448; larger values saturate); each query row (token, head) is scaled
- * by 2^-e, e the smallest integer with max |q| <= 448 * 2^e, and the logits are scaled back
- * by 2^e, so the E4M3 rounding (to nearest, ties to even) is the only inexact step before
- * the softmax.  fk_quantize_e4m3 applies the same rounding.  FP8_QK requires head_dim 128. */
+ * rounded to E4M3 unscaled (E4M3 keeps the same relative precision over its normal range,
+ * 2^-6 to 448): FP8_QK requires key elements within +-448, larger ones saturate.  Each query
+ * row (token, head) is scaled by 2^-e, e the smallest integer with max |q| <= 448 * 2^e, and
+ * the logits are scaled back by 2^e, so the E4M3 rounding (to nearest, ties to even) is the
+ * only inexact step before the softmax.  fk_quantize_e4m3 applies the same rounding.
+ * FP8_QK requires head_dim 128. */
 enum {
   FK_ATTN_BF16 = 0,
   FK_ATTN_FP8_QK = 1

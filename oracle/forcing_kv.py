@@ -230,8 +230,8 @@ def attention_fp64(Q: np.ndarray, K: np.ndarray, V: np.ndarray, row_block: int =
 # --------------------------------------------------------------------------------------
 # FP8 attention (App. on quantization: FP8 attention on the compressed cache).  The paper
 # names the technique only; the reading taken here: Q K^T on OCP FP8 E4M3 operands, P V
-# unquantised.  K is rounded to e4m3 unscaled (the scoring precondition |K| <= 256 keeps
-# it inside the e4m3 range, largest finite 448); each query row (token, head) is scaled
+# unquantised.  K is rounded to e4m3 unscaled (e4m3's relative precision is the same over
+# its normal range 2^-6..448; elements beyond 448 saturate); each query row (token, head) is scaled
 # by a power of two 2^-e, e the smallest integer with max|q| <= 448 * 2^e, so scaling and
 # unscaling are exact and the only rounding is the e4m3 rounding itself.
 # --------------------------------------------------------------------------------------

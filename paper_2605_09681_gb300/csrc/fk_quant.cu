@@ -3,8 +3,9 @@
 // or key row ranges:
 //   queries  row r scaled by 2^-e_r, e_r the smallest integer with max |x_r| <= 448 * 2^e_r,
 //            so the scaling is exact and the E4M3 rounding is the only inexact step;
-//   keys     rounded unscaled (the scoring precondition |K| <= 256 keeps them inside the
-//            E4M3 range; larger magnitudes saturate at 448).
+//   keys     rounded unscaled (E4M3's relative precision is the same across its normal
+//            range 2^-6..448; key elements beyond 448 saturate, so FP8_QK requires keys
+//            within +-448).
 // The rounding is the hardware conversion cvt.rn.satfinite.e4m3x2.f32 (to nearest, ties to
 // even, saturating to the largest finite value) and the exponent rule is e4m3_row_exponent,
 // both in fk_internal.h and shared with the attention kernel, which quantizes its own query
