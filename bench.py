@@ -634,7 +634,7 @@ NCU_TRAFFIC = {
         "attend": ("fk_attn.cu", "06886eb57167", 119274474),
         "attend_fp8": ("fk_attn.cu", "06886eb57167", 92321365),
         "compact": ("fk_copy.cu", "e373e101c0f6", 73879072),
-        "score": ("fk_score.cu", "b939942305b6", 43160576),
+        "score": ("fk_score.cu", "8a76e34bff85", 43158016),
     },
 }
 

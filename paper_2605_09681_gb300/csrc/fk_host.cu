@@ -955,14 +955,15 @@ fk_status fk_compress(fk_handle* h, void* stream) {
       // comparison rules: no scoring; the selection kernel ranks the whole window by the
       // rule's values
       if (r.n_scoreable > 0) {
-        sa.run[l] = {r.t_lo, r.n_scoreable + 1};
+        sa.run[l] = {r.t_lo, r.n_scoreable + 1, 0};
         any_run = true;
       }
     } else if (ls.dirty && scores_here) {
       const int t_first = h->incremental ? std::max(r.t_lo, ls.scored_upto) : r.t_lo;
       const int last_t = r.t_lo + r.n_scoreable - 1;
       if (r.n_scoreable > 0 && t_first <= last_t) {
-        sa.run[l] = {t_first, last_t + 2 - t_first};
+        // the chunk the last append retired, [nh - C, nh), may still be in flight
+        sa.run[l] = {t_first, last_t + 2 - t_first, std::max(0, ls.nh - h->C)};
         any_run = true;
       }
       ls.scored_upto = r.anchor >= 0 ? r.anchor : ls.scored_upto;

@@ -125,6 +125,8 @@ struct SelectTarget {           // one kept set: its layer and the score items f
 struct LayerRun {               // per layer: frames t_first..t_first+n_run-1 are read
   int t_first;
   int n_run;                    // 0 = nothing to score in this layer
+  int t_fresh;                  // frames >= t_fresh may come from the kernel launched just
+                                // before (the chunk it retired): read after its completion
 };
 
 // Scoring of new frame pairs (score kernel), then the finish of the scores and BottomK

@@ -363,7 +363,7 @@ struct ScoreSmem {
 // Returns false when a wait expired (the status word records it).
 template <int D>
 __device__ __forceinline__ bool score_run(const ScoreArgs& a, int y, int j, int c, int k_first,
-                                          int k_last, uint8_t* smem, uint32_t& seq) {
+                                          int k_last, uint8_t* smem, uint32_t& seq, bool& waited) {
   using L = ScoreSmem<D>;
   constexpr int GPL = D / 32;
   const ScoreItem it = a.items[y];
@@ -392,6 +392,12 @@ __device__ __forceinline__ bool score_run(const ScoreArgs& a, int y, int j, int 
   const bf16* src0 = it.pagesK + (int64_t)tok0 * D;
   const int64_t frame_elems = (int64_t)a.F * D;
   auto issue = [&](int u) {
+    // frames the previous kernel of the stream wrote (the chunk it retired) are read only
+    // after that kernel has completed; older frames stream while it still runs
+    if (!waited && run.t_first + k_load0 + u >= run.t_fresh) {
+      pdl_wait();
+      waited = true;
+    }
     const uint32_t st = (seq + u) % kScoreStages;
     const uint32_t bar = sbase + L::kBarOff + st * 8;
     mbar_expect_tx(bar, bytes);
@@ -493,7 +499,11 @@ __device__ __forceinline__ bool score_run(const ScoreArgs& a, int y, int j, int 
 
 // Persistent grid: the frame-chunks of all scored items (item, segment, token chunk, frame)
 // form one flattened range split into equal contiguous pieces, one per CTA; a piece walks
-// its runs in order.
+// its runs in order.  Launched with programmatic dependent launch after the current-chunk
+// kernel: a CTA streams frames older than the retired chunk while that kernel still runs,
+// waits for it (griddepcontrol.wait, thread 0, before its first fresh frame) and waits in
+// any case before it exits, so this grid completes only after that kernel, and the
+// selection and compaction chained behind it see the retired frames.
 template <int D>
 __global__ void __launch_bounds__(kScoreThreads, 4) score_kernel(const ScoreArgs a) {
   extern __shared__ __align__(128) uint8_t smem[];
@@ -504,7 +514,7 @@ __global__ void __launch_bounds__(kScoreThreads, 4) score_kernel(const ScoreArgs
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   __syncthreads();
-  pdl_wait();                                    // the keys were written by earlier kernels
+  bool waited = false;                           // thread 0: the previous kernel has completed
   const long long T = a.total_units;
   long long g = T * blockIdx.x / gridDim.x;
   const long long g_end = T * (blockIdx.x + 1) / gridDim.x;
@@ -526,10 +536,12 @@ __global__ void __launch_bounds__(kScoreThreads, 4) score_kernel(const ScoreArgs
     const int j = r / a.chunks;
     const long long left = g_end - g;
     const int k_last = (int)(left < run.n_run - k ? k + left - 1 : run.n_run - 1);
-    if (!score_run<D>(a, a.act_first_item[lo] + item_local, j, r - j * a.chunks, k, k_last, smem, seq))
-      return;
+    if (!score_run<D>(a, a.act_first_item[lo] + item_local, j, r - j * a.chunks, k, k_last, smem, seq,
+                      waited))
+      break;
     g += k_last - k + 1;
   }
+  if (threadIdx.x == 0 && !waited) pdl_wait();
 }
 
 template <int D>
