@@ -59,6 +59,22 @@ def _workload(name: str):
     return w.with_(window_frames=window, incremental=False)
 
 
+def _config(w, keys, l2, parallelism):
+    """The workload part of the JSON line's config (shared by both arms) plus the arm's own
+    timing method (l2, parallelism)."""
+    return {
+        "workload": w.name + " streamed through an %d-frame window" % w.window_frames,
+        "heads": w.n_heads, "static_heads": int(sum(_workload_static(w))),
+        "head_dim": w.head_dim, "tokens_per_frame": w.tokens_per_frame,
+        "queries": w.n_queries, "sink_frames": w.n_sink_frames,
+        "history_frames": w.n_history_frames - w.n_sink_frames,
+        "segments": w.n_segments, "keep_budget": w.keep_budget_permille / 1000,
+        "keys_per_head": list(keys), "selection": w.selection,
+        "rescore": "whole window every step" if w.selection == "similarity" else "no scoring (comparison rule)",
+        "l2": l2, "parallelism": parallelism,
+    }
+
+
 def _algorithmic(w, key_counts):
     """Per-step algorithmic work: attention FLOPs sum_h 4*Nq*Nk_h*D; scoring bytes = keys of the
     scored frames of every dynamic head; compaction bytes = keys and values of every dynamic
@@ -307,18 +323,8 @@ def run_fk(args, rank, world, local_rank):
         "vs_baseline": None,
         "dtype": "bf16",
         "data": "synthetic (seeded AR(1) bf16 K/V, iid Q; no model weights)",
-        "config": {
-            "workload": w.name + " streamed through an %d-frame window" % w.window_frames,
-            "heads": w.n_heads, "static_heads": int(sum(_workload_static(w))),
-            "head_dim": w.head_dim, "tokens_per_frame": w.tokens_per_frame,
-            "queries": w.n_queries, "sink_frames": w.n_sink_frames,
-            "history_frames": w.n_history_frames - w.n_sink_frames,
-            "segments": w.n_segments, "keep_budget": w.keep_budget_permille / 1000,
-            "keys_per_head": keys, "selection": w.selection,
-            "rescore": "whole window every step" if w.selection == "similarity" else "no scoring (comparison rule)",
-            "l2": "flushed between timed steps (512 MiB write outside the step events)",
-            "parallelism": "replicas" if world > 1 else "single GPU",
-        },
+        "config": _config(w, keys, l2="flushed between timed steps (512 MiB write outside the step events)",
+                          parallelism="replicas" if world > 1 else "single GPU"),
         "gpu_launches": int(launches),
         "e2e": {"value": round(e2e_value, 3), "unit": "TFLOP/s", "ms_per_step": round(e2e_ms / args.steps, 4),
                 "h2d_bytes_per_step": 3 * nbytes, "d2h_bytes_per_step": nbytes,
@@ -362,6 +368,7 @@ def run_fk(args, rank, world, local_rank):
         out["stack_480p_fp8"] = run_stack(local_rank, "fp8_qk")
     if rank == 0 and not args.no_cpu_baseline:
         out["cpu_baseline"] = cpu_baseline(w, budget_s=args.cpu_seconds)
+        out["cpu_baseline"].pop("keys_per_head", None)
     return out
 
 
@@ -692,7 +699,7 @@ def cpu_baseline(w, budget_s=15.0, steps=1):
                       "step time extrapolated to all rows = %.1f s; BLAS threads = host cores"
                       % (sum(1 for x in hm[0] if not x), t_compress, len(rows), w.n_queries,
                          t_attn, step_s),
-            "step_s": round(step_s, 3)}
+            "step_s": round(step_s, 3), "keys_per_head": keys}
 
 
 def run_reference(args, rank, world):
@@ -713,7 +720,8 @@ def run_reference(args, rank, world):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(secs / args.steps * 1e3, 1),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic (seeded AR(1) bf16 K/V, iid Q; no model weights)",
-        "config": {"workload": w.name + " streamed through an %d-frame window" % w.window_frames},
+        "config": _config(w, r.pop("keys_per_head"), l2="n/a (host CPU)",
+                          parallelism="host cores, rank 0 only"),
         "impl": "reference", "cpu_baseline": r,
         "e2e": {"value": round(value, 6), "unit": "TFLOP/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
