@@ -6,6 +6,8 @@ import socket
 import pytest
 import torch.multiprocessing as mp
 
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
 
 def _free_port():
     s = socket.socket()
@@ -46,3 +48,29 @@ def test_single_rank_needs_no_process_group():
     import bench
     assert bench.reduce_max(3.5, 1) == 3.5
     bench.barrier(1)
+
+
+def test_reference_arm_json_contract():
+    # the oracle arm on the host cores: one JSON line with the base contract's keys, the
+    # reference markers, and the same workload config as the GPU arm
+    import json
+    import subprocess
+    import sys
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference",
+                        "--steps", "1", "--warmup", "3"], capture_output=True, text=True,
+                       timeout=600, cwd=ROOT)
+    assert r.returncode == 0, r.stderr[-2000:]
+    line = json.loads(r.stdout.strip().splitlines()[-1])
+    for k in ("metric", "value", "unit", "n_gpus", "steps", "warmup", "ms_per_step",
+              "higher_is_better", "scaling", "vs_baseline", "dtype", "data", "config", "e2e"):
+        assert k in line, k
+    assert line["impl"] == "reference" and line["value"] > 0 and line["higher_is_better"] is True
+    assert (line["steps"], line["warmup"], line["n_gpus"]) == (1, 3, 1)
+    cb = line["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["sample"] and cb["value"] == line["value"]
+    assert line["e2e"] == {"value": line["value"], "unit": line["unit"], "h2d_bytes_per_step": 0,
+                           "d2h_bytes_per_step": 0}
+    cfg = line["config"]
+    assert cfg["keys_per_head"] == [7800, 7800, 25480, 25480, 25480, 7800, 7800, 25480, 7800,
+                                    25480, 7800, 25480]
+    assert cfg["queries"] == 4680 and cfg["head_dim"] == 128 and cfg["heads"] == 12
