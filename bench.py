@@ -638,8 +638,8 @@ def run_stack(local_rank, attn_precision="bf16"):
 # is reported only while that source is unchanged.
 NCU_TRAFFIC = {
     "480p_layer": {
-        "attend": ("fk_attn.cu", "06886eb57167", 119274474),
-        "attend_fp8": ("fk_attn.cu", "06886eb57167", 92321365),
+        "attend": ("fk_attn.cu", "da6b58031078", 119412117),
+        "attend_fp8": ("fk_attn.cu", "da6b58031078", 92557994),
         "compact": ("fk_copy.cu", "e373e101c0f6", 73879072),
         "score": ("fk_score.cu", "8a76e34bff85", 43158016),
     },

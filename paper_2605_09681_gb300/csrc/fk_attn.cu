@@ -21,11 +21,11 @@
 // 2^e_row along with 1/sqrt(D); P V is unchanged (bf16).
 // Every mbarrier wait is bounded (%globaltimer); on expiry the CTA records
 // FK_ERR_TIMEOUT in the status word, drains its own TMA loads and MMAs and frees TMEM.
-// The kernel is launched with programmatic dependent launch: its setup and query loads may
+// The kernel is launched with programmatic dependent launch: its setup (barriers, TMEM) may
 // overlap the tail of the kernel before it in the stream (the compaction or current-chunk
-// kernel, which write the K/V views), and the TMA thread waits for that kernel
-// (griddepcontrol.wait) before its first K/V load; every global write of this kernel follows
-// MMAs that consume those loads.  It never triggers its own dependents early.
+// kernel, which write the K/V views, or whatever kernel produced Q), and the TMA thread waits
+// for that kernel (griddepcontrol.wait) before its first load; every global write of this
+// kernel follows MMAs that consume those loads.  It never triggers its own dependents early.
 #include "fk_internal.h"
 
 namespace fk {
@@ -357,6 +357,8 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
     if (lane == 0) {
       int lastK[2] = {-1, -1}, lastV[2] = {-1, -1};
       bool ok = true;
+      // Q, K and V may have been written by the previous kernel of the stream
+      asm volatile("griddepcontrol.wait;" ::: "memory");
       // bf16 query tiles: the MMA operand, or (FP8) the softmax threads' quantization input
       uint8_t* q_dst = kFp8 ? sQ16 : sQ;
       constexpr int kQBytes = kAttnBM * D * 2;
@@ -365,8 +367,6 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
         for (int h = 0; h < kHalves; ++h)
           tma_load_3d(q_dst + t * kQBytes + h * 16384, &tmQ, &bar->q_full, h * 64, head,
                       q0 + t * kAttnBM);
-      // the K/V views were written by the previous kernel of the stream
-      asm volatile("griddepcontrol.wait;" ::: "memory");
       for (int j = 0; j < nt && ok; ++j) {
         const int st = j & 1, u = j >> 1;
         if (j >= 2 && !wait_phase(&bar->k_empty[st], (u - 1) & 1, bar, a.status)) { ok = false; break; }
