@@ -74,3 +74,18 @@ def test_reference_arm_json_contract():
     assert cfg["keys_per_head"] == [7800, 7800, 25480, 25480, 25480, 7800, 7800, 25480, 7800,
                                     25480, 7800, 25480]
     assert cfg["queries"] == 4680 and cfg["head_dim"] == 128 and cfg["heads"] == 12
+
+
+def test_algorithmic_work_of_the_480p_step():
+    # the figures every roofline fraction divides by, worked out by hand for the 480P layer:
+    # 6 static heads see 7800 keys (current 4680 + sink 1560 + anchor 1560), 6 dynamic heads
+    # 25480 (current + sink + anchor + 17 frames x 4 kept segments x 260 tokens)
+    import bench
+    w = bench._workload("480p_layer")
+    keys = [7800] * 6 + [25480] * 6
+    alg = bench._algorithmic(w, keys)
+    assert alg["attn_flops"] == 4 * 4680 * 128 * (6 * 7800 + 6 * 25480)            # 478.47 GFLOP
+    assert alg["score_bytes"] == 6 * 18 * 1560 * 128 * 2                           # 43.13 MB
+    assert alg["compact_bytes"] == 6 * (1560 + 17 * 4 * 260 + 1560) * 128 * 2 * 2 * 2  # 127.8 MB
+    cfg = bench._config(w, keys, l2="x", parallelism="y")
+    assert cfg["queries"] == 4680 and cfg["history_frames"] == 18 and cfg["keys_per_head"] == keys
