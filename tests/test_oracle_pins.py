@@ -124,6 +124,91 @@ def test_token_dot_within_fp32_error_bound(D):
     assert (err <= bound * 1.0001 + 1e-30).all()
 
 
+def _contract_golden():
+    """Tokens of tests/golden/contract_token_dot.txt: (name, D, a, b, values by column)."""
+    cols = ("contract", "exact", "rev", "strd", "desc", "last2", "first2", "short", "n_a", "n_b")
+    out = []
+    for line in open(os.path.join(GOLDEN, "contract_token_dot.txt")):
+        line = line.split("#")[0].strip()
+        if not line:
+            continue
+        head, a_s, b_s, vals, alts, norms = (p.strip() for p in line.split("|"))
+        name, D = head.split()
+        D = int(D)
+        vec = []
+        for spec in (a_s, b_s):
+            v = np.zeros(D, dtype=np.float32)
+            for item in spec.split():
+                c, x = item.split(":")
+                v[int(c)] = float(x)
+            vec.append(v)
+        nums = [float(x) for x in (vals + " " + alts + " " + norms).split()]
+        out.append((name, D, vec[0], vec[1], dict(zip(cols, nums))))
+    return out
+
+
+def _dot_in_order(a, b, D, variant):
+    """The per-token dot under the contract ("contract") or one of the misreadings recorded in
+    the golden file, for inputs whose products are exact (fp64 sums of them are exact too)."""
+    G = D // 8
+    groups = [list(range(8 * g, 8 * g + 8)) for g in range(G)]
+    if variant == "strd":
+        groups = [[g + G * i for i in range(8)] for g in range(G)]
+    if variant == "desc":
+        groups = [grp[::-1] for grp in groups]
+    p = []
+    for grp in groups:
+        acc = np.float32(0.0)
+        for c in grp:
+            acc = np.float32(float(a[c]) * float(b[c]) + float(acc))
+        p.append(acc)
+    strides = [G >> k for k in range(1, G.bit_length())]      # G/2, ..., 2, 1
+    if variant == "rev":
+        strides = strides[::-1]
+    elif variant == "last2":
+        strides = strides[:-2] + [strides[-1], strides[-2]]
+    elif variant == "first2":
+        strides = [strides[1], strides[0]] + strides[2:]
+    elif variant == "short":
+        strides = strides[1:]
+    for s in strides:
+        p = [np.float32(p[g] + p[g ^ s]) for g in range(G)]
+    return float(p[0])
+
+
+def test_contract_token_dot_golden():
+    # hand-worked values (tests/golden/contract_token_dot.txt): the oracle's per-token dot and
+    # self-dots equal them bit for bit, so a reordered butterfly or a regrouped / reversed fma
+    # chain in the oracle fails here
+    toks = _contract_golden()
+    assert {D for _, D, *_ in toks} == {64, 128}
+    for name, D, a, b, v in toks:
+        A, B = a[None, :], b[None, :]
+        assert O.token_dots_contract(A, B)[0] == np.float32(v["contract"]), name
+        assert O.token_dots_contract(A, A)[0] == np.float32(v["n_a"]), name
+        assert O.token_dots_contract(B, B)[0] == np.float32(v["n_b"]), name
+        assert float(np.dot(a.astype(np.float64), b.astype(np.float64))) == v["exact"], name
+        # a one-token segment pair: N1 = n_a 2^24, N2 = n_b 2^24, Dsum = d 2^24, so
+        # s = d / sqrt(n_a n_b) exactly (here d 2^-21: 2^-24 or 2^-25)
+        s = O.segment_score_contract(A, B)
+        assert s == np.float32(v["contract"] / math.sqrt(v["n_a"] * v["n_b"])), name
+
+
+def test_contract_golden_file_is_consistent_and_discriminating():
+    # the recorded misreadings are what those orders give (each row's hand derivation is
+    # replayed in plain fp32 steps), and every misreading changes at least one token per D
+    toks = _contract_golden()
+    variants = ("rev", "strd", "desc", "last2", "first2", "short")
+    for name, D, a, b, v in toks:
+        assert _dot_in_order(a, b, D, "contract") == v["contract"], name
+        for var in variants:
+            assert _dot_in_order(a, b, D, var) == v[var], (name, var)
+    for D in (64, 128):
+        rows = [v for _, d, _, _, v in toks if d == D]
+        for var in variants:
+            assert any(r[var] != r["contract"] for r in rows), (D, var)
+
+
 def test_fixed_point_truncates_toward_zero():
     x = np.array([1.5, -1.5, 2.0 ** -25, -(2.0 ** -25), 3.0, 0.0], dtype=np.float64) * 2.0 ** -24
     assert O.fixed_point(x).tolist() == [1, -1, 0, 0, 3, 0]
