@@ -107,26 +107,36 @@ enum {
   FK_ATTN_FP8_QK = 1
 };
 
+/* Configuration of one cache.  The method's quantities (Sec. 4.2-4.3 and App. H): F tokens per
+ * frame and C frames per chunk (Eq. 2: the current chunk is tokens iCF..(i+1)CF-1); the sink
+ * frames preserved at the start of the video (App. H); n segments per frame and the keep budget
+ * b = 1 - r of dynamic heads (App. H sets n = 6, r = 0.3; Eq. 3 keeps the floor(b n) lowest-
+ * similarity segments); the static/dynamic head map produced by offline head profiling (Sec. 4.1,
+ * Eq. 1).  The remaining fields choose this library's execution (window capacity, selection
+ * scope and proxy, incremental scoring, device, the paper's comparison rules, FP8). */
 typedef struct fk_config {
   int32_t n_layers;             /* 1..256                                                  */
   int32_t n_heads;              /* 1..128                                                  */
   int32_t head_dim;             /* 64 or 128                                               */
-  int32_t tokens_per_frame;     /* F >= 1, a multiple of n_segments                        */
-  int32_t frames_per_chunk;     /* C >= 1                                                  */
-  int32_t n_sink_frames;        /* S >= 0: frames 0..S-1 are sinks, never evicted          */
+  int32_t tokens_per_frame;     /* F >= 1, a multiple of n_segments (Eq. 2, App. H)        */
+  int32_t frames_per_chunk;     /* C >= 1 (Eq. 2)                                          */
+  int32_t n_sink_frames;        /* S >= 0: frames 0..S-1 are sinks, never evicted (App. H) */
   int32_t window_frames;        /* W >= 0 non-sink history frames kept, anchor included;
-                                   0 = unbounded (capacity max_history_frames)            */
-  int32_t n_segments;           /* n >= 1 contiguous equal segments per frame              */
-  int32_t keep_budget_permille; /* b*1000 in [0, 1000]; k = floor(b*n) kept per frame      */
+                                   0 = unbounded (capacity max_history_frames); the model's
+                                   own attention window (App. H)                           */
+  int32_t n_segments;           /* n >= 1 contiguous equal segments per frame (App. H)     */
+  int32_t keep_budget_permille; /* b*1000 in [0, 1000]; k = floor(b*n) kept per frame
+                                   (Eq. 3 with b = 1 - r; App. H: r = 0.3)                */
   int32_t select_scope;         /* FK_SCOPE_*                                              */
-  int32_t score_source;         /* FK_SCORE_*                                              */
+  int32_t score_source;         /* FK_SCORE_* (Sec. 4.3: the first block's keys as proxy)  */
   int32_t incremental;          /* 1: fk_compress scores only frame pairs not scored yet
                                    (a frame's pairs never change once both frames exist);
                                    0: every fk_compress rescores the whole window         */
   int32_t max_history_frames;   /* history capacity in frames, sinks included, when W = 0 */
   int32_t device;               /* CUDA device ordinal                                     */
-  const uint8_t* head_is_static;/* host [n_layers*n_heads]: 1 = static head, 0 = dynamic;
-                                   copied by fk_create                                     */
+  const uint8_t* head_is_static;/* host [n_layers*n_heads]: 1 = static head, 0 = dynamic
+                                   (the classification of Sec. 4.1, Eq. 1); copied by
+                                   fk_create                                               */
   int32_t selection;            /* FK_SELECT_* (0 = the method)                            */
   uint32_t select_seed;         /* seed of FK_SELECT_RANDOM                                */
   int32_t static_drop_anchor;   /* 1: static heads keep sink + current chunk only (Dummy
@@ -140,8 +150,12 @@ typedef struct fk_handle fk_handle;
  * FK_ERR_ARG.  fk_create runs the same checks first. */
 FK_API fk_status fk_validate_config(const fk_config* cfg);
 
-/* Create a cache on cfg->device and allocate all of its device memory.
- * *out receives the handle (NULL on failure). */
+/* Create a cache on cfg->device and allocate all of its device memory: per head the packed
+ * view of its key set (Eq. 2 for static heads, Eq. 4 plus the anchor for dynamic heads) and,
+ * for dynamic heads, the history pages that scoring reads (the paper keeps history frames for
+ * similarity computation, Sec. 5.2).  *out receives the handle (NULL on failure).  Errors:
+ * FK_ERR_CONFIG / FK_ERR_ARG as fk_validate_config, FK_ERR_CUDA (no device, kernel setup),
+ * FK_ERR_NOMEM (allocation). */
 FK_API fk_status fk_create(const fk_config* cfg, fk_handle** out);
 
 /* Release the handle and its device memory (synchronizes the device first). NULL is a no-op. */
@@ -182,7 +196,9 @@ FK_API fk_status fk_compress(fk_handle* h, void* stream);
 FK_API fk_status fk_attend(fk_handle* h, int layer, const void* Q, void* O, void* stream);
 
 /* Bytes of device memory currently holding live cache state: retained history pages,
- * the used part of every packed view (current chunk included), scores and kept lists. */
+ * the used part of every packed view (current chunk included), scores and kept lists.  The
+ * cache-memory figure of Sec. 5.2 (KV memory of the compressed cache; the paper notes that
+ * dynamic heads also keep history frames for similarity computation, counted here). */
 FK_API size_t fk_cache_bytes(const fk_handle* h);
 
 /* Bytes of device memory the handle allocated (all buffers, live or not). */
@@ -192,7 +208,8 @@ FK_API size_t fk_reserved_bytes(const fk_handle* h);
 FK_API fk_status fk_key_count(const fk_handle* h, int layer, int head, int* n_keys);
 
 /* Kept segment ids (t*n + j, ascending) of dynamic head (layer, head) after the last
- * fk_compress; *n_out = 0 for a static head.  Synchronizes `stream`.  FK_ERR_ARG if
+ * fk_compress: the index set I_keep of Eq. 3 (Sec. 4.3); *n_out = 0 for a static head.  `out`
+ * is caller-owned host memory of `capacity` ints.  Synchronizes `stream`.  FK_ERR_ARG if
  * capacity is too small (then *n_out holds the required count). */
 FK_API fk_status fk_get_kept(fk_handle* h, int layer, int head, int32_t* out, int capacity, int* n_out,
                       void* stream);
@@ -254,17 +271,22 @@ FK_API int64_t fk_launch_count(const fk_handle* h);
  * first, 16-byte aligned).  scores: device memory [n_frames - 1][n_segments] fp32; on
  * completion scores[t][j] = s_t^(j), the cosine of segment j of frames t and t+1 (Eq. 3) under
  * the same score contract as fk_compress, bit-identical to fk_get_scores for the same frames.
- * Requires every token's contract squared key norm <= 2^23 (else the scores are unspecified).
+ * status: NULL, or a caller-owned device int that the caller zeroes; the kernels OR into it the
+ * conditions fk_sync_status would report for a handle: 1 when a token's contract squared key
+ * norm exceeds 2^23 (the condition of FK_ERR_RANGE: the scores are then unspecified) and 2 when
+ * a bounded device wait expired (the condition of FK_ERR_TIMEOUT: the scores are undefined).
+ * With status NULL these conditions go unreported.
  * Limits: head_dim 64 or 128, 2 <= n_frames <= 256, 1 <= n_segments <= 32, n_frames *
  * n_segments <= 4096, tokens_per_frame a multiple of n_segments; larger sizes return
- * FK_ERR_CONFIG, host pointers FK_ERR_ARG.  The scratch is one fixed 65,728-byte array per
- * device that loads the library (held until the process exits), shared by every call: calls
- * whose work overlaps on the GPU (e.g. on two streams) race and must be ordered by the caller.
- * The first call on a device resolves that array's address and must come before any stream
- * capture.  Asynchronous on `stream`; uses the current device. */
+ * FK_ERR_CONFIG; host, null (K, scores) or misaligned pointers FK_ERR_ARG.  The scratch is one
+ * fixed 65,728-byte array per device that loads the library (held until the process exits),
+ * shared by every call and holding the last call's contents (each call clears what must start
+ * at zero): calls whose work overlaps on the GPU (e.g. on two streams) race and must be ordered
+ * by the caller.  The first call on a device resolves that array's address and must come before
+ * any stream capture.  Asynchronous on `stream`; uses the current device. */
 FK_API fk_status fk_segment_scores_noalloc(const void* K, int n_frames, int tokens_per_frame,
                                            int head_dim, int n_segments, float* scores,
-                                           void* stream);
+                                           int* status, void* stream);
 
 /* Offline head profiling (Sec. 4.1, Eq. 1): attention mass per key class.
  * Q: device [n_queries][n_heads][head_dim] bf16, the queries of the generated chunk.
@@ -306,8 +328,9 @@ FK_API fk_status fk_quantize_e4m3(const void* X, int64_t rows, int dim, int row_
 /* Static text for a status code. */
 FK_API const char* fk_status_str(fk_status s);
 
-/* ABI version of this header: 3 (fk_config gained selection, select_seed and
- * static_drop_anchor after head_is_static in version 2, attn_precision in version 3). */
+/* ABI version of this header: 4 (fk_config gained selection, select_seed and
+ * static_drop_anchor after head_is_static in version 2, attn_precision in version 3;
+ * fk_segment_scores_noalloc gained its status argument in version 4). */
 FK_API int fk_abi_version(void);
 
 #ifdef __cplusplus

@@ -89,7 +89,7 @@ def load(path: str | None = None) -> ctypes.CDLL:
         "fk_wait_outputs": (st, [vp, vp]),
         "fk_status_str": (cp, [i32]),
         "fk_abi_version": (i32, []),
-        "fk_segment_scores_noalloc": (st, [vp, i32, i32, i32, i32, vp, vp]),
+        "fk_segment_scores_noalloc": (st, [vp, i32, i32, i32, i32, vp, vp, vp]),
         "fk_head_profile": (st, [vp, vp, i32, i32, i32, i32, i32, i32, i32, vp, vp, vp]),
         "fk_classify_heads": (st, [ctypes.POINTER(ctypes.c_double), i32, i32,
                                    ctypes.POINTER(ctypes.c_uint8)]),

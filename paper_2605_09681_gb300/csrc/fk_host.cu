@@ -578,7 +578,7 @@ fk_status fk_wait_outputs(fk_handle* h, void* stream) {
   return FK_OK;
 }
 
-int fk_abi_version(void) { return 3; }
+int fk_abi_version(void) { return 4; }
 
 const char* fk_status_str(fk_status s) {
   switch (s) {

@@ -669,6 +669,7 @@ constexpr size_t kNoAllocItemOff = kNoAllocCtrOff + 64;
 constexpr size_t kNoAllocTargetOff = kNoAllocItemOff + 64;
 constexpr size_t kNoAllocBytes = kNoAllocTargetOff + 64;   // 65,728 bytes
 static_assert(kNoAllocBytes == 65728, "documented size");
+static_assert(sizeof(ScoreItem) <= 64 && sizeof(SelectTarget) <= 32, "table slots");
 
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocBytes];
 
@@ -690,15 +691,30 @@ bool device_pointer(const void* p) {
   return at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged;
 }
 
+// Prepares the scratch array for one call: zeroes the first n_words int64 sums and the status
+// word, and writes the one-entry item table (K arrives as a kernel parameter, so no host memory
+// is read) and the one-entry target table.
+__global__ void noalloc_setup_kernel(unsigned char* sc, const bf16* K, int n_words) {
+  unsigned long long* sums = reinterpret_cast<unsigned long long*>(sc);
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n_words; i += gridDim.x * blockDim.x)
+    sums[i] = 0ull;
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    reinterpret_cast<int*>(sc + kNoAllocCtrOff)[3] = 0;
+    *reinterpret_cast<ScoreItem*>(sc + kNoAllocItemOff) = ScoreItem{K, 0, 0};
+    *reinterpret_cast<SelectTarget*>(sc + kNoAllocTargetOff) = SelectTarget{0, 0, 1};
+  }
+}
+
 }  // namespace
 }  // namespace fk
 
 extern "C" fk_status fk_segment_scores_noalloc(const void* K, int n_frames, int tokens_per_frame,
                                                 int head_dim, int n_segments, float* scores,
-                                                void* stream) {
+                                                int* status, void* stream) {
   using namespace fk;
   if (!K || !scores) return FK_ERR_ARG;
-  if ((reinterpret_cast<uintptr_t>(K) & 15u) || (reinterpret_cast<uintptr_t>(scores) & 3u))
+  if ((reinterpret_cast<uintptr_t>(K) & 15u) || (reinterpret_cast<uintptr_t>(scores) & 3u) ||
+      (reinterpret_cast<uintptr_t>(status) & 3u))
     return FK_ERR_ARG;
   if (head_dim != 64 && head_dim != 128) return FK_ERR_CONFIG;
   if (n_segments < 1 || n_segments > kNoAllocMaxSegments) return FK_ERR_CONFIG;
@@ -706,7 +722,8 @@ extern "C" fk_status fk_segment_scores_noalloc(const void* K, int n_frames, int 
   if ((int64_t)tokens_per_frame * head_dim > (1 << 28)) return FK_ERR_CONFIG;
   if (n_frames < 2 || n_frames > kNoAllocMaxFrames || n_frames * n_segments > kNoAllocMaxCells)
     return FK_ERR_CONFIG;
-  if (!device_pointer(K) || !device_pointer(scores)) return FK_ERR_ARG;
+  if (!device_pointer(K) || !device_pointer(scores) || (status && !device_pointer(status)))
+    return FK_ERR_ARG;
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kNoAllocMaxDevices) {
     cudaGetLastError();
@@ -732,22 +749,10 @@ extern "C" fk_status fk_segment_scores_noalloc(const void* K, int n_frames, int 
   }
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   unsigned char* sc = nd.scratch;
-  // the sums and the status word must start at zero; the previous call leaves the sums
-  // cleared, but clear them here anyway
-  const size_t sums_bytes = (size_t)n_frames * n_segments * 2 * sizeof(unsigned long long);
-  if (cudaMemsetAsync(sc, 0, sums_bytes, s) != cudaSuccess ||
-      cudaMemsetAsync(sc + kNoAllocCtrOff, 0, 64, s) != cudaSuccess) {
-    cudaGetLastError();
-    return FK_ERR_CUDA;
-  }
-  const ScoreItem item{static_cast<const bf16*>(K), 0, 0};
-  const SelectTarget target{0, 0, 1};
-  if (cudaMemcpyAsync(sc + kNoAllocItemOff, &item, sizeof(item), cudaMemcpyHostToDevice, s) != cudaSuccess ||
-      cudaMemcpyAsync(sc + kNoAllocTargetOff, &target, sizeof(target), cudaMemcpyHostToDevice, s) !=
-          cudaSuccess) {
-    cudaGetLastError();
-    return FK_ERR_CUDA;
-  }
+  // the sums and the status word must start at zero: the previous call leaves the sums
+  // cleared, but the setup kernel clears them anyway (and writes the tables)
+  const int n_words = n_frames * n_segments * 2;
+  noalloc_setup_kernel<<<(n_words + 255) / 256, 256, 0, s>>>(sc, static_cast<const bf16*>(K), n_words);
   ScoreArgs a{};
   a.items = reinterpret_cast<const ScoreItem*>(sc + kNoAllocItemOff);
   a.targets = reinterpret_cast<const SelectTarget*>(sc + kNoAllocTargetOff);
@@ -771,14 +776,19 @@ extern "C" fk_status fk_segment_scores_noalloc(const void* K, int n_frames, int 
   a.k_frame = 0;
   a.kmax = 1;
   a.sums = reinterpret_cast<unsigned long long*>(sc);
-  a.status = reinterpret_cast<int*>(sc + kNoAllocCtrOff) + 3;
+  a.status = status ? status : reinterpret_cast<int*>(sc + kNoAllocCtrOff) + 3;
   a.scores = scores;
   a.kept = reinterpret_cast<int*>(sc + kNoAllocTargetOff + 32);   // unused: no selection
-  a.run[0] = {0, n_frames};
+  a.run[0] = {0, n_frames, 0};
   a.t_lo[0] = 0;
   a.n_scoreable[0] = 0;
   a.n_keep[0] = 0;
-  launch_score(a, s);
-  launch_select(a, 1, s);
+  // plain launches (no programmatic dependent launch): each kernel starts after the one
+  // before it has completed, so the scoring kernel reads the tables the setup kernel wrote
+  const unsigned grid = (unsigned)std::min<long long>(a.total_units, a.max_ctas);
+  const size_t smem = score_smem_bytes(head_dim, a.max_run);
+  if (head_dim == 128) score_kernel<128><<<grid, kScoreThreads, smem, s>>>(a);
+  else score_kernel<64><<<grid, kScoreThreads, smem, s>>>(a);
+  select_kernel<<<1, kSelectThreads, select_smem_bytes(a.max_run, a.n_seg), s>>>(a);
   return cudaGetLastError() == cudaSuccess ? FK_OK : FK_ERR_CUDA;
 }

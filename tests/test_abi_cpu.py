@@ -53,7 +53,7 @@ def test_config_struct_layout():
 
 
 def test_abi_version(lib):
-    assert lib.fk_abi_version() == 3
+    assert lib.fk_abi_version() == 4
 
 
 @pytest.mark.parametrize("bad", [
@@ -88,7 +88,7 @@ def test_null_config_and_status_strings(lib):
     assert lib.fk_validate_config(None) == 2
     for s in range(9):
         assert lib.fk_status_str(s)
-    assert lib.fk_abi_version() == 3
+    assert lib.fk_abi_version() == 4
 
 
 @pytest.mark.skipif(os.path.exists("/dev/nvidia0"), reason="checks the no-GPU error path")
@@ -181,3 +181,20 @@ def test_kernel_kinds_match_header():
     for name, v in KERNEL_KINDS.items():
         assert re.search(r"FK_KERNEL_%s = %d\b" % (name.upper(), v), text), name
     assert "FK_KERNEL_KINDS = %d" % len(KERNEL_KINDS) in text
+
+
+def test_noalloc_rejects_bad_arguments_on_the_host(lib):
+    # sizes beyond the documented limits and null / misaligned pointers are rejected before any
+    # CUDA call (the pointer values below are never dereferenced)
+    f = lib.fk_segment_scores_noalloc
+    K, S = 1 << 20, 2 << 20
+    assert f(None, 4, 64, 128, 8, S, None, None) == 2
+    assert f(K, 4, 64, 128, 8, None, None, None) == 2
+    assert f(K + 8, 4, 64, 128, 8, S, None, None) == 2            # K not 16-byte aligned
+    assert f(K, 4, 64, 128, 8, S, K + 2, None) == 2               # status not 4-byte aligned
+    assert f(K, 4, 64, 96, 8, S, None, None) == 1                 # head_dim
+    assert f(K, 4, 64, 128, 33, S, None, None) == 1               # segments
+    assert f(K, 257, 64, 128, 8, S, None, None) == 1              # frames
+    assert f(K, 1, 64, 128, 8, S, None, None) == 1
+    assert f(K, 256, 64, 128, 32, S, None, None) == 1             # frames x segments
+    assert f(K, 4, 60, 128, 8, S, None, None) == 1                # segments must divide F
