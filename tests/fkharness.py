@@ -73,8 +73,10 @@ def compare_layer(cache, orc, layer, Q_bits, O_dev, rows=None, heads=None, check
     return stats
 
 
-def run_snapshot(w: W.Workload, rows=None, check_scores=True, inputs=None, head_map=None, **cache_over):
-    """Load a snapshot workload into the library and the oracle, compress, attend, compare."""
+def run_snapshot(w: W.Workload, rows=None, check_scores=True, inputs=None, head_map=None,
+                 full_heads=None, **cache_over):
+    """Load a snapshot workload into the library and the oracle, compress, attend, compare
+    (`rows` of every head, then every row of the heads in `full_heads`)."""
     import torch
     from paper_2605_09681_gb300 import ForcingKVCache
     hk, hv, ck, cv, q = inputs if inputs is not None else snapshot(w)
@@ -89,7 +91,13 @@ def run_snapshot(w: W.Workload, rows=None, check_scores=True, inputs=None, head_
         orc = O.ForcingKVOracle.from_workload(w, hm)
         orc.append_frames(0, hk, hv)
         orc.set_current(0, ck, cv)
-        return compare_layer(cache, orc, 0, q, Od, rows=rows, check_scores=check_scores, label=w.name)
+        st = compare_layer(cache, orc, 0, q, Od, rows=rows, check_scores=check_scores, label=w.name)
+        if full_heads:
+            full = compare_layer(cache, orc, 0, q, Od, heads=list(full_heads), check_scores=False,
+                                 label=w.name + " every row")
+            st["full_heads"] = list(full_heads)
+            st["full_max_abs"], st["full_mean_abs"] = full["max_abs"], full["mean_abs"]
+        return st
 
 
 def run_stream(w, track_layers=(0,), compare_every=1, step_filter=None, layer_data=None):

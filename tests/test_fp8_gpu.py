@@ -127,7 +127,7 @@ def _layer_fp8_vs_both(w, n_rows):
     from paper_2605_09681_gb300 import ForcingKVCache
     hk, hv, ck, cv, q = snapshot(w.with_(attn_precision="bf16"))
     hm = W.head_map(w)
-    rows = sample_rows(w.n_queries, n_rows)
+    rows = np.arange(w.n_queries) if n_rows is None else sample_rows(w.n_queries, n_rows)
     with ForcingKVCache.from_workload(w, hm) as cache:
         cache.append_frames(0, to_dev(hk), to_dev(hv))
         cache.set_current(0, to_dev(ck), to_dev(cv))
@@ -149,7 +149,8 @@ def _layer_fp8_vs_both(w, n_rows):
 
 
 def test_fp8_480p_layer():
-    print("fp8 480p", _layer_fp8_vs_both(W.P480_LAYER_FP8, 96))
+    # every query row of every head
+    print("fp8 480p", _layer_fp8_vs_both(W.P480_LAYER_FP8, None))
 
 
 def test_fp8_1080p_layer():

@@ -194,17 +194,49 @@ def test_range_precondition_reported():
         assert c.sync_status() == 0                     # the status word is cleared
 
 
-# ------------------------------------------------------------------ full-size workloads (sampled rows)
+# ------------------------------------------------------------------ full-size workloads
 def test_480p_layer():
-    w = W.P480_LAYER
-    st = run_snapshot(w, rows=sample_rows(w.n_queries, 96))
+    # every query row of every head: all 19 query-tile pairs of each of the 12 heads
+    st = run_snapshot(W.P480_LAYER)
     print("480p", st)
 
 
 def test_1080p_layer():
+    # sampled rows of every head, then every row of the first static and the first dynamic head
+    # (all 96 query-tile pairs of each)
     w = W.P1080_LAYER
-    st = run_snapshot(w, rows=sample_rows(w.n_queries, 64))
+    hm = W.head_map(w)[0]
+    full = [int(np.flatnonzero(hm == 1)[0]), int(np.flatnonzero(hm == 0)[0])]
+    st = run_snapshot(w, rows=sample_rows(w.n_queries, 64), full_heads=full)
     print("1080p", st)
+
+
+def test_contract_golden_tokens_on_gpu():
+    # the hand-worked tokens of tests/golden/contract_token_dot.txt through the GPU scorer: one
+    # token per segment, frame 0 = the a rows, frame 1 = the b rows, frame 2 = zeros.  Every
+    # self-dot is 2^21, so s_0^(j) = d_j 2^24 / (2^21 2^24) = d_j 2^-21 (the hand value), and
+    # frame 1 against the zero frame scores 0.
+    from paper_2605_09681_gb300 import ForcingKVCache
+    from test_oracle_pins import _contract_golden
+    toks = _contract_golden()
+    for D in (64, 128):
+        rows = [t for t in toks if t[1] == D]
+        n = len(rows)
+        frames = np.zeros((3, n, 1, D), dtype=np.float32)
+        for j, (_name, _D, a, b, _v) in enumerate(rows):
+            frames[0, j, 0], frames[1, j, 0] = a, b
+        kb = W.to_bf16_bits(frames.reshape(3 * n, 1, D))
+        kd = to_dev(kb)
+        with ForcingKVCache(n_layers=1, n_heads=1, head_dim=D, tokens_per_frame=n, frames_per_chunk=1,
+                            n_sink_frames=0, window_frames=0, n_segments=n, keep_budget_permille=500,
+                            head_is_static=[[0]], max_history_frames=3) as c:
+            c.append_frames(0, kd, kd)
+            c.compress()
+            first, sc = c.scores(0, 0)
+            assert c.sync_status() == 0
+        assert first == 0 and sc.shape == (2, n)
+        want = np.array([[v["contract"] * 2.0 ** -21 for *_x, v in rows], [0.0] * n], dtype=np.float32)
+        assert np.array_equal(sc.view(np.uint32), want.view(np.uint32)), (D, sc, want)
 
 
 def test_rolling_full():
