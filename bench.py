@@ -59,9 +59,8 @@ def _workload(name: str):
     return w.with_(window_frames=window, incremental=False)
 
 
-def _config(w, keys, l2, parallelism):
-    """The workload part of the JSON line's config (shared by both arms) plus the arm's own
-    timing method (l2, parallelism)."""
+def _config(w, keys):
+    """The JSON line's config, identical in both arms: the workload and how each arm times it."""
     return {
         "workload": w.name + " streamed through an %d-frame window" % w.window_frames,
         "heads": w.n_heads, "static_heads": int(sum(_workload_static(w))),
@@ -71,7 +70,10 @@ def _config(w, keys, l2, parallelism):
         "segments": w.n_segments, "keep_budget": w.keep_budget_permille / 1000,
         "keys_per_head": list(keys), "selection": w.selection,
         "rescore": "whole window every step" if w.selection == "similarity" else "no scoring (comparison rule)",
-        "l2": l2, "parallelism": parallelism,
+        "l2": "GPU arm: flushed between timed steps (512 MiB write outside the step events); "
+              "reference arm (CPU oracle): not applicable",
+        "parallelism": "GPU arm: one GPU per rank, independent replicas; reference arm: host cores "
+                       "of rank 0",
     }
 
 
@@ -186,50 +188,52 @@ def barrier(world: int) -> None:
         dist.barrier()
 
 
-def run_fk(args, rank, world, local_rank):
+def _layer_inputs(w, dev, n_pool):
+    """Seeded inputs of a single-layer workload: the history frames, a pool of chunks (K, V)
+    and their queries, on the device and in pinned host memory."""
     import numpy as np
     import torch
 
     import workloads as W
-    from paper_2605_09681_gb300 import ForcingKVCache, build
-
-    build.build()
-    torch.cuda.set_device(local_rank)
-    dev = torch.device("cuda", local_rank)
-    w = _workload(args.workload)
-    hm = W.head_map(w)
     fs = W.FrameStream(w, 0)
     hk, hv = fs.frames(w.n_history_frames)
-    n_pool = 4
     chunks = [fs.frames(w.frames_per_chunk) for _ in range(n_pool)]
     qs = [W.queries(w, 0, c, 0) for c in range(n_pool)]
     to_t = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16)
-    dK = [to_t(k).to(dev) for k, _ in chunks]
-    dV = [to_t(v).to(dev) for _, v in chunks]
-    dQ = [to_t(q).to(dev) for q in qs]
-    dO = torch.empty_like(dQ[0])
-    hK = [to_t(k).pin_memory() for k, _ in chunks]
-    hV = [to_t(v).pin_memory() for _, v in chunks]
-    hQ = [to_t(q).pin_memory() for q in qs]
-    hO = torch.empty(dQ[0].shape, dtype=torch.bfloat16).pin_memory()
-    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
-    stream = torch.cuda.current_stream(dev)
+    d = {"hk": to_t(hk).to(dev), "hv": to_t(hv).to(dev),
+         "dK": [to_t(k).to(dev) for k, _ in chunks], "dV": [to_t(v).to(dev) for _, v in chunks],
+         "dQ": [to_t(q).to(dev) for q in qs],
+         "hK": [to_t(k).pin_memory() for k, _ in chunks], "hV": [to_t(v).pin_memory() for _, v in chunks],
+         "hQ": [to_t(q).pin_memory() for q in qs]}
+    d["dO"] = torch.empty_like(d["dQ"][0])
+    d["hO"] = torch.empty(d["dQ"][0].shape, dtype=torch.bfloat16).pin_memory()
+    return d
 
+
+def measure_layer(args, w, hm, inp, flush, stream, world, local_rank, peaks):
+    """One single-layer workload streamed through its window: device-timed steps (L2 flushed
+    before each), per-kernel event times, and the end-to-end time through the C ABI with pinned
+    host inputs and outputs.  Returns the measurements and the cache's key counts."""
+    import torch
+
+    from paper_2605_09681_gb300 import ForcingKVCache
+
+    n_pool = len(inp["dK"])
     cache = ForcingKVCache.from_workload(w, hm, device=local_rank)
-    cache.append_frames(0, to_t(hk).to(dev), to_t(hv).to(dev))
-    cache.set_current(0, dK[0], dV[0])
+    cache.append_frames(0, inp["hk"], inp["hv"])
+    cache.set_current(0, inp["dK"][0], inp["dV"][0])
     cache.compress()
 
     def step(i, host=False):
         j = i % n_pool
         if host:
-            cache.append_chunk(0, hK[j], hV[j])
+            cache.append_chunk(0, inp["hK"][j], inp["hV"][j])
             cache.compress()
-            cache.attend(0, hQ[j], hO)
+            cache.attend(0, inp["hQ"][j], inp["hO"])
         else:
-            cache.append_chunk(0, dK[j], dV[j])
+            cache.append_chunk(0, inp["dK"][j], inp["dV"][j])
             cache.compress()
-            cache.attend(0, dQ[j], dO)
+            cache.attend(0, inp["dQ"][j], inp["dO"])
 
     def timed(n, host):
         evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
@@ -250,7 +254,7 @@ def run_fk(args, rank, world, local_rank):
     torch.cuda.synchronize()
     st = cache.sync_status()
     if st != 0:
-        raise SystemExit("device status %d during warm-up" % st)
+        raise SystemExit("device status %d during warm-up (%s)" % (st, w.name))
     keys = [cache.key_count(0, h) for h in range(w.n_heads)]
     alg = _algorithmic(w, keys)
 
@@ -267,12 +271,12 @@ def run_fk(args, rank, world, local_rank):
     cache.profile_enable(False)
     st = cache.sync_status()
     if st != 0:
-        raise SystemExit("device status %d during the timed region" % st)
+        raise SystemExit("device status %d during the timed region (%s)" % (st, w.name))
     total_ms = reduce_max(total_ms, world)
 
     # end to end: pinned host inputs copied (on the handle's copy stream, overlapping the work
     # already queued) and the output copied back every step; one continuous timed interval over
-    # all steps (the step's working set, ~0.3 GB of views and pages, exceeds the L2)
+    # all steps (the step's working set of views and pages exceeds the L2)
     cache.set_host_overlap(True)
     for i in range(min(args.warmup, 3)):
         step(i, host=True)
@@ -288,12 +292,8 @@ def run_fk(args, rank, world, local_rank):
     barrier(world)
     e2e_ms = reduce_max(e_begin.elapsed_time(e_end), world)
     if cache.sync_status() != 0:
-        raise SystemExit("device status error during the end-to-end region")
-
-    peaks = _peaks()
-    ms_step = total_ms / args.steps
-    value = world * alg["attn_flops"] * args.steps / (total_ms * 1e-3) / 1e12
-    e2e_value = world * alg["attn_flops"] * args.steps / (e2e_ms * 1e-3) / 1e12
+        raise SystemExit("device status error during the end-to-end region (%s)" % w.name)
+    cache.close()
 
     def per_launch(kind):
         ms, n = prof[kind]
@@ -304,41 +304,30 @@ def run_fk(args, rank, world, local_rank):
     compact_ms, score_ms = per_launch("compact"), per_launch("score")
     compact_gbs = alg["compact_bytes"] / (compact_ms * 1e-3) / 1e9
     score_gbs = alg["score_bytes"] / (score_ms * 1e-3) / 1e9 if prof["score"][1] else None
-    append_ms = prof["append"][0] / max(1, prof["append"][1])
     append_total = prof["append"][0] / args.steps
     compress_ms = (prof["score"][0] + prof["select"][0] + prof["compact"][0]) / args.steps
     attn_fps = w.frames_per_chunk / (DIT_LAYERS * (DENOISE_STEPS * attn_ms + append_total + compress_ms) * 1e-3)
-    traffic = _traffic(args.workload)
-    nbytes = dQ[0].numel() * 2
-    out = {
-        "metric": METRIC,
-        "value": round(value, 3),
-        "unit": "TFLOP/s",
-        "n_gpus": world,
-        "steps": args.steps,
-        "warmup": args.warmup,
-        "ms_per_step": round(ms_step, 4),
-        "higher_is_better": True,
-        "scaling": "weak",
-        "vs_baseline": None,
-        "dtype": "bf16",
-        "data": "synthetic (seeded AR(1) bf16 K/V, iid Q; no model weights)",
-        "config": _config(w, keys, l2="flushed between timed steps (512 MiB write outside the step events)",
-                          parallelism="replicas" if world > 1 else "single GPU"),
-        "gpu_launches": int(launches),
-        "e2e": {"value": round(e2e_value, 3), "unit": "TFLOP/s", "ms_per_step": round(e2e_ms / args.steps, 4),
+    traffic = _traffic(w.name)
+    nbytes = inp["dQ"][0].numel() * 2
+    return {
+        "keys": keys, "alg": alg, "prof": prof, "launches": int(launches),
+        "ms_step": total_ms / args.steps,
+        "value": world * alg["attn_flops"] * args.steps / (total_ms * 1e-3) / 1e12,
+        "e2e": {"value": round(world * alg["attn_flops"] * args.steps / (e2e_ms * 1e-3) / 1e12, 3),
+                "unit": "TFLOP/s", "ms_per_step": round(e2e_ms / args.steps, 4),
                 "h2d_bytes_per_step": 3 * nbytes, "d2h_bytes_per_step": nbytes,
                 "note": "pinned host K, V, Q in and O out every step through the C ABI; host copies "
                         "overlap queued work (fk_set_host_overlap, outputs joined by fk_wait_outputs "
                         "before the end event); one continuous interval over all steps",
-                "l2": "not flushed between steps (each step touches ~0.4 GB of inputs, views and "
-                      "pages, more than the L2); the device-timed value flushes before every step"},
+                "l2": "not flushed between steps (each step touches more inputs, views and pages than "
+                      "the L2 holds); the device-timed value flushes before every step"},
         "roofline": {
             "bound": "tensor", "kernel": "attention (tcgen05)", "achieved": round(attn_tflops, 2),
             "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
             "frac": round(attn_tflops / peaks["bf16_tflops"], 4),
             "peak_source": peaks["source"] + " bf16 dense burst (cuBLAS)",
             "traffic": traffic.get("attend"),
+            "traffic_source": TRAFFIC_SOURCE if traffic.get("attend") is not None else None,
         },
         "roofline_hbm": {
             "compact": {"achieved": round(compact_gbs, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
@@ -349,19 +338,65 @@ def run_fk(args, rank, world, local_rank):
                        "us": round(score_ms * 1e3, 2), "traffic": traffic.get("score")}
                       if score_gbs is not None else None),
             "peak_source": peaks["source"] + " HBM copy bandwidth",
+            "traffic_source": TRAFFIC_SOURCE if traffic else None,
         },
         "kernels_us_per_step": {k: round(prof[k][0] / args.steps * 1e3, 2) for k in prof},
         "attn_fps_extrapolated": round(attn_fps, 2),
-        "attn_fps_note": "C frames / (30 layers x (4 attends + append + compress)) from one layer",
         "attn_gflop_per_step": round(alg["attn_flops"] / 1e9, 2),
         "clocks": clk.summary(),
     }
-    cache.close()
-    out["incremental"] = run_incremental(args, w, hm, local_rank, to_t(hk).to(dev), to_t(hv).to(dev),
-                                         dK, dV, dQ, dO, flush, stream, world, peaks)
+
+
+def run_fk(args, rank, world, local_rank):
+    import torch
+
+    import workloads as W
+    from paper_2605_09681_gb300 import build
+
+    build.build()
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    peaks = _peaks()
+
+    w = _workload(args.workload)
+    hm = W.head_map(w)
+    inp = _layer_inputs(w, dev, 4)
+    m = measure_layer(args, w, hm, inp, flush, stream, world, local_rank, peaks)
+    out = {
+        "metric": METRIC,
+        "value": round(m["value"], 3),
+        "unit": "TFLOP/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(m["ms_step"], 4),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic (seeded AR(1) bf16 K/V, iid Q; no model weights)",
+        "config": _config(w, m["keys"]),
+        "gpu_launches": m["launches"],
+        "e2e": m["e2e"],
+        "roofline": m["roofline"],
+        "roofline_hbm": m["roofline_hbm"],
+        "kernels_us_per_step": m["kernels_us_per_step"],
+        "attn_fps_extrapolated": m["attn_fps_extrapolated"],
+        "attn_fps_note": "C frames / (30 layers x (4 attends + append + compress)) from one layer",
+        "attn_gflop_per_step": m["attn_gflop_per_step"],
+        "clocks": m["clocks"],
+    }
+    out["incremental"] = run_incremental(args, w, hm, local_rank, inp["hk"], inp["hv"], inp["dK"], inp["dV"],
+                                         inp["dQ"], inp["dO"], flush, stream, world, peaks)
+    prof = m["prof"]
     if w.head_dim == 128:
-        out["fp8_qk"] = run_fp8(args, w, hm, local_rank, to_t(hk).to(dev), to_t(hv).to(dev),
-                                dK, dV, dQ, dO, flush, stream, world, peaks, prof)
+        out["fp8_qk"] = run_fp8(args, w, hm, local_rank, inp["hk"], inp["hv"], inp["dK"], inp["dV"],
+                                inp["dQ"], inp["dO"], flush, stream, world, peaks, prof)
+    del inp
+    if not args.no_1080p and args.workload == "480p_layer":
+        out["p1080"] = run_1080p(args, world, local_rank, flush, stream, peaks)
     out["head_profile_480p"] = run_head_profile(args, local_rank, flush, peaks)
     if not args.no_stack:
         out["stack_480p"] = run_stack(local_rank)
@@ -370,6 +405,37 @@ def run_fk(args, rank, world, local_rank):
         out["cpu_baseline"] = cpu_baseline(w, budget_s=args.cpu_seconds)
         out["cpu_baseline"].pop("keys_per_head", None)
     return out
+
+
+def run_1080p(args, world, local_rank, flush, stream, peaks):
+    """The 1080P single-layer workload (24480 queries, 1 sink + 9 history frames of 8160
+    tokens), measured exactly as the headline 480P layer: device-timed steps with the L2
+    flushed, per-kernel rooflines, end to end through the C ABI, and clocks."""
+    import torch
+
+    import workloads as W
+    w = _workload("1080p_layer")
+    hm = W.head_map(w)
+    inp = _layer_inputs(w, torch.device("cuda", local_rank), 2)   # 75 MB per tensor: above the L2
+    m = measure_layer(args, w, hm, inp, flush, stream, world, local_rank, peaks)
+    del inp
+    return {
+        "workload": _config(w, m["keys"])["workload"],
+        "ms_per_step": round(m["ms_step"], 4),
+        "value": round(m["value"], 3),
+        "unit": "TFLOP/s",
+        "gpu_launches": m["launches"],
+        "keys_per_head": m["keys"],
+        "e2e": m["e2e"],
+        "roofline": m["roofline"],
+        "roofline_hbm": m["roofline_hbm"],
+        "kernels_us_per_step": m["kernels_us_per_step"],
+        "attn_fps_extrapolated": m["attn_fps_extrapolated"],
+        "attn_gflop_per_step": m["attn_gflop_per_step"],
+        "clocks": m["clocks"],
+        "note": "the paper's 1080P scaling case (Sec. 5.2); attention-path frames/s extrapolated as "
+                "for 480P: C frames / (30 layers x (4 attends + append + compress))",
+    }
 
 
 def run_incremental(args, w, hm, local_rank, hk, hv, dK, dV, dQ, dO, flush, stream, world, peaks):
@@ -646,6 +712,11 @@ NCU_TRAFFIC = {
 }
 
 
+TRAFFIC_SOURCE = ("stored DRAM bytes per launch from an earlier ncu capture of the same kernel "
+                  "source (profiles/hbm_kernels_480p_layer.md, profiles/attn_kernel_480p_layer.md); "
+                  "reported only while the source hash matches, not observed in this run")
+
+
 def _traffic(workload):
     import hashlib
     out = {}
@@ -709,19 +780,25 @@ def run_reference(args, rank, world):
     for _ in range(args.warmup):
         cpu_baseline(w, budget_s=budget)
     vals, secs = [], 0.0
+    t0 = time.perf_counter()
     for _ in range(args.steps):
         r = cpu_baseline(w, budget_s=budget)
         vals.append(r["value"])
         secs += r["step_s"]
+    wall = time.perf_counter() - t0
     value = statistics.mean(vals)
     r["value"] = round(value, 6)
     return {
         "metric": METRIC, "value": round(value, 6), "unit": "TFLOP/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(secs / args.steps * 1e3, 1),
+        "extrapolated": True,
+        "measured_ms_per_step": round(wall / args.steps * 1e3, 1),
+        "extrapolation": "each step times the oracle's full compress and attention of a sample of "
+                         "query rows; ms_per_step and value scale the attention to all rows "
+                         "(measured_ms_per_step is the wall time actually spent per step)",
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic (seeded AR(1) bf16 K/V, iid Q; no model weights)",
-        "config": _config(w, r.pop("keys_per_head"), l2="n/a (host CPU)",
-                          parallelism="host cores, rank 0 only"),
+        "config": _config(w, r.pop("keys_per_head")),
         "impl": "reference", "cpu_baseline": r,
         "e2e": {"value": round(value, 6), "unit": "TFLOP/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
@@ -738,6 +815,7 @@ def main(argv=None):
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-stack", action="store_true", help="skip the directly measured 480P stack")
+    ap.add_argument("--no-1080p", action="store_true", help="skip the 1080P single-layer leg")
     args = ap.parse_args(argv)
     if args.warmup < 3:
         ap.error("--warmup must be at least 3")

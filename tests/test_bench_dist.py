@@ -74,6 +74,7 @@ def test_reference_arm_json_contract():
     assert cfg["keys_per_head"] == [7800, 7800, 25480, 25480, 25480, 7800, 7800, 25480, 7800,
                                     25480, 7800, 25480]
     assert cfg["queries"] == 4680 and cfg["head_dim"] == 128 and cfg["heads"] == 12
+    assert line["extrapolated"] is True and line["measured_ms_per_step"] > 0
 
 
 def test_algorithmic_work_of_the_480p_step():
@@ -87,5 +88,15 @@ def test_algorithmic_work_of_the_480p_step():
     assert alg["attn_flops"] == 4 * 4680 * 128 * (6 * 7800 + 6 * 25480)            # 478.47 GFLOP
     assert alg["score_bytes"] == 6 * 18 * 1560 * 128 * 2                           # 43.13 MB
     assert alg["compact_bytes"] == 6 * (1560 + 17 * 4 * 260 + 1560) * 128 * 2 * 2 * 2  # 127.8 MB
-    cfg = bench._config(w, keys, l2="x", parallelism="y")
+    cfg = bench._config(w, keys)
     assert cfg["queries"] == 4680 and cfg["history_frames"] == 18 and cfg["keys_per_head"] == keys
+
+
+def test_both_arms_print_the_same_config():
+    # the reference arm's config is built by the same function from the same workload and key
+    # counts, and carries no arm-specific field
+    import bench
+    import workloads as W
+    w = bench._workload("480p_layer")
+    keys = [7800 if s else 25480 for s in W.head_map(w)[0]]
+    assert bench._config(w, keys) == bench._config(bench._workload("480p_layer"), list(keys))
