@@ -259,30 +259,6 @@ __device__ __forceinline__ float2 fadd2(float2 a, float2 b) {
   return d;
 }
 
-// 2^x on the FMA pipe for a pair: range reduction x = n + f, n = round(x) (by adding and
-// subtracting 1.5 * 2^23), f in [-1/2, 1/2]; 2^f by a degree-3 polynomial fitted for
-// minimum relative error (7.5e-5; exp2_poly_fit.py); 2^n added to the exponent field.
-// x is clamped at -126 (results below 2^-126 are flushed to that magnitude; they are
-// far below the bf16 resolution of P relative to the row maximum 1).
-#ifndef FK_POLY_EVERY
-#define FK_POLY_EVERY 0
-#endif
-constexpr int kPolyEvery = FK_POLY_EVERY;          // one pair in kPolyEvery uses the polynomial
-__device__ __forceinline__ float2 exp2_poly2(float2 x) {
-  x.x = fmaxf(x.x, -126.0f);
-  x.y = fmaxf(x.y, -126.0f);
-  const float2 magic = make_float2(12582912.0f, 12582912.0f);
-  const float2 t = fadd2(x, magic);
-  const float2 n = fadd2(t, make_float2(-12582912.0f, -12582912.0f));
-  const float2 f = fadd2(x, make_float2(-n.x, -n.y));
-  float2 p = ffma2(make_float2(5.517166493e-02f, 5.517166493e-02f), f,
-                   make_float2(2.426111219e-01f, 2.426111219e-01f));
-  p = ffma2(p, f, make_float2(6.932609862e-01f, 6.932609862e-01f));
-  p = ffma2(p, f, make_float2(9.999280736e-01f, 9.999280736e-01f));
-  return make_float2(__int_as_float(__float_as_int(p.x) + (__float_as_int(t.x) << 23)),
-                     __int_as_float(__float_as_int(p.y) + (__float_as_int(t.y) << 23)));
-}
-
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   const __nv_bfloat162 p = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<const uint32_t*>(&p);
@@ -574,12 +550,8 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
             const float2 x = ffma2(make_float2(__uint_as_float(sv[2 * q]), __uint_as_float(sv[2 * q + 1])),
                                    sc2, nm2);
             float2 e;
-            if (kPolyEvery > 0 && q % (kPolyEvery > 0 ? kPolyEvery : 1) == kPolyEvery - 1) {
-              e = exp2_poly2(x);                     // FMA pipe
-            } else {
-              e.x = fast_exp2(x.x);                  // MUFU
-              e.y = fast_exp2(x.y);
-            }
+            e.x = fast_exp2(x.x);                    // MUFU
+            e.y = fast_exp2(x.y);
             acc[q & 3] = fadd2(acc[q & 3], e);
             pk[q] = pack_bf16(e.x, e.y);
           }
