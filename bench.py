@@ -78,11 +78,14 @@ def _config(w, keys):
 
 
 def _algorithmic(w, key_counts):
-    """Per-step algorithmic work: attention FLOPs sum_h 4*Nq*Nk_h*D; scoring bytes = keys of the
-    scored frames of every dynamic head; compaction bytes = keys and values of every dynamic
-    head's view units, read and written; append bytes = the chunk's K/V read and written plus
-    the retired frames copied into the history."""
-    D, F, H = w.head_dim, w.tokens_per_frame, w.n_heads
+    """Per-step algorithmic work of a step that streams one chunk through a full window:
+    attention FLOPs sum_h 4*Nq*Nk_h*D; scoring-kernel bytes = the keys it reads, i.e. the window
+    frames up to the frame before the retired chunk of every dynamic head (the current-chunk
+    kernel forms the sums of the retired frames, whose keys it moves anyway); compaction bytes =
+    keys and values of every dynamic head's view units, read and written; append bytes = the
+    chunk's K/V read and written, the retired frames copied into the history, and the key frame
+    before the retired chunk that the in-kernel scoring reads as the first frame's partner."""
+    D, F, H, C = w.head_dim, w.tokens_per_frame, w.n_heads, w.frames_per_chunk
     nq = w.n_queries
     flops = sum(4.0 * nq * nk * D for nk in key_counts)
     nh, S, Wn = w.n_history_frames, w.n_sink_frames, w.window_frames
@@ -93,15 +96,19 @@ def _algorithmic(w, key_counts):
     static = _workload_static(w)
     n_dyn = sum(1 for st in static if not st)
     scored = w.selection == "similarity"                 # comparison rules skip scoring
-    score_bytes = n_dyn * (n_scoreable + 1 if n_scoreable else 0) * F * D * 2 if scored else 0
+    # the current-chunk kernel scores the retired chunk when the frame before it stays a
+    # non-sink window frame (the chunk has at most 15 frames)
+    fused = scored and C <= 15 and nh - C - 1 >= max(S, lo)
+    read_frames = (n_scoreable + 1 - C) if fused else (n_scoreable + 1 if n_scoreable else 0)
+    score_bytes = n_dyn * read_frames * F * D * 2 if scored else 0
     k_frame = w.n_segments if w.selection == "all" else w.keep_budget_permille * w.n_segments // 1000
     n_keep = n_scoreable * k_frame
     unit_tokens = n_sink * F + n_keep * (F // w.n_segments) + (F if has_anchor else 0)
     compact_bytes = n_dyn * 2 * 2 * unit_tokens * D * 2
     append_bytes = 2 * 2 * nq * H * D * 2 + sum(
-        2 * 2 * (F if st else w.frames_per_chunk * F) * D * 2 for st in static)
+        2 * 2 * (F if st else C * F) * D * 2 for st in static) + (n_dyn * F * D * 2 if fused else 0)
     return dict(attn_flops=flops, score_bytes=score_bytes, compact_bytes=compact_bytes,
-                append_bytes=append_bytes)
+                append_bytes=append_bytes, score_fused=fused)
 
 
 def _workload_static(w):
@@ -210,7 +217,27 @@ def _layer_inputs(w, dev, n_pool):
     return d
 
 
-def measure_layer(args, w, hm, inp, flush, stream, world, local_rank, peaks):
+def _read_floor(args, nbytes, calib, flush, stream):
+    """Mean event-timed duration (us) of fk_stream_read over `nbytes` after the L2 flush."""
+    import torch
+
+    from paper_2605_09681_gb300 import stream_read
+    if not nbytes or calib is None:
+        return None
+    nbytes = min(int(nbytes) // 16 * 16, calib.numel())
+    reps = max(3, min(args.steps, 50))
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(reps)]
+    torch.cuda.synchronize()
+    for i in range(reps):
+        flush.zero_()
+        evs[i][0].record(stream)
+        stream_read(calib, nbytes)
+        evs[i][1].record(stream)
+    torch.cuda.synchronize()
+    return sum(a.elapsed_time(b) for a, b in evs) / reps * 1e3
+
+
+def measure_layer(args, w, hm, inp, flush, stream, world, local_rank, peaks, calib=None):
     """One single-layer workload streamed through its window: device-timed steps (L2 flushed
     before each), per-kernel event times, and the end-to-end time through the C ABI with pinned
     host inputs and outputs.  Returns the measurements and the cache's key counts."""
@@ -273,6 +300,7 @@ def measure_layer(args, w, hm, inp, flush, stream, world, local_rank, peaks):
     if st != 0:
         raise SystemExit("device status %d during the timed region (%s)" % (st, w.name))
     total_ms = reduce_max(total_ms, world)
+    floor = _read_floor(args, alg["score_bytes"], calib, flush, stream)
 
     # end to end: pinned host inputs copied (on the handle's copy stream, overlapping the work
     # already queued) and the output copied back every step; one continuous timed interval over
@@ -335,10 +363,20 @@ def measure_layer(args, w, hm, inp, flush, stream, world, local_rank, peaks):
                         "us": round(compact_ms * 1e3, 2), "traffic": traffic.get("compact")},
             "score": ({"achieved": round(score_gbs, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
                        "frac": round(score_gbs / peaks["hbm_gbs"], 4), "bytes": alg["score_bytes"],
-                       "us": round(score_ms * 1e3, 2), "traffic": traffic.get("score")}
+                       "us": round(score_ms * 1e3, 2), "traffic": traffic.get("score"),
+                       "read_floor_us": round(floor, 2) if floor else None,
+                       "frac_of_read_floor": round(floor / (score_ms * 1e3), 4) if floor else None}
                       if score_gbs is not None else None),
+            "append": {"achieved": round(alg["append_bytes"] / (per_launch("append") * 1e-3) / 1e9, 1),
+                       "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                       "frac": round(alg["append_bytes"] / (per_launch("append") * 1e-3) / 1e9 / peaks["hbm_gbs"], 4),
+                       "bytes": alg["append_bytes"], "us": round(per_launch("append") * 1e3, 2),
+                       "scores_retired_chunk": alg["score_fused"]},
             "peak_source": peaks["source"] + " HBM copy bandwidth",
             "traffic_source": TRAFFIC_SOURCE if traffic else None,
+            "read_floor_note": "read_floor_us: event-timed fk_stream_read of the scoring kernel's bytes "
+                               "after the same L2 flush (a plain streaming read: the floor for any "
+                               "launch that reads those bytes); frac_of_read_floor = floor / kernel time",
         },
         "kernels_us_per_step": {k: round(prof[k][0] / args.steps * 1e3, 2) for k in prof},
         "attn_fps_extrapolated": round(attn_fps, 2),
@@ -359,11 +397,12 @@ def run_fk(args, rank, world, local_rank):
     flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream(dev)
     peaks = _peaks()
+    calib = torch.ones(256 << 20, dtype=torch.uint8, device=dev)   # read-floor calibration data
 
     w = _workload(args.workload)
     hm = W.head_map(w)
     inp = _layer_inputs(w, dev, 4)
-    m = measure_layer(args, w, hm, inp, flush, stream, world, local_rank, peaks)
+    m = measure_layer(args, w, hm, inp, flush, stream, world, local_rank, peaks, calib)
     out = {
         "metric": METRIC,
         "value": round(m["value"], 3),
@@ -396,7 +435,7 @@ def run_fk(args, rank, world, local_rank):
                                 inp["dQ"], inp["dO"], flush, stream, world, peaks, prof)
     del inp
     if not args.no_1080p and args.workload == "480p_layer":
-        out["p1080"] = run_1080p(args, world, local_rank, flush, stream, peaks)
+        out["p1080"] = run_1080p(args, world, local_rank, flush, stream, peaks, calib)
     out["head_profile_480p"] = run_head_profile(args, local_rank, flush, peaks)
     if not args.no_stack:
         out["stack_480p"] = run_stack(local_rank)
@@ -407,7 +446,7 @@ def run_fk(args, rank, world, local_rank):
     return out
 
 
-def run_1080p(args, world, local_rank, flush, stream, peaks):
+def run_1080p(args, world, local_rank, flush, stream, peaks, calib=None):
     """The 1080P single-layer workload (24480 queries, 1 sink + 9 history frames of 8160
     tokens), measured exactly as the headline 480P layer: device-timed steps with the L2
     flushed, per-kernel rooflines, end to end through the C ABI, and clocks."""
@@ -417,7 +456,7 @@ def run_1080p(args, world, local_rank, flush, stream, peaks):
     w = _workload("1080p_layer")
     hm = W.head_map(w)
     inp = _layer_inputs(w, torch.device("cuda", local_rank), 2)   # 75 MB per tensor: above the L2
-    m = measure_layer(args, w, hm, inp, flush, stream, world, local_rank, peaks)
+    m = measure_layer(args, w, hm, inp, flush, stream, world, local_rank, peaks, calib)
     del inp
     return {
         "workload": _config(w, m["keys"])["workload"],
@@ -509,9 +548,12 @@ def run_incremental(args, w, hm, local_rank, hk, hv, dK, dV, dQ, dO, flush, stre
         "keys_per_head": keys,
         "kernels_us_per_step": {k: round(prof[k][0] / args.steps * 1e3, 2) for k in prof},
         "score": kern("score", score_bytes),
+        "append": kern("append", alg["append_bytes"]),
         "compact": kern("compact", compact_bytes),
-        "note": "per step: scoring reads C + 1 frames per dynamic head, compaction copies C x k "
-                "segments + the anchor frame per dynamic head (ring-buffer views)",
+        "note": "per step: the current-chunk kernel forms the scoring sums of the C retired frames "
+                "(and the squared norms of the frame before them) while moving them, so no scoring "
+                "launch runs (score is null); compaction copies C x k segments + the anchor frame per "
+                "dynamic head (ring-buffer views)",
     }
 
 

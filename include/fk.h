@@ -259,6 +259,15 @@ FK_API fk_status fk_wait_outputs(fk_handle* h, void* stream);
  * `stream`.  FK_ERR_ARG for a null handle or a limit out of range. */
 FK_API fk_status fk_wait_selftest(fk_handle* h, int limit_us, void* stream);
 
+/* HBM calibration (no counterpart in the paper): reads `bytes` of device memory once with
+ * 16-byte streaming loads from a grid of 8 CTAs per SM and does nothing else.  Timed with CUDA
+ * events like the hot-path kernels, its duration is the practical floor for any single launch
+ * that must read that many bytes (it includes the launch and the first accesses' latency),
+ * which the benchmark reports beside the HBM-bound kernels' fractions of the copy bandwidth.
+ * src: device memory, 16-byte aligned; bytes: a multiple of 16 (0: no launch).  FK_ERR_ARG for
+ * null, misaligned or host pointers.  Asynchronous on `stream`; allocates nothing. */
+FK_API fk_status fk_stream_read(const void* src, size_t bytes, void* stream);
+
 /* Kernels launched by this handle since creation (all kinds). */
 FK_API int64_t fk_launch_count(const fk_handle* h);
 

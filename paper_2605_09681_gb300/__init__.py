@@ -14,7 +14,7 @@ from . import _lib as L
 from ._lib import FkError, KERNEL_KINDS, STATUS_NAMES
 
 __all__ = ["ForcingKVCache", "FkError", "KERNEL_KINDS", "STATUS_NAMES", "load_library",
-           "head_profile", "classify_heads", "quantize_e4m3"]
+           "head_profile", "classify_heads", "quantize_e4m3", "stream_read"]
 
 
 def load_library():
@@ -95,6 +95,17 @@ def quantize_e4m3(X, row_scaled: bool, q8=None, exps=None, stream=None):
                                 exps.data_ptr() if exps is not None else None, _stream(stream)),
            "fk_quantize_e4m3")
     return q8, exps
+
+
+def stream_read(X, nbytes: int | None = None, stream=None) -> None:
+    """Read the first `nbytes` (default: all) of a CUDA tensor once (fk_stream_read): the
+    event-timed floor of a launch that must read that many bytes."""
+    if not X.is_contiguous():
+        raise ValueError("expected a contiguous tensor")
+    n = X.numel() * X.element_size() if nbytes is None else int(nbytes)
+    if n > X.numel() * X.element_size():
+        raise ValueError("nbytes exceeds the tensor")
+    _check(L.load().fk_stream_read(X.data_ptr(), n, _stream(stream)), "fk_stream_read")
 
 
 def classify_heads(mass, alpha: float = 0.8) -> np.ndarray:

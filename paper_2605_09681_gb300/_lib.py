@@ -25,7 +25,7 @@ EXPORTS = [
     "fk_key_count", "fk_get_kept", "fk_get_scores", "fk_sync_status", "fk_profile_enable",
     "fk_profile_read", "fk_profile_reset", "fk_launch_count", "fk_status_str", "fk_abi_version",
     "fk_segment_scores_noalloc", "fk_head_profile", "fk_classify_heads", "fk_set_host_overlap",
-    "fk_wait_selftest", "fk_wait_outputs", "fk_quantize_e4m3",
+    "fk_wait_selftest", "fk_wait_outputs", "fk_quantize_e4m3", "fk_stream_read",
 ]
 
 
@@ -94,6 +94,7 @@ def load(path: str | None = None) -> ctypes.CDLL:
         "fk_classify_heads": (st, [ctypes.POINTER(ctypes.c_double), i32, i32,
                                    ctypes.POINTER(ctypes.c_uint8)]),
         "fk_quantize_e4m3": (st, [vp, ctypes.c_int64, i32, i32, vp, vp, vp]),
+        "fk_stream_read": (st, [vp, ctypes.c_size_t, vp]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)

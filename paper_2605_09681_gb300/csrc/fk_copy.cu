@@ -41,57 +41,152 @@ __device__ __forceinline__ int ring_slot(int f, int S, int cap) {
 __device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
-// One thread per 16-byte granule of the current chunk, indexed in the caller's token-major
-// order (row, head, granule) so that the reads of the new chunk are fully coalesced.
-__global__ void __launch_bounds__(256) current_kernel(const CurrentArgs a) {
-  pdl_trigger();   // the scoring kernel that follows may start its prologue; it waits for us
-  const int gpr = a.head_dim / 8;
-  const uint32_t per_row = (uint32_t)(a.heads * gpr);
-  const uint32_t total = (uint32_t)a.rows * per_row;   // < 2^31 (checked at configuration)
-  const int nh_new = a.nh_old + a.rows / a.F;
+// Current-chunk update.  A CTA owns TB = 256 / GPR consecutive tokens p of one head h (GPR =
+// D/8 16-byte granules per token row) across all C frames of the chunk: thread (p, c) moves
+// granule c of rows r*F + p, r < C, of the new chunk (token-major [C*F][H][D], 256 contiguous
+// bytes per token and head) into the view front, after copying the previous current chunk's
+// granule to its history location.  Frames go in batches of two with every load of a batch
+// issued before its first store.
+//
+// With a.score set, the CTA also forms the score-contract sums of the retired frames (Eq. 3):
+// the GPR lanes of a token hold its GPR channel groups in group order, so the contract's
+// per-group fma chains run in each lane and its butterfly p[g] += p[g ^ s], s = GPR/2 .. 1, is a
+// lane xor-shuffle; the partner of the first retired frame is the frame before the chunk, read
+// from the page ring.  Per (frame, segment) the tokens' int32 halves are summed in shared memory
+// and added to the run's int64 sums once per CTA (exact integer adds, order-free).
+constexpr int kBatch = 2;
+template <int GPR>
+__global__ void __launch_bounds__(256, 4) current_kernel(const CurrentArgs a) {
+  pdl_trigger();   // the kernel that follows may start its prologue; it waits for this one
+  constexpr int TB = 256 / GPR;
+  constexpr int D = GPR * 8;
+  __shared__ int acc[(kFuseMaxFrames + 1) * TB * 4];   // [frame][segment][N hi, N lo, D hi, D lo]
+  const int h = blockIdx.y;
+  const int p0 = blockIdx.x * TB;
+  const int p = p0 + threadIdx.x / GPR;
+  const int c = threadIdx.x % GPR;
+  const bool valid = p < a.F;
+  const int C = a.rows / a.F;
+  const int nh_new = a.nh_old + C;
   const int lo_new = a.W > 0 ? max(a.S, nh_new - a.W) : a.S;
-  for (uint32_t g = blockIdx.x * blockDim.x + threadIdx.x; g < total; g += gridDim.x * blockDim.x) {
-    const int row = (int)(g / per_row);
-    const int rem = (int)(g - row * per_row);
-    const int h = rem / gpr;
-    const int c = rem - h * gpr;
-    const int64_t vo = (int64_t)row * a.head_dim + c * 8;
-    bool to_page = false, to_slot = false;
-    int64_t po = 0, so = 0;
-    if (a.retire) {
-      const int f = a.nh_old + row / a.F;
-      const int p = row - (row / a.F) * a.F;
-      const bool sink = f < a.S;
-      // frames replaced within the retire are skipped; static views hold the sinks and
-      // (unless they drop it) the new anchor frame
-      to_page = a.pageK[h] != nullptr && (sink || f >= lo_new);
-      to_slot = a.is_static[h] && (sink || (a.static_anchor && f == nh_new - 1));
-      po = ((int64_t)ring_slot(f, a.S, a.cap_nonsink) * a.F + p) * a.head_dim + c * 8;
-      so = ((int64_t)a.rows + (int64_t)(sink ? f : a.S) * a.F + p) * a.head_dim + c * 8;
+  const int tgt = a.score ? (int)a.score_target[h] : -1;   // uniform over the CTA
+  const bool scoring = tgt >= 0;
+  const int j0 = p0 / (scoring ? a.seg_len : 1);
+  const int segl = valid && scoring ? p / a.seg_len - j0 : 0;   // local segment of token p
+  bool bad = false;
+  uint4 prev = make_uint4(0, 0, 0, 0);          // the previous frame's granule (contract partner)
+  if (scoring) {
+    for (int i = threadIdx.x; i < (C + 1) * TB * 4; i += 256) acc[i] = 0;
+    if (valid)
+      prev = ld_plain(a.pageK[h] + ((int64_t)ring_slot(a.nh_old - 1, a.S, a.cap_nonsink) * a.F + p) * D + c * 8);
+    __syncthreads();
+    if (a.score_partner_norm) {
+      float n = 0.0f, d = 0.0f;
+      fma_word(prev.x, prev.x, n, d);
+      fma_word(prev.y, prev.y, n, d);
+      fma_word(prev.z, prev.z, n, d);
+      fma_word(prev.w, prev.w, n, d);
+#pragma unroll
+      for (int sft = GPR / 2; sft >= 1; sft >>= 1) n = __fadd_rn(n, __shfl_xor_sync(0xffffffffu, n, sft));
+      if (valid && c == 0) {
+        bad |= !(n <= 8388608.0f);
+        int hi, lo;
+        fixed24_split(n, hi, lo);
+        atomicAdd(&acc[segl * 4 + 0], hi);
+        atomicAdd(&acc[segl * 4 + 1], lo);
+      }
     }
-    // every load first (old granule, new granule), then the stores
-    uint4 ko = make_uint4(0, 0, 0, 0), vo4 = ko, kn = ko, vn = ko;
-    if (to_page || to_slot) {
-      ko = ld_plain(a.viewK[h] + vo);
-      vo4 = ld_plain(a.viewV[h] + vo);
+  }
+  for (int r0 = 0; r0 < C; r0 += kBatch) {
+    uint4 ko[kBatch], vo[kBatch], kn[kBatch], vn[kBatch];
+    // where frame r's old granule goes (page ring, static view slot); frames replaced within
+    // the retire are skipped; static views hold the sinks and (unless they drop it) the anchor
+    auto to_page = [&](int r) {
+      const int f = a.nh_old + r;
+      return a.retire && a.pageK[h] != nullptr && (f < a.S || f >= lo_new);
+    };
+    auto to_slot = [&](int r) {
+      const int f = a.nh_old + r;
+      return a.retire && a.is_static[h] && (f < a.S || (a.static_anchor && f == nh_new - 1));
+    };
+#pragma unroll
+    for (int i = 0; i < kBatch; ++i) {
+      ko[i] = vo[i] = kn[i] = vn[i] = make_uint4(0, 0, 0, 0);
+      const int r = r0 + i;
+      if (r >= C || !valid) continue;
+      const int64_t vof = (int64_t)(r * a.F + p) * D + c * 8;
+      const bool keep_old = to_page(r) || to_slot(r);
+      if (keep_old || scoring) ko[i] = ld_plain(a.viewK[h] + vof);
+      if (keep_old) vo[i] = ld_plain(a.viewV[h] + vof);
+      if (a.srcK) {
+        const size_t src = ((size_t)(r * a.F + p) * a.heads + h) * D + c * 8;
+        kn[i] = ld_stream(a.srcK + src);
+        vn[i] = ld_stream(a.srcV + src);
+      }
     }
-    if (a.srcK) {
-      kn = ld_stream(a.srcK + (size_t)g * 8);
-      vn = ld_stream(a.srcV + (size_t)g * 8);
+#pragma unroll
+    for (int i = 0; i < kBatch; ++i) {
+      const int r = r0 + i;
+      if (r >= C || !valid) continue;
+      const int f = a.nh_old + r;
+      if (to_page(r)) {
+        const int64_t po = ((int64_t)ring_slot(f, a.S, a.cap_nonsink) * a.F + p) * D + c * 8;
+        st_v4(a.pageK[h] + po, ko[i]);
+        st_v4(a.pageV[h] + po, vo[i]);
+      }
+      if (to_slot(r)) {
+        const int64_t so = ((int64_t)a.rows + (int64_t)(f < a.S ? f : a.S) * a.F + p) * D + c * 8;
+        st_v4(a.viewK[h] + so, ko[i]);
+        st_v4(a.viewV[h] + so, vo[i]);
+        if (a.viewK8[h]) *reinterpret_cast<uint2*>(a.viewK8[h] + so) = e4m3x8(ko[i], 1.0f);
+      }
+      if (a.srcK) {
+        const int64_t vof = (int64_t)(r * a.F + p) * D + c * 8;
+        st_v4(a.viewK[h] + vof, kn[i]);
+        st_v4(a.viewV[h] + vof, vn[i]);
+        if (a.viewK8[h]) *reinterpret_cast<uint2*>(a.viewK8[h] + vof) = e4m3x8(kn[i], 1.0f);
+      }
     }
-    if (to_page) {
-      st_v4(a.pageK[h] + po, ko);
-      st_v4(a.pageV[h] + po, vo4);
+    if (scoring) {
+#pragma unroll
+      for (int i = 0; i < kBatch; ++i) {
+        if (r0 + i >= C) break;                 // uniform over the CTA
+        // channel-group partials (one fma chain per lane, channel order), then the butterfly
+        float n = 0.0f, d = 0.0f;
+        fma_word(ko[i].x, prev.x, n, d);
+        fma_word(ko[i].y, prev.y, n, d);
+        fma_word(ko[i].z, prev.z, n, d);
+        fma_word(ko[i].w, prev.w, n, d);
+#pragma unroll
+        for (int sft = GPR / 2; sft >= 1; sft >>= 1) {
+          n = __fadd_rn(n, __shfl_xor_sync(0xffffffffu, n, sft));
+          d = __fadd_rn(d, __shfl_xor_sync(0xffffffffu, d, sft));
+        }
+        prev = ko[i];
+        if (valid && c < 2) {                   // lane 0: N of this frame, lane 1: D with the last
+          const float v = c == 0 ? n : d;
+          if (c == 0) bad |= !(n <= 8388608.0f);
+          int hi, lo;
+          fixed24_split(v, hi, lo);
+          int* slot = &acc[((r0 + i + 1) * TB + segl) * 4 + 2 * c];
+          atomicAdd(slot, hi);
+          atomicAdd(slot + 1, lo);
+        }
+      }
     }
-    if (to_slot) {
-      st_v4(a.viewK[h] + so, ko);
-      st_v4(a.viewV[h] + so, vo4);
-      if (a.viewK8[h]) *reinterpret_cast<uint2*>(a.viewK8[h] + so) = e4m3x8(ko, 1.0f);
-    }
-    if (a.srcK) {
-      st_v4(a.viewK[h] + vo, kn);
-      st_v4(a.viewV[h] + vo, vn);
-      if (a.viewK8[h]) *reinterpret_cast<uint2*>(a.viewK8[h] + vo) = e4m3x8(kn, 1.0f);
+  }
+  if (scoring) {
+    if (bad) atomicOr(a.status, kStatusRange);
+    __syncthreads();
+    const int n_loc = min(TB, (min(p0 + TB, a.F) - 1) / a.seg_len - j0 + 1);   // segments here
+    for (int i = threadIdx.x; i < (C + 1) * n_loc * 2; i += 256) {
+      const int kk = i / (n_loc * 2), rem = i - kk * n_loc * 2;
+      const int sl = rem >> 1, which = rem & 1;
+      const int hi = acc[(kk * TB + sl) * 4 + 2 * which], lo = acc[(kk * TB + sl) * 4 + 2 * which + 1];
+      if (hi == 0 && lo == 0) continue;
+      const long long v = (long long)hi * 16777216ll + (long long)lo;
+      atomicAdd(a.sums + (((int64_t)tgt * a.max_run + a.score_k0 + kk) * a.n_seg + j0 + sl) * 2 + which,
+                (unsigned long long)v);
     }
   }
 }
@@ -222,6 +317,23 @@ __global__ void __launch_bounds__(256) compact_kernel(const CompactArgs a) {
   }
 }
 
+// Streaming read of `n` 16-byte granules (calibration of the HBM-bound kernels): a grid-stride
+// loop with four loads in flight per thread and no other work; the xor of the data decides a
+// store that never happens for the bench's data, so the loads cannot be removed.
+__device__ unsigned g_read_sink;
+__global__ void __launch_bounds__(256) stream_read_kernel(const uint4* __restrict__ src, int64_t n) {
+  uint32_t acc = 0;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  for (; i + 3 * stride < n; i += 4 * stride) {
+    const uint4 v0 = ld_stream(src + i), v1 = ld_stream(src + i + stride);
+    const uint4 v2 = ld_stream(src + i + 2 * stride), v3 = ld_stream(src + i + 3 * stride);
+    acc ^= v0.x ^ v1.y ^ v2.z ^ v3.w;
+  }
+  for (; i < n; i += stride) acc ^= ld_stream(src + i).x;
+  if (acc == 0x5EEDF00Du) atomicAdd(&g_read_sink, 1u);
+}
+
 unsigned grid_for(int64_t granules) {
   int64_t blocks = (granules + 255) / 256;
   if (blocks > 152 * 16) blocks = 152 * 16;
@@ -231,9 +343,11 @@ unsigned grid_for(int64_t granules) {
 }  // namespace
 
 void launch_current(const CurrentArgs& a, cudaStream_t s) {
-  const int64_t total = (int64_t)a.rows * a.heads * (a.head_dim / 8);
-  if (total == 0) return;
-  current_kernel<<<grid_for(total), 256, 0, s>>>(a);
+  if (a.rows == 0 || a.heads == 0) return;
+  const int gpr = a.head_dim / 8, tb = 256 / gpr;
+  const dim3 grid((unsigned)((a.F + tb - 1) / tb), (unsigned)a.heads);
+  if (gpr == 16) current_kernel<16><<<grid, 256, 0, s>>>(a);
+  else current_kernel<8><<<grid, 256, 0, s>>>(a);
 }
 
 void launch_scatter(const ScatterArgs& a, cudaStream_t s) {
@@ -257,6 +371,16 @@ void launch_compact(const CompactArgs& a, cudaStream_t s) {
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   cudaLaunchKernelEx(&cfg, compact_kernel, a);
+}
+
+cudaError_t launch_stream_read(const void* src, int64_t bytes, cudaStream_t s) {
+  if (bytes <= 0) return cudaSuccess;
+  int dev = 0, sms = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e != cudaSuccess) return e;
+  stream_read_kernel<<<sms * 8, 256, 0, s>>>(static_cast<const uint4*>(src), bytes / 16);
+  return cudaGetLastError();
 }
 
 }  // namespace fk

@@ -62,6 +62,13 @@ struct LayerState {
   int ring_end = 0;
   int ring_head = 0;
   int sinks_done = 0;     // sink frames already in the dynamic views
+  // scoring sums formed by the current-chunk kernel since the last fk_compress: 0 none,
+  // 1 the sums of run frames [fuse_t_first, fuse_end) except the first fuse_n_read (which the
+  // scoring kernel reads), 2 sums that match no run (fk_compress clears them and rescores)
+  int fuse_state = 0;
+  int fuse_t_first = 0;
+  int fuse_end = 0;
+  int fuse_n_read = 0;
 };
 
 struct Staging {
@@ -147,6 +154,7 @@ struct fk_handle {
   float* scores = nullptr;
   int* kept = nullptr;
   unsigned long long* sums = nullptr;
+  size_t sums_bytes = 0;
   int* status = nullptr;
   // host-input staging: two slots per kind (K with V; Q), each with a ready event (copy done)
   // and a freed event (the kernel that read the slot has run); optional copy stream
@@ -418,8 +426,49 @@ fk_status push_history(fk_handle* h, int layer, const bf16* tokK, const bf16* to
   }
   ls.nh = nh1;
   ls.dirty = true;
+  if (ls.fuse_state == 1) ls.fuse_state = 2;   // frames the fused sums do not cover
   update_lengths(h, layer);
   return FK_OK;
+}
+
+// Whether the current-chunk kernel that retires layer `layer`'s current chunk can form the
+// pending scoring run's sums of the retired frames itself (Eq. 3 under the score contract):
+// the layer scores keys, the chunk has at most kFuseMaxFrames frames, the frame before the
+// chunk is a non-sink frame that stays in the window, and no other append since the last
+// fk_compress has touched the sums.  Fills the kernel's scoring fields and the layer's state.
+void plan_fused_scoring(fk_handle* h, int layer, CurrentArgs& a) {
+  LayerState& ls = h->layers[layer];
+  if (h->selection != FK_SELECT_SIMILARITY || h->layer_items[layer].second == 0) return;
+  const int anchor_old = ls.nh - 1, nh_new = ls.nh + h->C;
+  const int lo_new = h->W > 0 ? std::max(h->S, nh_new - h->W) : h->S;
+  bool ok = ls.fuse_state == 0 && h->C <= kFuseMaxFrames && anchor_old >= h->S && anchor_old >= lo_new;
+  int t_first = lo_new;            // whole-window rescoring: the run starts at the window
+  if (ok && h->incremental) {      // incremental: the run starts at the last scored anchor
+    ok = ls.scored_upto == anchor_old;
+    t_first = anchor_old;
+  }
+  if (!ok) {
+    if (ls.fuse_state == 1) ls.fuse_state = 2;
+    return;
+  }
+  a.score = 1;
+  a.score_partner_norm = h->incremental ? 1 : 0;
+  a.score_k0 = anchor_old - t_first;
+  a.n_seg = h->n;
+  a.seg_len = h->seg;
+  a.max_run = h->max_run;
+  a.sums = h->sums;
+  a.status = h->status;
+  const bool pooled = h->source == FK_SCORE_LAYER0_POOLED;
+  for (int hd = 0; hd < h->H; ++hd) {
+    const HeadBuf& hb = h->heads[layer * h->H + hd];
+    a.score_target[hd] = (short)(pooled ? 0 : (hb.is_static ? -1 : hb.target));
+  }
+  ls.fuse_state = 1;
+  ls.fuse_t_first = t_first;
+  ls.fuse_end = nh_new;
+  // the scoring kernel reads frames t_first .. anchor_old unless the kernel forms N(anchor_old)
+  ls.fuse_n_read = a.score_partner_norm ? 0 : a.score_k0 + 1;
 }
 
 // One pass of the current-chunk kernel: optionally retire the current chunk (view fronts)
@@ -459,6 +508,7 @@ fk_status update_current(fk_handle* h, int layer, bool retire, const void* K, co
     a.viewK8[hd] = h->fp8 ? h->viewK8 + hb.row_base * h->D : nullptr;
     a.is_static[hd] = hb.is_static ? 1 : 0;
   }
+  if (retire) plan_fused_scoring(h, layer, a);
   fk_status st = launch(h, s, FK_KERNEL_APPEND, [&] { launch_current(a, s); });
   if (st != FK_OK) return st;
   if (slot >= 0) FK_CUDA(cudaEventRecord(h->st_kv.freed[slot], s));
@@ -551,6 +601,15 @@ fk_status fk_classify_heads(const double* mass, int n_heads, int alpha_permille,
     head_is_static[hd] = (window <= 0.0 || local * 1000.0 > (double)alpha_permille * window) ? 1 : 0;
   }
   return FK_OK;
+}
+
+fk_status fk_stream_read(const void* src, size_t bytes, void* stream) {
+  if (!src || !aligned16(src) || (bytes & 15u)) return FK_ERR_ARG;
+  if (bytes == 0) return FK_OK;
+  if (!is_device_ptr(src)) return FK_ERR_ARG;
+  return launch_stream_read(src, (int64_t)bytes, static_cast<cudaStream_t>(stream)) == cudaSuccess
+             ? FK_OK
+             : FK_ERR_CUDA;
 }
 
 fk_status fk_wait_selftest(fk_handle* h, int limit_us, void* stream) {
@@ -751,8 +810,8 @@ fk_status fk_create(const fk_config* cfg, fk_handle** out) {
   if ((st = dev_alloc(h, nt * h->kmax * sizeof(int), &p)) != FK_OK) return fail(st);
   h->kept = static_cast<int*>(p);
   const size_t n_items = std::max<size_t>(1, h->score_items.size());
-  if ((st = dev_alloc(h, nt * h->max_run * h->n * 2 * sizeof(unsigned long long), &p)) != FK_OK)
-    return fail(st);
+  h->sums_bytes = nt * h->max_run * h->n * 2 * sizeof(unsigned long long);
+  if ((st = dev_alloc(h, h->sums_bytes, &p)) != FK_OK) return fail(st);
   h->sums = static_cast<unsigned long long*>(p);
   if ((st = dev_alloc(h, 256, &p)) != FK_OK) return fail(st);
   h->status = static_cast<int*>(p);
@@ -941,7 +1000,7 @@ fk_status fk_compress(fk_handle* h, void* stream) {
   }
   ScoreArgs sa{};
   CompactArgs ca{};
-  bool any_run = false, any_compact = false;
+  bool any_run = false, any_compact = false, clear_sums = false;
   // incremental compaction needs kept sets that never change once decided: per-frame scope
   const bool inc_compact = h->incremental && h->scope == FK_SCOPE_PER_FRAME;
   std::vector<int> keep_of(h->L, 0);
@@ -955,7 +1014,7 @@ fk_status fk_compress(fk_handle* h, void* stream) {
       // comparison rules: no scoring; the selection kernel ranks the whole window by the
       // rule's values
       if (r.n_scoreable > 0) {
-        sa.run[l] = {r.t_lo, r.n_scoreable + 1, 0};
+        sa.run[l] = {r.t_lo, r.n_scoreable + 1, 0, r.n_scoreable + 1};
         any_run = true;
       }
     } else if (ls.dirty && scores_here) {
@@ -963,11 +1022,20 @@ fk_status fk_compress(fk_handle* h, void* stream) {
       const int last_t = r.t_lo + r.n_scoreable - 1;
       if (r.n_scoreable > 0 && t_first <= last_t) {
         // the chunk the last append retired, [nh - C, nh), may still be in flight
-        sa.run[l] = {t_first, last_t + 2 - t_first, std::max(0, ls.nh - h->C)};
+        const int n_run = last_t + 2 - t_first;
+        int n_read = n_run;
+        if (ls.fuse_state == 1 && ls.fuse_t_first == t_first && ls.fuse_end == t_first + n_run)
+          n_read = ls.fuse_n_read;   // the current-chunk kernel formed the rest of the sums
+        else if (ls.fuse_state != 0)
+          clear_sums = true;         // partial sums that match no run: clear, rescore all
+        sa.run[l] = {t_first, n_run, std::max(0, ls.nh - h->C), n_read};
         any_run = true;
+      } else if (ls.fuse_state != 0) {
+        clear_sums = true;
       }
       ls.scored_upto = r.anchor >= 0 ? r.anchor : ls.scored_upto;
     }
+    if (scores_here) ls.fuse_state = 0;
     sa.t_lo[l] = r.t_lo;
     sa.n_scoreable[l] = r.n_scoreable;
     sa.n_keep[l] = keep;
@@ -1031,11 +1099,12 @@ fk_status fk_compress(fk_handle* h, void* stream) {
     // flattened (layer, item, segment, chunk, frame) range; items are grouped by layer
     long long units = 0;
     for (int l = 0; l < h->L; ++l) {
-      if (sa.run[l].n_run == 0 || h->layer_items[l].second == 0) continue;
+      if (clear_sums) sa.run[l].n_read = sa.run[l].n_run;
+      if (sa.run[l].n_read == 0 || h->layer_items[l].second == 0) continue;
       sa.act_layer[sa.n_active] = l;
       sa.act_first_item[sa.n_active] = h->layer_items[l].first;
       sa.act_start[sa.n_active] = units;
-      units += (long long)h->layer_items[l].second * h->n * h->chunks * sa.run[l].n_run;
+      units += (long long)h->layer_items[l].second * h->n * h->chunks * sa.run[l].n_read;
       ++sa.n_active;
     }
     sa.total_units = units;
@@ -1044,7 +1113,9 @@ fk_status fk_compress(fk_handle* h, void* stream) {
     sa.status = h->status;
     sa.rule = h->selection;
     sa.seed = h->select_seed;
-    if (h->selection == FK_SELECT_SIMILARITY &&
+    if (clear_sums)
+      FK_CUDA(cudaMemsetAsync(h->sums, 0, h->sums_bytes, s));
+    if (h->selection == FK_SELECT_SIMILARITY && units > 0 &&
         (st = launch(h, s, FK_KERNEL_SCORE, [&] { launch_score(sa, s); })) != FK_OK)
       return st;
     const int nt = (int)h->targets.size();

@@ -72,12 +72,37 @@ __device__ __forceinline__ int e4m3_row_exponent(float amax) {
 }
 // 2^k as a float for k in [-126, 127] (exact)
 __device__ __forceinline__ float pow2f(int k) { return __uint_as_float((uint32_t)(127 + k) << 23); }
+
+// Score contract (Eq. 3 under the kernel's precision), shared by the scoring kernel and the
+// current-chunk kernel.  Two channels (one 32-bit word: low half first) of the norm and dot fma
+// chains, with the bf16 values used directly as fma operands (fp32 product and accumulation, one
+// rounding): n += c*c and d += p*c for the low channel, then for the high channel.
+__device__ __forceinline__ void fma_word(uint32_t cw, uint32_t pw, float& n, float& d) {
+  asm("{\n .reg .b16 cl, ch, pl, ph;\n mov.b32 {cl, ch}, %2;\n mov.b32 {pl, ph}, %3;\n"
+      " fma.rn.f32.bf16 %0, cl, cl, %0;\n fma.rn.f32.bf16 %1, pl, cl, %1;\n"
+      " fma.rn.f32.bf16 %0, ch, ch, %0;\n fma.rn.f32.bf16 %1, ph, ch, %1;\n}"
+      : "+f"(n), "+f"(d) : "r"(cw), "r"(pw));
+}
+
+// trunc(v * 2^24) = hi * 2^24 + lo exactly, as two int32: hi = trunc(v) (|hi| <= 2^23 under
+// the precondition), v - hi is exact in fp32 (the low-order bits of v), lo = trunc((v - hi) *
+// 2^24) with |lo| < 2^24; hi and lo carry the sign of v, so both truncations go toward zero.
+// 32-bit conversions only (a float-to-int64 conversion would run on the FP64 pipe).
+__device__ __forceinline__ void fixed24_split(float v, int& hi, int& lo) {
+  hi = __float2int_rz(v);
+  lo = __float2int_rz(__fmul_rn(__fsub_rn(v, __int2float_rn(hi)), 16777216.0f));
+}
 #endif
 
 // ------------------------------------------------------------------ copy kernels
 // Current chunk update in one pass: each 16-byte granule of the previous current chunk (in
 // the view fronts) is first copied to its history location, then overwritten by the new
 // chunk's granule from the caller's token-major [C*F][H][D] buffer.
+// The retired chunk's frames pass through the current-chunk kernel's registers; when the layer
+// scores its keys, the same kernel forms their score-contract sums (Sec. 4.3, Eq. 3): the
+// squared norms N and the dots D with the previous frame, per (head, frame, segment), added into
+// the pending scoring run's int64 sums, so no scoring launch re-reads those frames.
+constexpr int kFuseMaxFrames = 15;   // chunks of at most this many frames can be scored in-kernel
 struct CurrentArgs {
   const bf16* srcK;             // new chunk, token-major; nullptr = retire only
   const bf16* srcV;
@@ -94,6 +119,16 @@ struct CurrentArgs {
   bf16* pageV[kMaxHeads];
   uint8_t* viewK8[kMaxHeads];   // FP8_QK: E4M3 copies of the K views, same rows (else nullptr)
   unsigned char is_static[kMaxHeads];   // static: sink / anchor slots live in the view
+  // in-kernel scoring of the retired chunk (requires retire; every retired frame and the frame
+  // before the chunk are non-sink window frames, and C <= kFuseMaxFrames)
+  int score;                    // 1: form the sums of the retired frames
+  int score_partner_norm;       // 1: also N of the frame before the chunk (run frame score_k0)
+  int score_k0;                 // run-relative index of the frame before the chunk; retired
+                                // frame r is run frame score_k0 + 1 + r
+  int n_seg, seg_len, max_run;
+  unsigned long long* sums;     // [target][max_run][n_seg][2]: {N, D}, as the scoring kernel
+  int* status;
+  short score_target[kMaxHeads];   // sums target of head h, -1: not scored
 };
 void launch_current(const CurrentArgs& a, cudaStream_t s);
 
@@ -122,11 +157,13 @@ struct SelectTarget {           // one kept set: its layer and the score items f
   int n_items;
 };
 
-struct LayerRun {               // per layer: frames t_first..t_first+n_run-1 are read
+struct LayerRun {               // per layer: the run of frames t_first..t_first+n_run-1
   int t_first;
-  int n_run;                    // 0 = nothing to score in this layer
+  int n_run;                    // frames whose sums the selection kernel finishes; 0 = none
   int t_fresh;                  // frames >= t_fresh may come from the kernel launched just
                                 // before (the chunk it retired): read after its completion
+  int n_read;                   // frames t_first.. the scoring kernel reads (the rest of the
+                                // run's sums were formed by the current-chunk kernel)
 };
 
 // Scoring of new frame pairs (score kernel), then the finish of the scores and BottomK
@@ -199,6 +236,8 @@ struct CompactArgs {
 };
 constexpr int kCompactPiece = 16384;
 void launch_compact(const CompactArgs& a, cudaStream_t s);
+// streaming read of `bytes` (a multiple of 16) from 16-byte aligned device memory: calibration
+cudaError_t launch_stream_read(const void* src, int64_t bytes, cudaStream_t s);
 
 // ------------------------------------------------------------------ attention
 struct AttnArgs {

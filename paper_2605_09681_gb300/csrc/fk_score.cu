@@ -35,25 +35,6 @@ __device__ __forceinline__ uint4 lds128(uint32_t smem) {
   return v;
 }
 
-// Two channels (one 32-bit word: low half first) of the norm and dot fma chains, with the
-// bf16 values used directly as fma operands (fp32 product and accumulation, one rounding):
-// n += c*c and d += p*c for the low channel, then for the high channel.
-__device__ __forceinline__ void fma_word(uint32_t cw, uint32_t pw, float& n, float& d) {
-  asm("{\n .reg .b16 cl, ch, pl, ph;\n mov.b32 {cl, ch}, %2;\n mov.b32 {pl, ph}, %3;\n"
-      " fma.rn.f32.bf16 %0, cl, cl, %0;\n fma.rn.f32.bf16 %1, pl, cl, %1;\n"
-      " fma.rn.f32.bf16 %0, ch, ch, %0;\n fma.rn.f32.bf16 %1, ph, ch, %1;\n}"
-      : "+f"(n), "+f"(d) : "r"(cw), "r"(pw));
-}
-
-// trunc(v * 2^24) = hi * 2^24 + lo exactly, as two int32: hi = trunc(v) (|hi| <= 2^23 under
-// the precondition), v - hi is exact in fp32 (the low-order bits of v), lo = trunc((v - hi) *
-// 2^24) with |lo| < 2^24; hi and lo carry the sign of v, so both truncations go toward zero.
-// 32-bit conversions only (a float-to-int64 conversion would run on the FP64 pipe).
-__device__ __forceinline__ void fixed24_split(float v, int& hi, int& lo) {
-  hi = __float2int_rz(v);
-  lo = __float2int_rz(__fmul_rn(__fsub_rn(v, __int2float_rn(hi)), 16777216.0f));
-}
-
 __device__ __forceinline__ int ring_slot(int f, int S, int cap) {
   return f < S ? f : S + (f - S) % cap;
 }
@@ -529,13 +510,13 @@ __global__ void __launch_bounds__(kScoreThreads, 4) score_kernel(const ScoreArgs
     }
     const LayerRun run = a.run[a.act_layer[lo]];
     const long long idx = g - a.act_start[lo];
-    const long long chunk_id = idx / run.n_run;
-    const int k = (int)(idx - chunk_id * run.n_run);
+    const long long chunk_id = idx / run.n_read;
+    const int k = (int)(idx - chunk_id * run.n_read);
     const int item_local = (int)(chunk_id / per_item);
     const int r = (int)(chunk_id - (long long)item_local * per_item);
     const int j = r / a.chunks;
     const long long left = g_end - g;
-    const int k_last = (int)(left < run.n_run - k ? k + left - 1 : run.n_run - 1);
+    const int k_last = (int)(left < run.n_read - k ? k + left - 1 : run.n_read - 1);
     if (!score_run<D>(a, a.act_first_item[lo] + item_local, j, r - j * a.chunks, k, k_last, smem, seq,
                       waited))
       break;
@@ -779,7 +760,7 @@ extern "C" fk_status fk_segment_scores_noalloc(const void* K, int n_frames, int 
   a.status = status ? status : reinterpret_cast<int*>(sc + kNoAllocCtrOff) + 3;
   a.scores = scores;
   a.kept = reinterpret_cast<int*>(sc + kNoAllocTargetOff + 32);   // unused: no selection
-  a.run[0] = {0, n_frames, 0};
+  a.run[0] = {0, n_frames, 0, n_frames};
   a.t_lo[0] = 0;
   a.n_scoreable[0] = 0;
   a.n_keep[0] = 0;

@@ -86,7 +86,13 @@ def test_algorithmic_work_of_the_480p_step():
     keys = [7800] * 6 + [25480] * 6
     alg = bench._algorithmic(w, keys)
     assert alg["attn_flops"] == 4 * 4680 * 128 * (6 * 7800 + 6 * 25480)            # 478.47 GFLOP
-    assert alg["score_bytes"] == 6 * 18 * 1560 * 128 * 2                           # 43.13 MB
+    # the scoring kernel reads frames 1..15 (the frame before the retired chunk included); the
+    # current-chunk kernel forms the sums of the retired frames 16..18 as it moves them
+    assert alg["score_fused"] and alg["score_bytes"] == 6 * 15 * 1560 * 128 * 2    # 35.94 MB
+    # chunk K, V read + written; each static head's anchor slot and each dynamic head's three
+    # retired frames (K, V read + written); each dynamic head's partner key frame
+    assert alg["append_bytes"] == (2 * 2 * 4680 * 12 * 128 * 2 + 6 * 2 * 2 * 1560 * 128 * 2
+                                   + 6 * 2 * 2 * 3 * 1560 * 128 * 2 + 6 * 1560 * 128 * 2)
     assert alg["compact_bytes"] == 6 * (1560 + 17 * 4 * 260 + 1560) * 128 * 2 * 2 * 2  # 127.8 MB
     cfg = bench._config(w, keys)
     assert cfg["queries"] == 4680 and cfg["history_frames"] == 18 and cfg["keys_per_head"] == keys

@@ -150,6 +150,39 @@ def test_stream_incremental_matches_rescore():
     assert got[0] == got[1]
 
 
+@pytest.mark.parametrize("incremental", [True, False])
+@pytest.mark.parametrize("D", [64, 128])
+def test_stream_irregular_appends(incremental, D):
+    # the current-chunk kernel forms the scoring sums of the chunk it retires when nothing else
+    # touched them since the last compress; two chunk appends before one compress, or a history
+    # prefill after a chunk, leave sums that match no run: they are cleared and rescored.  Kept
+    # sets and scores bit-exact, attention in tolerance, at every compress.
+    from paper_2605_09681_gb300 import ForcingKVCache
+    w = W.ROLLING.with_(name="irregular", head_dim=D, tokens_per_frame=72, n_segments=4, n_heads=4,
+                        window_frames=7, n_chunks=12, incremental=incremental, scene_cut_every_chunks=5)
+    hm = W.head_map(w)
+    orc = O.ForcingKVOracle.from_workload(w, hm)
+    fs = W.FrameStream(w, 0)
+    skip = {2, 5, 6}          # chunks appended without a compress right after them
+    with ForcingKVCache.from_workload(w, hm) as cache:
+        for c in range(w.n_chunks):
+            if c == 8:        # a prefill of two frames after a chunk, before the compress
+                k, v = fs.frames(2)
+                cache.append_frames(0, to_dev(k), to_dev(v))
+                orc.append_frames(0, k, v)
+            k, v = fs.frames(w.frames_per_chunk)
+            cache.append_chunk(0, to_dev(k), to_dev(v))
+            orc.append_chunk(0, k, v)
+            if c in skip:
+                continue
+            cache.compress()
+            q = W.queries(w, 0, c, 0)
+            Od = cache.attend(0, to_dev(q))
+            torch.cuda.synchronize()
+            compare_layer(cache, orc, 0, q, Od, label="irregular c%d" % c)
+        assert cache.sync_status() == 0
+
+
 def test_stream_layer0_pooled_small():
     w = W.P480_STACK.with_(name="stack_small", n_layers=3, n_heads=4, head_dim=64,
                            tokens_per_frame=60, n_chunks=5, denoise_steps=2)
