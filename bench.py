@@ -89,7 +89,6 @@ def _algorithmic(w, key_counts):
     nq = w.n_queries
     flops = sum(4.0 * nq * nk * D for nk in key_counts)
     nh, S, Wn = w.n_history_frames, w.n_sink_frames, w.window_frames
-    n_sink = min(S, nh)
     lo = max(S, nh - Wn) if Wn > 0 else S
     has_anchor = nh - 1 >= lo
     n_scoreable = (nh - 1 - lo) if has_anchor else 0
@@ -103,10 +102,13 @@ def _algorithmic(w, key_counts):
     score_bytes = n_dyn * read_frames * F * D * 2 if scored else 0
     k_frame = w.n_segments if w.selection == "all" else w.keep_budget_permille * w.n_segments // 1000
     n_keep = n_scoreable * k_frame
-    unit_tokens = n_sink * F + n_keep * (F // w.n_segments) + (F if has_anchor else 0)
-    compact_bytes = n_dyn * 2 * 2 * unit_tokens * D * 2
+    # compaction gathers the kept segments; the sinks and the anchor reach the views in the
+    # current-chunk kernel (a static head's anchor slot, a dynamic head's retired frames into
+    # its pages plus the new anchor into its view)
+    compact_bytes = n_dyn * 2 * 2 * n_keep * (F // w.n_segments) * D * 2
     append_bytes = 2 * 2 * nq * H * D * 2 + sum(
-        2 * 2 * (F if st else C * F) * D * 2 for st in static) + (n_dyn * F * D * 2 if fused else 0)
+        2 * 2 * (F if st else C * F) * D * 2 for st in static) + (n_dyn * F * D * 2 if fused else 0) \
+        + (n_dyn * 2 * F * D * 2 if has_anchor else 0)
     return dict(attn_flops=flops, score_bytes=score_bytes, compact_bytes=compact_bytes,
                 append_bytes=append_bytes, score_fused=fused)
 
@@ -529,7 +531,7 @@ def run_incremental(args, w, hm, local_rank, hk, hv, dK, dV, dQ, dO, flush, stre
     n_dyn = sum(1 for st in _workload_static(w) if not st)
     k_frame = w.keep_budget_permille * w.n_segments // 1000
     score_bytes = n_dyn * (C + 1) * F * D * 2
-    compact_bytes = n_dyn * 2 * 2 * (C * k_frame * (F // w.n_segments) + F) * D * 2
+    compact_bytes = n_dyn * 2 * 2 * C * k_frame * (F // w.n_segments) * D * 2
     alg = _algorithmic(w, keys)
 
     def kern(kind, nbytes):
@@ -553,7 +555,8 @@ def run_incremental(args, w, hm, local_rank, hk, hv, dK, dV, dQ, dO, flush, stre
         "note": "per step: the current-chunk kernel forms the scoring sums of the C retired frames "
                 "(and the squared norms of the frame before them) while moving them, so no scoring "
                 "launch runs (score is null); compaction copies C x k segments + the anchor frame per "
-                "dynamic head (ring-buffer views)",
+                "dynamic head into its ring of kept segments (the anchor frame reaches the view in "
+                "the current-chunk kernel)",
     }
 
 

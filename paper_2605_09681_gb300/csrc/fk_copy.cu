@@ -1,9 +1,10 @@
 // Data-movement kernels of the Forcing-KV cache: the current-chunk update (the previous
-// current chunk joins the history pages and the new chunk is scattered from the caller's
-// token-major [tokens][H][D] layout into the per-head views, in one pass), the prefill
-// scatter of history frames, and the select-and-compact gather of kept segments into the
-// packed per-head views of dynamic heads (Sec. 4.3, Eq. 4: sink, kept segments and the
-// anchor frame; attention does not depend on the order of the keys, so a view holds them as
+// current chunk joins the history pages, and the views' sink and anchor slots where it holds
+// those frames, and the new chunk is scattered from the caller's token-major [tokens][H][D]
+// layout into the per-head views, in one pass; it can also form the scoring sums of the frames
+// it retires), the prefill scatter of history frames, and the gather of kept segments into the
+// packed per-head views of dynamic heads (Sec. 4.3, Eq. 4: sink, kept segments and the anchor
+// frame; attention does not depend on the order of the keys, so a view holds them as
 // [sinks | anchor | kept-segment ring] and incremental compaction only appends).
 // All of them are HBM-bound: every byte is read once and written once in 16-byte accesses.
 // Under FP8_QK attention each of them also writes the E4M3 codes of every view K row it writes
@@ -45,7 +46,9 @@ __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;"
 // D/8 16-byte granules per token row) across all C frames of the chunk: thread (p, c) moves
 // granule c of rows r*F + p, r < C, of the new chunk (token-major [C*F][H][D], 256 contiguous
 // bytes per token and head) into the view front, after copying the previous current chunk's
-// granule to its history location.  Frames go in batches of two with every load of a batch
+// granule to its history locations: the page ring (heads that keep history), and the view's
+// sink slots and anchor slot (a retired sink frame; the new anchor frame, which every dynamic
+// view and, unless they drop it, every static view holds).  Frames go in batches of two with every load of a batch
 // issued before its first store.
 //
 // With a.score set, the CTA also forms the score-contract sums of the retired frames (Eq. 3):
@@ -105,9 +108,9 @@ __global__ void __launch_bounds__(256, 4) current_kernel(const CurrentArgs a) {
       const int f = a.nh_old + r;
       return a.retire && a.pageK[h] != nullptr && (f < a.S || f >= lo_new);
     };
-    auto to_slot = [&](int r) {
+    auto to_slot = [&](int r) {   // every view holds the sinks; dynamic views the new anchor too
       const int f = a.nh_old + r;
-      return a.retire && a.is_static[h] && (f < a.S || (a.static_anchor && f == nh_new - 1));
+      return a.retire && (f < a.S || (f == nh_new - 1 && (!a.is_static[h] || a.static_anchor)));
     };
 #pragma unroll
     for (int i = 0; i < kBatch; ++i) {
@@ -212,37 +215,20 @@ __global__ void __launch_bounds__(256) scatter_kernel(const ScatterArgs a) {
   }
 }
 
-// Source and destination element offsets of unit u of a dynamic head's compaction; false
-// when u is past the layer's units.  Units in order: the sink frames to copy (n units each),
-// the anchor frame (n units), the kept segments to copy (one unit each, from the target's kept
-// list).  View rows after the current chunk: sink frame f at S-slot f, the anchor after the
-// sinks, kept segment i in ring slot (rp0 + i) mod kmax after the anchor.
+// Source and destination element offsets of unit u of a dynamic head's compaction (its u-th
+// kept segment to copy, from the target's kept list); false when u is past the layer's units.
+// The segment goes to ring slot (rp0 + u) mod kmax of the view's kept-segment ring, after the
+// current chunk, the sinks and the anchor (which the current-chunk and prefill kernels write).
 __device__ __forceinline__ bool unit_offsets(const CompactArgs& a, const CompactItem& it, int u,
                                              int64_t& src_off, int64_t& dst_off) {
   const int l = it.layer;
-  const int n_sink_units = a.n_sink_copy[l] * a.n_seg;
-  const int n_anchor_units = a.anchor[l] >= 0 ? a.n_seg : 0;
-  if (u >= n_sink_units + n_anchor_units + a.n_kept_copy[l]) return false;
-  int frame, seg;
-  int64_t dst_row = a.CF;
-  if (u < n_sink_units) {
-    frame = a.sink_first[l] + u / a.n_seg;
-    seg = u - (u / a.n_seg) * a.n_seg;
-    dst_row += (int64_t)frame * a.F + (int64_t)seg * a.seg_len;
-  } else if (u < n_sink_units + n_anchor_units) {
-    frame = a.anchor[l];
-    seg = u - n_sink_units;
-    dst_row += (int64_t)a.S * a.F + (int64_t)seg * a.seg_len;
-  } else {
-    const int i = u - n_sink_units - n_anchor_units;
-    const int sid = a.kept[(int64_t)it.target * a.kmax + a.kp0[l] + i];
-    frame = sid / a.n_seg;
-    seg = sid - frame * a.n_seg;
-    const int slot = (a.rp0[l] + i) % a.kmax;
-    dst_row += (int64_t)a.S * a.F + a.F + (int64_t)slot * a.seg_len;
-  }
-  const int slot = ring_slot(frame, a.S, a.cap_nonsink);
-  src_off = ((int64_t)slot * a.F + (int64_t)seg * a.seg_len) * a.D;
+  if (u >= a.n_kept_copy[l]) return false;
+  const int sid = a.kept[(int64_t)it.target * a.kmax + a.kp0[l] + u];
+  const int frame = sid / a.n_seg;
+  const int seg = sid - frame * a.n_seg;
+  const int slot = (a.rp0[l] + u) % a.kmax;
+  const int64_t dst_row = a.CF + (int64_t)a.S * a.F + a.F + (int64_t)slot * a.seg_len;
+  src_off = ((int64_t)ring_slot(frame, a.S, a.cap_nonsink) * a.F + (int64_t)seg * a.seg_len) * a.D;
   dst_off = dst_row * a.D;
   return true;
 }

@@ -61,7 +61,6 @@ struct LayerState {
   int ring_first = 0;
   int ring_end = 0;
   int ring_head = 0;
-  int sinks_done = 0;     // sink frames already in the dynamic views
   // scoring sums formed by the current-chunk kernel since the last fk_compress: 0 none,
   // 1 the sums of run frames [fuse_t_first, fuse_end) except the first fuse_n_read (which the
   // scoring kernel reads), 2 sums that match no run (fk_compress clears them and rescores)
@@ -407,7 +406,9 @@ fk_status push_history(fk_handle* h, int layer, const bf16* tokK, const bf16* to
         pa.dstV[hd] = hb.pageV + ring_slot(h, f) * frame_elems;
         any_p = true;
       }
-      if (hb.is_static && (sink || (is_anchor && !h->drop_anchor))) {
+      // every view holds the sinks; every dynamic view (and, unless they drop it, every
+      // static view) holds the anchor
+      if (sink || (is_anchor && (!hb.is_static || !h->drop_anchor))) {
         const int64_t row = h->CF + (int64_t)(sink ? f : h->S) * h->F;
         va.dstK[hd] = hb.viewK + row * h->D;
         va.dstV[hd] = hb.viewV + row * h->D;
@@ -1040,14 +1041,9 @@ fk_status fk_compress(fk_handle* h, void* stream) {
     sa.n_scoreable[l] = r.n_scoreable;
     sa.n_keep[l] = keep;
     keep_of[l] = keep;
-    ca.anchor[l] = r.anchor;
     ca.active[l] = ls.dirty ? 1 : 0;
     if (!ls.dirty) continue;
     if (inc_compact) {
-      // sinks not yet in the views
-      ca.sink_first[l] = ls.sinks_done;
-      ca.n_sink_copy[l] = r.n_sink - ls.sinks_done;
-      ls.sinks_done = r.n_sink;
       // frames below the window leave the ring; the newly decided frames are appended.  A
       // frame leaves only once the window is full, and then the ring is full again after the
       // append, so the valid slots are always [0, count) or all kmax: one contiguous key range
@@ -1066,14 +1062,11 @@ fk_status fk_compress(fk_handle* h, void* stream) {
       ls.ring_end = std::max(ls.ring_end, t_hi);
       if (ls.ring_head != 0 && keep != h->kmax) return FK_ERR_STATE;   // cannot happen (see above)
     } else {
-      ca.sink_first[l] = 0;
-      ca.n_sink_copy[l] = r.n_sink;
       ca.n_kept_copy[l] = keep;
       ca.kp0[l] = 0;
       ca.rp0[l] = 0;
     }
-    const int units = ca.n_sink_copy[l] * h->n + ca.n_kept_copy[l] + (r.anchor >= 0 ? h->n : 0);
-    ca.max_units = std::max(ca.max_units, units);
+    ca.max_units = std::max(ca.max_units, ca.n_kept_copy[l]);
   }
   for (const auto& ci : h->compact_items) any_compact |= ca.active[ci.layer] != 0;
   fk_status st;

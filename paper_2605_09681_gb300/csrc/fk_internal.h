@@ -223,11 +223,9 @@ struct CompactArgs {
   int splits;                   // pieces per unit (each at most kCompactPiece bytes per tensor)
   int units_per_cta;            // whole units per CTA when a unit is smaller (then splits = 1)
   const int* kept;
-  // per layer: what this launch copies into the dynamic views [current | sinks | anchor |
-  // kept ring of kmax segment slots]
-  int sink_first[kMaxLayers];   // first sink frame to copy
-  int n_sink_copy[kMaxLayers];  // sink frames to copy
-  int anchor[kMaxLayers];       // anchor frame (copied whole), -1 = none
+  // per layer: the kept segments this launch copies into the dynamic views' kept-segment rings
+  // (views are [current | sinks | anchor | kept ring of kmax segment slots]; the sinks and the
+  // anchor are written by the current-chunk and prefill kernels)
   int n_kept_copy[kMaxLayers];  // kept segments to copy
   int kp0[kMaxLayers];          // their first position in the target's kept list
   int rp0[kMaxLayers];          // ring slot of the first one (slots wrap modulo kmax)

@@ -90,10 +90,12 @@ def test_algorithmic_work_of_the_480p_step():
     # current-chunk kernel forms the sums of the retired frames 16..18 as it moves them
     assert alg["score_fused"] and alg["score_bytes"] == 6 * 15 * 1560 * 128 * 2    # 35.94 MB
     # chunk K, V read + written; each static head's anchor slot and each dynamic head's three
-    # retired frames (K, V read + written); each dynamic head's partner key frame
+    # retired frames (K, V read + written); each dynamic head's partner key frame; each dynamic
+    # head's new anchor frame (K, V) written into its view
     assert alg["append_bytes"] == (2 * 2 * 4680 * 12 * 128 * 2 + 6 * 2 * 2 * 1560 * 128 * 2
-                                   + 6 * 2 * 2 * 3 * 1560 * 128 * 2 + 6 * 1560 * 128 * 2)
-    assert alg["compact_bytes"] == 6 * (1560 + 17 * 4 * 260 + 1560) * 128 * 2 * 2 * 2  # 127.8 MB
+                                   + 6 * 2 * 2 * 3 * 1560 * 128 * 2 + 6 * 1560 * 128 * 2
+                                   + 6 * 2 * 1560 * 128 * 2)
+    assert alg["compact_bytes"] == 6 * 17 * 4 * 260 * 128 * 2 * 2 * 2             # 108.7 MB
     cfg = bench._config(w, keys)
     assert cfg["queries"] == 4680 and cfg["history_frames"] == 18 and cfg["keys_per_head"] == keys
 
