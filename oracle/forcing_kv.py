@@ -278,6 +278,35 @@ def attention_fp8_qk(Q: np.ndarray, K: np.ndarray, V: np.ndarray) -> np.ndarray:
     return attention_fp64(q8 * np.ldexp(1.0, e)[:, None], e4m3_round(K), V)
 
 
+# FP8 attention with P V on E4M3 operands too (the reading of the quantization appendix that
+# also quantizes the value path): Q K^T exactly as in `attention_fp8_qk`; the softmax
+# numerators p = exp(l - max_l) of each row are scaled by 2^6 and rounded to e4m3, V is rounded
+# to e4m3 unscaled, and the row's normaliser is the sum of the unrounded numerators:
+#   O = sum_k e4m3(2^6 p_k) e4m3(V_k) / (2^6 sum_k p_k).
+# The scale keeps 2^6 p <= 64 on the e4m3 grid (max 448), with relative precision 2^-4 down to
+# p = 2^-12 and subnormal steps of 2^-9 / 2^6 below; a kernel that lets its running maximum lag
+# the row maximum by a factor up to 4 scales p by up to 2^8 and stays within 448.
+P_SCALE_EXP = 6
+
+
+def attention_fp8(Q: np.ndarray, K: np.ndarray, V: np.ndarray, row_block: int = 256) -> np.ndarray:
+    """FP8 attention with both products on e4m3 operands, in fp64 on the rounded values."""
+    q8, e = quantize_q_rows(Q)
+    Qs = q8 * np.ldexp(1.0, e)[:, None]
+    K8 = e4m3_round(K)
+    V8 = e4m3_round(V)
+    scale = 1.0 / np.sqrt(Qs.shape[1])
+    ps = np.ldexp(1.0, P_SCALE_EXP)
+    out = np.empty((Qs.shape[0], V8.shape[1]), dtype=np.float64)
+    for r0 in range(0, Qs.shape[0], row_block):
+        logits = (Qs[r0:r0 + row_block] @ K8.T) * scale
+        logits -= logits.max(axis=1, keepdims=True)
+        p = np.exp(logits)
+        p8 = e4m3_round(p * ps)
+        out[r0:r0 + row_block] = (p8 @ V8) / (ps * p.sum(axis=1, keepdims=True))
+    return out
+
+
 # --------------------------------------------------------------------------------------
 # comparison selection rules (App. H, Sec. 5.3): ranking values replacing the scores
 # --------------------------------------------------------------------------------------
@@ -384,7 +413,7 @@ class ForcingKVOracle:
             raise ValueError(selection)
         self.selection, self.seed = selection, int(select_seed) & 0xFFFFFFFF
         self.keep_anchor_static = not static_drop_anchor
-        if attn_precision not in ("bf16", "fp8_qk"):
+        if attn_precision not in ("bf16", "fp8_qk", "fp8"):
             raise ValueError(attn_precision)
         self.attn_precision = attn_precision
         self.static = np.asarray(head_is_static, dtype=np.uint8).reshape(n_layers, n_heads)
@@ -534,14 +563,16 @@ class ForcingKVOracle:
 
     def attend(self, layer, Q_bits, heads=None, rows=None, kept=None) -> np.ndarray:
         """O [rows, H, D] fp64: each head's queries over its Eq. 2 / Eq. 4 key set (Q K^T
-        on e4m3 operands when the attention precision is "fp8_qk")."""
+        on e4m3 operands when the attention precision is "fp8_qk", both products when it is
+        "fp8")."""
         Q = _bf16_to_f32(Q_bits)
         rows = np.arange(Q.shape[0]) if rows is None else np.asarray(rows)
         heads = range(self.H) if heads is None else heads
         O = np.full((len(rows), self.H, self.D), np.nan)
         for h in heads:
             K, V = self.gather_kv(layer, h, None if kept is None else kept.get(h))
-            att = attention_fp8_qk if self.attn_precision == "fp8_qk" else attention_fp64
+            att = {"fp8_qk": attention_fp8_qk, "fp8": attention_fp8}.get(self.attn_precision,
+                                                                         attention_fp64)
             O[:, h, :] = att(Q[rows, h, :], K, V)
         return O
 
