@@ -279,13 +279,16 @@ def attention_fp8_qk(Q: np.ndarray, K: np.ndarray, V: np.ndarray) -> np.ndarray:
 
 
 # FP8 attention with P V on E4M3 operands too (the reading of the quantization appendix that
-# also quantizes the value path): Q K^T exactly as in `attention_fp8_qk`; the softmax
-# numerators p = exp(l - max_l) of each row are scaled by 2^6 and rounded to e4m3, V is rounded
-# to e4m3 unscaled, and the row's normaliser is the sum of the unrounded numerators:
-#   O = sum_k e4m3(2^6 p_k) e4m3(V_k) / (2^6 sum_k p_k).
-# The scale keeps 2^6 p <= 64 on the e4m3 grid (max 448), with relative precision 2^-4 down to
-# p = 2^-12 and subnormal steps of 2^-9 / 2^6 below; a kernel that lets its running maximum lag
-# the row maximum by a factor up to 4 scales p by up to 2^8 and stays within 448.
+# also quantizes the value path): Q K^T exactly as in `attention_fp8_qk`; with each row's
+# logits in log2 units, y_k = l_k / ln 2, and the row's reference R = ceil(max_k y_k) (the row
+# maximum rounded up to an integer), the softmax numerators are n_k = 2^(y_k - R + 6), rounded
+# to e4m3; V is rounded to e4m3 unscaled; the row's normaliser is the sum of the unrounded
+# numerators:
+#   O = sum_k e4m3(n_k) e4m3(V_k) / sum_k n_k.
+# The numerators lie in (0, 2^6] (e4m3 max 448), with relative precision 2^-4 down to 2^-6 and
+# subnormal steps of 2^-9 below.  An integer reference makes the rounding independent of where
+# a kernel's running reference stands: two integer references differ by an exact power of two,
+# under which e4m3 rounding of normal values is invariant.
 P_SCALE_EXP = 6
 
 
@@ -295,15 +298,13 @@ def attention_fp8(Q: np.ndarray, K: np.ndarray, V: np.ndarray, row_block: int = 
     Qs = q8 * np.ldexp(1.0, e)[:, None]
     K8 = e4m3_round(K)
     V8 = e4m3_round(V)
-    scale = 1.0 / np.sqrt(Qs.shape[1])
-    ps = np.ldexp(1.0, P_SCALE_EXP)
+    scale = 1.0 / (np.sqrt(Qs.shape[1]) * np.log(2.0))     # logits in log2 units
     out = np.empty((Qs.shape[0], V8.shape[1]), dtype=np.float64)
     for r0 in range(0, Qs.shape[0], row_block):
-        logits = (Qs[r0:r0 + row_block] @ K8.T) * scale
-        logits -= logits.max(axis=1, keepdims=True)
-        p = np.exp(logits)
-        p8 = e4m3_round(p * ps)
-        out[r0:r0 + row_block] = (p8 @ V8) / (ps * p.sum(axis=1, keepdims=True))
+        y = (Qs[r0:r0 + row_block] @ K8.T) * scale
+        R = np.ceil(y.max(axis=1, keepdims=True))
+        n = np.exp2(y - R + P_SCALE_EXP)
+        out[r0:r0 + row_block] = (e4m3_round(n) @ V8) / n.sum(axis=1, keepdims=True)
     return out
 
 

@@ -632,31 +632,47 @@ def test_fp8_attention_quantizes_within_e4m3_error():
 
 # ---- FP8 attention with P V on e4m3 operands too
 def test_fp8_pv_one_key_returns_the_rounded_value():
-    # a single key: p = 1, e4m3(2^6) = 64 exactly, so O = e4m3(V) / 1 exactly
+    # a single key with logit 0: reference ceil(0) = 0, numerator 2^6 = 64 (on the grid), so
+    # O = e4m3(V) exactly, whatever the query
     rng = _rng(41)
-    Q, K, V = _bf16(rng.standard_normal((5, 128))), _bf16(rng.standard_normal((1, 128))), \
-        _bf16(rng.standard_normal((1, 128)) * 3)
-    out = O.attention_fp8(Q, K, V)
+    Q, V = _bf16(rng.standard_normal((5, 128))), _bf16(rng.standard_normal((1, 128)) * 3)
+    out = O.attention_fp8(Q, np.zeros((1, 128)), V)
     assert np.array_equal(out, np.repeat(O.e4m3_round(V), 5, axis=0))
 
 
+def test_fp8_pv_reference_is_the_row_max_rounded_up():
+    # one key, logit 2.75 / 8 = 0.34375 (q = 1 and k = 2.75 on channel 0, both e4m3-exact; the
+    # query row scales to 256): y = 0.34375 / ln 2 = 0.496, reference ceil(y) = 1, numerator
+    # n = 2^(y + 5) = 45.13, which rounds to 44 on the e4m3 grid (binade [32, 64), step 4);
+    # O = 44 / n x e4m3(V).  With the exact row maximum as reference (n = 64) O would be e4m3(V).
+    D = 64
+    Q = np.zeros((1, D))
+    Q[0, 0] = 1.0
+    K = np.zeros((1, D))
+    K[0, 0] = 2.75
+    V = np.full((1, D), 3.0)
+    n = 2.0 ** (0.34375 / math.log(2.0) + 5.0)
+    assert 44.0 < n < 46.0
+    out = O.attention_fp8(Q, K, V)
+    assert np.allclose(out, 44.0 / n * 3.0, rtol=1e-14, atol=0)
+
+
 def test_fp8_pv_equal_keys_average_the_rounded_values():
-    # equal keys: every numerator is 1 (64 after scaling, exact), O = mean of e4m3(V)
+    # equal keys with logit 0: every numerator is 64 (exact), O = mean of e4m3(V)
     rng = _rng(42)
     Q = _bf16(rng.standard_normal((3, 64)))
-    K = np.repeat(_bf16(rng.standard_normal((1, 64))), 7, axis=0)
     V = _bf16(rng.standard_normal((7, 64)))
-    out = O.attention_fp8(Q, K, V)
+    out = O.attention_fp8(Q, np.zeros((7, 64)), V)
     want = O.e4m3_round(V).mean(axis=0)
     assert np.abs(out - want[None, :]).max() <= 1e-15
 
 
 def test_fp8_pv_scale_is_two_to_the_six():
     # two keys with logits 0 and -12 (q = 8 on channel 0, keys 0 and -12 there: all exact in
-    # e4m3, the query row scaled by 2^5 to 256): numerators 1 and e^-12 = 6.1e-6, which lies in
-    # (2^-18, 2^-16).  Scaled by 2^6 it stays below half the smallest e4m3 step (2^-10) and
-    # rounds to 0, so O = 0 exactly although the second key's value is 448; a scale of 2^8
-    # (or an unrounded numerator) would leave a visible 448 e^-12 / (1 + e^-12) = 2.7e-3
+    # e4m3, the query row scaled by 2^5 to 256): reference 0, numerators 2^6 and 2^6 e^-12 =
+    # 3.9e-4, below half the smallest e4m3 step (2^-10): it rounds to 0, so O = 0 exactly although
+    # the second key's value is 448; a scale of 2^8 (or an unrounded numerator) would leave a
+    # visible 448 e^-12 / (1 + e^-12) = 2.7e-3
     D = 64
     Q = np.zeros((1, D))
     Q[0, 0] = 8.0
@@ -668,14 +684,14 @@ def test_fp8_pv_scale_is_two_to_the_six():
     assert np.array_equal(out, np.zeros((1, D)))
     assert np.allclose(O.attention_fp8_qk(Q, K, V), 448.0 * math.exp(-12) / (1 + math.exp(-12)),
                        rtol=1e-12, atol=0)
-    # the first key alone: numerator 1 -> 64 on the grid, weight 64 / (64 (1 + e^-12))
+    # the first key alone: numerator 64 on the grid, weight 64 / (64 (1 + e^-12))
     V[0, :], V[1, :] = 2.0, 0.0
     assert np.allclose(O.attention_fp8(Q, K, V), 2.0 / (1 + math.exp(-12)), rtol=1e-14, atol=0)
 
 
 def test_fp8_pv_within_the_e4m3_error_of_its_numerators():
     # against the same attention with unrounded numerators (fp8_qk on e4m3(V)): each numerator
-    # moves by at most max(2^-4 x, 2^-10) of its scaled value x = 2^6 p (half an e4m3 step)
+    # x moves by at most max(2^-4 x, 2^-10) (half an e4m3 step)
     rng = _rng(43)
     D = 128
     Q = _bf16(rng.standard_normal((40, D)))
@@ -684,10 +700,18 @@ def test_fp8_pv_within_the_e4m3_error_of_its_numerators():
     got = O.attention_fp8(Q, K, V)
     ref = O.attention_fp8_qk(Q, K, O.e4m3_round(V))
     q8, e = O.quantize_q_rows(Q)
-    logits = (q8 * np.ldexp(1.0, e)[:, None]) @ O.e4m3_round(K).T / math.sqrt(D)
-    p = np.exp(logits - logits.max(axis=1, keepdims=True))
-    x = p * 64.0
-    bound = (np.maximum(x * 2.0 ** -4, 2.0 ** -10) @ np.abs(O.e4m3_round(V))) / (64.0 * p.sum(axis=1, keepdims=True))
+    y = (q8 * np.ldexp(1.0, e)[:, None]) @ O.e4m3_round(K).T / (math.sqrt(D) * math.log(2.0))
+    x = np.exp2(y - np.ceil(y.max(axis=1, keepdims=True)) + 6)
+    assert x.max() <= 64.0 and x.max(axis=1).min() > 32.0
+    bound = (np.maximum(x * 2.0 ** -4, 2.0 ** -10) @ np.abs(O.e4m3_round(V))) / x.sum(axis=1, keepdims=True)
     assert (np.abs(got - ref) <= bound * (1 + 1e-9) + 1e-15).all()
     assert np.abs(got - ref).max() > 0                    # the rounding is not a no-op
 
+
+def test_fp8_pv_power_of_two_reference_shift_changes_nothing():
+    # scaling every numerator by 2^k (a kernel's running reference below the row's) leaves the
+    # e4m3 rounding of normal values unchanged: numerators above 2^-6 for k in {0, 1, 2}
+    rng = _rng(44)
+    x = np.exp2(rng.uniform(-6.0, 6.0, 5000))
+    for k in (1, 2):
+        assert np.array_equal(O.e4m3_round(x * 2.0 ** k), O.e4m3_round(x) * 2.0 ** k)
