@@ -93,18 +93,23 @@ enum {
   FK_SELECT_RANDOM = 3
 };
 
-/* Operand precision of the chunk attention's Q K^T product (the paper's quantization
- * appendix: FP8 attention on the compressed cache).  BF16: Q, K, V in bf16 (the method).
+/* Operand precision of the chunk attention (the paper's quantization appendix: FP8 attention
+ * on the compressed cache).  BF16: Q, K, V in bf16 (the method).
  * FP8_QK: Q K^T on OCP FP8 E4M3 operands with f32 accumulation; P V stays bf16.  Keys are
  * rounded to E4M3 unscaled (E4M3 keeps the same relative precision over its normal range,
  * 2^-6 to 448): FP8_QK requires key elements within +-448, larger ones saturate.  Each query
  * row (token, head) is scaled by 2^-e, e the smallest integer with max |q| <= 448 * 2^e, and
  * the logits are scaled back by 2^e, so the E4M3 rounding (to nearest, ties to even) is the
  * only inexact step before the softmax.  fk_quantize_e4m3 applies the same rounding.
- * FP8_QK requires head_dim 128. */
+ * FP8: Q K^T as FP8_QK, and P V on E4M3 operands too, f32 accumulation: values are rounded to
+ * E4M3 unscaled (elements within +-448), and each softmax numerator exp(l - m) is scaled by
+ * 2^6 before its E4M3 rounding, m being the running row maximum, which lags the row maximum by
+ * at most a factor 2 (so a numerator stays within 2^7); the row normaliser is the sum of the
+ * unrounded scaled numerators.  Both FP8 precisions require head_dim 128. */
 enum {
   FK_ATTN_BF16 = 0,
-  FK_ATTN_FP8_QK = 1
+  FK_ATTN_FP8_QK = 1,
+  FK_ATTN_FP8 = 2
 };
 
 /* Configuration of one cache.  The method's quantities (Sec. 4.2-4.3 and App. H): F tokens per
@@ -191,7 +196,7 @@ FK_API fk_status fk_compress(fk_handle* h, void* stream);
 /* O [C*F][H][D] = per head softmax(Q K^T / sqrt(D)) V over the head's key set: Eq. 2
  * for static heads, Eq. 4 plus the anchor frame for dynamic heads.  Q: [C*F][H][D].
  * Under FK_ATTN_FP8_QK, Q K^T runs on E4M3 operands (the rounding described there; P V in
- * bf16).  FK_ERR_STATE if `layer` has no current chunk or was appended to since the last
+ * bf16); under FK_ATTN_FP8 P V too.  FK_ERR_STATE if `layer` has no current chunk or was appended to since the last
  * fk_compress. */
 FK_API fk_status fk_attend(fk_handle* h, int layer, const void* Q, void* O, void* stream);
 

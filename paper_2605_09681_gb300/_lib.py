@@ -16,7 +16,7 @@ STATUS_NAMES = {0: "FK_OK", 1: "FK_ERR_CONFIG", 2: "FK_ERR_ARG", 3: "FK_ERR_STAT
 FK_SCOPE_PER_FRAME, FK_SCOPE_POOLED = 0, 1
 FK_SCORE_PER_HEAD, FK_SCORE_LAYER0_POOLED = 0, 1
 FK_SELECT = {"similarity": 0, "all": 1, "uniform": 2, "random": 3}
-FK_ATTN = {"bf16": 0, "fp8_qk": 1}
+FK_ATTN = {"bf16": 0, "fp8_qk": 1, "fp8": 2}
 KERNEL_KINDS = {"append": 0, "score": 1, "select": 2, "compact": 3, "attend": 4}
 
 EXPORTS = [

@@ -33,6 +33,11 @@ namespace {
 
 constexpr uint64_t kWaitLimitNs = 2000000000ull;   // 2 s per wait
 constexpr float kRescaleThreshold = 8.0f;          // log2 units: rescale O when max grows > 2^8
+// FP8 P V: P is stored as e4m3 of 2^6 exp2(s c - m), m an integer running reference (the
+// running max rounded up) that lags the row max by at most 2 (rescale threshold), so P stays
+// within 2^8 < 448; reference changes rescale O and l by exact powers of two
+constexpr float kRescaleThresholdFp8 = 2.0f;
+constexpr float kPShiftFp8 = 6.0f;
 
 constexpr int kWarpTma = 8;                        // warps 0-3 / 4-7: softmax of query tile 0 / 1
 constexpr int kWarpMma = 9;
@@ -49,11 +54,11 @@ struct AttnBarriers {
   volatile int abort;
 };
 
-template <int D, bool kFp8 = false>
+template <int D, bool kFp8 = false, bool kFp8PV = false>
 struct Layout {
   static constexpr int kQ = kAttnBM * D * (kFp8 ? 1 : 2);   // one 128-row query tile (MMA operand)
   static constexpr int kK = kAttnBN * D * (kFp8 ? 1 : 2);   // one 128-key K tile
-  static constexpr int kKV = kAttnBN * D * 2;               // one 128-key V tile (bf16)
+  static constexpr int kKV = kAttnBN * D * (kFp8PV ? 1 : 2);  // one 128-key V tile
   static constexpr int kQ16 = kFp8 ? kAttnBM * D * 2 : 0;   // FP8: one bf16 query tile as loaded
   static constexpr int kOffQ = 0;                 // two query tiles
   static constexpr int kOffK = kOffQ + 2 * kQ;    // two K stages
@@ -155,9 +160,9 @@ __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, int b_mn) {
          ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
 }
 // Instruction descriptor, kind::f8f6f4: f32 accumulate, A and B E4M3 (type code 0 at bits
-// 7 and 10), both K-major.
-__host__ __device__ constexpr uint32_t idesc_e4m3(int M, int N) {
-  return (1u << 4) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+// 7 and 10), A K-major, B K-major (b_mn = 0) or MN-major (b_mn = 1).
+__host__ __device__ constexpr uint32_t idesc_e4m3(int M, int N, int b_mn = 0) {
+  return (1u << 4) | ((uint32_t)b_mn << 16) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
 }
 
 __device__ __forceinline__ void umma(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
@@ -182,6 +187,15 @@ __device__ __forceinline__ void umma_f8(uint32_t d_tmem, uint64_t a, uint64_t b,
       "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
       " tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n}\n"
       :: "r"(d_tmem), "l"(a), "l"(b), "r"(idesc), "r"(accumulate) : "memory");
+}
+// D[tmem] (+)= A[tmem] * B[smem] on E4M3 operands: A (M x 32, four codes per 32-bit column) in
+// tensor memory, B from a shared-memory descriptor
+__device__ __forceinline__ void umma_ts_f8(uint32_t d_tmem, uint32_t a_tmem, uint64_t b, uint32_t idesc,
+                                           uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], [%1], %2, %3, p;\n}\n"
+      :: "r"(d_tmem), "r"(a_tmem), "l"(b), "r"(idesc), "r"(accumulate) : "memory");
 }
 __device__ __forceinline__ void umma_commit(uint64_t* b) {
   asm volatile(
@@ -230,6 +244,23 @@ __device__ __forceinline__ void umma_commit(uint64_t* b) {
         "r"(v[20]), "r"(v[21]), "r"(v[22]), "r"(v[23]), "r"(v[24]), "r"(v[25]), "r"(v[26]),  \
         "r"(v[27]), "r"(v[28]), "r"(v[29]), "r"(v[30]), "r"(v[31]) : "memory")
 
+#define FK_TMEM_LD16(taddr, v)                                                              \
+  asm volatile(                                                                             \
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,"  \
+      "%13,%14,%15}, [%16];"                                                                \
+      : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]),  \
+        "=r"(v[7]), "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]),           \
+        "=r"(v[13]), "=r"(v[14]), "=r"(v[15])                                               \
+      : "r"(taddr))
+
+#define FK_TMEM_ST16(taddr, v)                                                              \
+  asm volatile(                                                                             \
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,"   \
+      "%12,%13,%14,%15,%16};"                                                               \
+      :: "r"(taddr), "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]),      \
+        "r"(v[6]), "r"(v[7]), "r"(v[8]), "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]),      \
+        "r"(v[13]), "r"(v[14]), "r"(v[15]) : "memory")
+
 __device__ __forceinline__ void tmem_wait_ld() {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
@@ -259,19 +290,34 @@ __device__ __forceinline__ float2 fadd2(float2 a, float2 b) {
   return d;
 }
 
+// four e4m3 codes (one TMEM column of P, lowest key in the low byte) times alpha, re-rounded
+__device__ __forceinline__ uint32_t scale_e4m3x4(uint32_t w, float alpha) {
+  uint32_t lo, hi;
+  asm("{\n .reg .b16 a, b;\n mov.b32 {a, b}, %2;\n cvt.rn.f16x2.e4m3x2 %0, a;\n"
+      " cvt.rn.f16x2.e4m3x2 %1, b;\n}" : "=r"(lo), "=r"(hi) : "r"(w));
+  const float2 f0 = __half22float2(*reinterpret_cast<const __half2*>(&lo));
+  const float2 f1 = __half22float2(*reinterpret_cast<const __half2*>(&hi));
+  return e4m3x2(f0.x * alpha, f0.y * alpha) | (e4m3x2(f1.x * alpha, f1.y * alpha) << 16);
+}
+
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   const __nv_bfloat162 p = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<const uint32_t*>(&p);
 }
 
 // kSplit: a launch with key splits (kv_splits > 1); the unsplit instantiation carries none of
-// the split bookkeeping.  kFp8: Q K^T on E4M3 operands (D = 128).
-template <int D, bool kSplit, bool kFp8>
+// the split bookkeeping.  kFp8: Q K^T on E4M3 operands (D = 128).  kFp8PV (with kFp8): P V on
+// E4M3 operands too: V tiles from the E4M3 copy of the V view arena (one 128-byte swizzle atom
+// per key row), P written as e4m3 of 2^6 exp2(s c - m), four keys per TMEM column.
+template <int D, bool kSplit, bool kFp8, bool kFp8PV = false>
 __global__ void __launch_bounds__(kAttnThreads, 1)
 attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
             const __grid_constant__ CUtensorMap tmV, const AttnArgs a) {
   static_assert(!kFp8 || D == 128, "FP8_QK: one 128-byte swizzle atom per Q / K row");
-  using Lay = Layout<D, kFp8>;
+  static_assert(!kFp8PV || kFp8, "FP8 P V comes with FP8 Q K^T");
+  using Lay = Layout<D, kFp8, kFp8PV>;
+  constexpr float kThr = kFp8PV ? kRescaleThresholdFp8 : kRescaleThreshold;
+  constexpr float kPShift = kFp8PV ? kPShiftFp8 : 0.0f;
   constexpr int kHalves = D / 64;                 // 64-column (128-byte) swizzle atoms
   constexpr uint32_t kTmemCols = 512;
   constexpr uint32_t kColO = 2 * kAttnBN;         // S0 = cols 0..127, S1 = 128..255, O0, O1 after
@@ -357,9 +403,13 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
         lastK[st] = u;
         if (j >= 2 && !wait_phase(&bar->v_empty[st], (u - 1) & 1, bar, a.status)) { ok = false; break; }
         mbar_expect_tx(&bar->v_full[st], Lay::kKV);
-        for (int h = 0; h < kHalves; ++h)
-          tma_load_2d(sV + st * Lay::kKV + h * 16384, &tmV, &bar->v_full[st], h * 64,
-                      row0 + j * kAttnBN);
+        if constexpr (kFp8PV) {
+          tma_load_2d(sV + st * Lay::kKV, &tmV, &bar->v_full[st], 0, row0 + j * kAttnBN);
+        } else {
+          for (int h = 0; h < kHalves; ++h)
+            tma_load_2d(sV + st * Lay::kKV + h * 16384, &tmV, &bar->v_full[st], h * 64,
+                        row0 + j * kAttnBN);
+        }
         lastV[st] = u;
       }
       if (!ok) {   // drain every load this thread issued before the CTA exits
@@ -379,7 +429,7 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
     // S_t(j+1) overwriting P_t(j) (same columns) happens after PV_t(j) has read it.
     if (lane == 0) {
       constexpr uint32_t kIdQK = kFp8 ? idesc_e4m3(kAttnBM, kAttnBN) : idesc_bf16(kAttnBM, kAttnBN, 0);
-      constexpr uint32_t kIdPV = idesc_bf16(kAttnBM, D, 1);
+      constexpr uint32_t kIdPV = kFp8PV ? idesc_e4m3(kAttnBM, D, 1) : idesc_bf16(kAttnBM, D, 1);
       const uint32_t aQ = su32(sQ), aK = su32(sK), aV = su32(sV);
       auto qk = [&](int j, int t) {
         const int st = j & 1;
@@ -403,11 +453,22 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
       };
       auto pv = [&](int j, int t) {
         const int st = j & 1;
+        if constexpr (kFp8PV) {
+          // 32 keys per step: P columns 8 kk .. 8 kk + 7 (four codes each); V rows 32 kk .. +31,
+          // MN-major (d contiguous, 128 bytes per key row), 8-row groups 1024 bytes apart
 #pragma unroll
-        for (int kk = 0; kk < kAttnBN / 16; ++kk) {
-          const uint64_t db = sdesc(aV + st * Lay::kKV + kk * 2048, 16384, 1024);
-          umma_ts(tmem + kColO + (uint32_t)(t * D), tmem + (uint32_t)(t * kAttnBN + kk * 8), db,
-                  kIdPV, (j > 0 || kk > 0) ? 1u : 0u);
+          for (int kk = 0; kk < kAttnBN / 32; ++kk) {
+            const uint64_t db = sdesc(aV + st * Lay::kKV + kk * 4096, 16384, 1024);
+            umma_ts_f8(tmem + kColO + (uint32_t)(t * D), tmem + (uint32_t)(t * kAttnBN + kk * 8), db,
+                       kIdPV, (j > 0 || kk > 0) ? 1u : 0u);
+          }
+        } else {
+#pragma unroll
+          for (int kk = 0; kk < kAttnBN / 16; ++kk) {
+            const uint64_t db = sdesc(aV + st * Lay::kKV + kk * 2048, 16384, 1024);
+            umma_ts(tmem + kColO + (uint32_t)(t * D), tmem + (uint32_t)(t * kAttnBN + kk * 8), db,
+                    kIdPV, (j > 0 || kk > 0) ? 1u : 0u);
+          }
         }
       };
       bool ok = wait_phase(kFp8 ? &bar->q8_ready : &bar->q_full, 0, bar, a.status) &&
@@ -500,7 +561,9 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
       // One pass per 64-column half: the half's maximum (eight independent chains), a lazy
       // update of the running max m (only when it grows by more than 2^8), then
       // P = exp2(S*c - m) as bf16 pairs written over the S columns already read (P columns
-      // 32h..32h+31 come from S columns 64h..64h+63): the A operand of PV.  If the second
+      // 32h..32h+31 come from S columns 64h..64h+63): the A operand of PV.  FP8 P V: m is the
+      // running max rounded up to an integer, updated when it grows by more than 2, and P the
+      // e4m3 codes of 2^6 exp2(S*c - m), four per column (P columns 16h..16h+15).  If the second
       // half raises m, the first half's stored P is rescaled in place.
 #pragma unroll
       for (int half = 0; half < 2; ++half) {
@@ -520,29 +583,70 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
         }
         const float mx = fmaxf(fmaxf(fmaxf(mxa[0], mxa[1]), fmaxf(mxa[2], mxa[3])),
                                fmaxf(fmaxf(mxa[4], mxa[5]), fmaxf(mxa[6], mxa[7])));
-        const float m_new = fmaxf(m, mx * sl2);
-        if (__any_sync(0xffffffffu, m_new > m + kRescaleThreshold)) {   // warp-uniform
-          const float alpha = fast_exp2(m - m_new);  // 0 when m = -inf
+        const float m_new = fmaxf(m, kFp8PV ? ceilf(mx * sl2) : mx * sl2);
+        if (__any_sync(0xffffffffu, m_new > m + kThr)) {               // warp-uniform
+          float alpha;                               // 0 when m = -inf
+          if constexpr (kFp8PV) {                    // integer references: an exact power of two
+            const float dm = m - m_new;
+            alpha = (m == -INFINITY || dm < -126.0f) ? 0.0f : pow2f((int)dm);
+          } else {
+            alpha = fast_exp2(m - m_new);
+          }
           l *= alpha;
 #pragma unroll
           for (int i = 0; i < 4; ++i) acc[i] = make_float2(acc[i].x * alpha, acc[i].y * alpha);
           if (half == 1) {                           // rare: first half of P was stored with the old m
-            uint32_t p0[32];
-            tmem_wait_st();
-            FK_TMEM_LD32(tS, p0);
-            tmem_wait_ld();
+            if constexpr (kFp8PV) {
+              uint32_t p0[16];
+              tmem_wait_st();
+              FK_TMEM_LD16(tS, p0);
+              tmem_wait_ld();
 #pragma unroll
-            for (int e = 0; e < 32; ++e) {
-              const __nv_bfloat162 b = *reinterpret_cast<const __nv_bfloat162*>(&p0[e]);
-              p0[e] = pack_bf16(__low2float(b) * alpha, __high2float(b) * alpha);
+              for (int e = 0; e < 16; ++e) p0[e] = scale_e4m3x4(p0[e], alpha);
+              FK_TMEM_ST16(tS, p0);
+            } else {
+              uint32_t p0[32];
+              tmem_wait_st();
+              FK_TMEM_LD32(tS, p0);
+              tmem_wait_ld();
+#pragma unroll
+              for (int e = 0; e < 32; ++e) {
+                const __nv_bfloat162 b = *reinterpret_cast<const __nv_bfloat162*>(&p0[e]);
+                p0[e] = pack_bf16(__low2float(b) * alpha, __high2float(b) * alpha);
+              }
+              FK_TMEM_ST32(tS, p0);
             }
-            FK_TMEM_ST32(tS, p0);
           }
           alpha_tile *= alpha;
           rescaled = true;
           m = m_new;
         }
-        const float2 nm2 = make_float2(-m, -m);
+        const float2 nm2 = make_float2(kPShift - m, kPShift - m);
+        if constexpr (kFp8PV) {
+          uint32_t pk[16];
+          if (!full) {                               // the ragged last tile: masked keys give 0
+#pragma unroll
+            for (int c = 0; c < 64; ++c)
+              if (half * 64 + c >= valid) sv[c] = __float_as_uint(-INFINITY);
+          }
+#pragma unroll
+          for (int q = 0; q < 16; ++q) {
+            const float2 x0 = ffma2(make_float2(__uint_as_float(sv[4 * q]), __uint_as_float(sv[4 * q + 1])),
+                                    sc2, nm2);
+            const float2 x1 = ffma2(make_float2(__uint_as_float(sv[4 * q + 2]), __uint_as_float(sv[4 * q + 3])),
+                                    sc2, nm2);
+            float2 e0, e1;
+            e0.x = fast_exp2(x0.x);
+            e0.y = fast_exp2(x0.y);
+            e1.x = fast_exp2(x1.x);
+            e1.y = fast_exp2(x1.y);
+            acc[(2 * q) & 3] = fadd2(acc[(2 * q) & 3], e0);
+            acc[(2 * q + 1) & 3] = fadd2(acc[(2 * q + 1) & 3], e1);
+            pk[q] = e4m3x2(e0.x, e0.y) | (e4m3x2(e1.x, e1.y) << 16);
+          }
+          FK_TMEM_ST16(tS + half * 16, pk);
+          continue;
+        }
         uint32_t pk[32];
         if (full) {
 #pragma unroll
@@ -923,19 +1027,25 @@ cudaError_t attention_prepare(int head_dim) {
     if ((e = set((const void*)attn_kernel<128, false, false>, Layout<128>::kSmem)) != cudaSuccess) return e;
     if ((e = set((const void*)attn_kernel<128, true, false>, Layout<128>::kSmem)) != cudaSuccess) return e;
     if ((e = set((const void*)attn_kernel<128, false, true>, Layout<128, true>::kSmem)) != cudaSuccess) return e;
-    return set((const void*)attn_kernel<128, true, true>, Layout<128, true>::kSmem);
+    if ((e = set((const void*)attn_kernel<128, true, true>, Layout<128, true>::kSmem)) != cudaSuccess) return e;
+    if ((e = set((const void*)attn_kernel<128, false, true, true>, Layout<128, true, true>::kSmem)) != cudaSuccess)
+      return e;
+    return set((const void*)attn_kernel<128, true, true, true>, Layout<128, true, true>::kSmem);
   }
   if ((e = set((const void*)attn_kernel<64, false, false>, Layout<64>::kSmem)) != cudaSuccess) return e;
   return set((const void*)attn_kernel<64, true, false>, Layout<64>::kSmem);
 }
 
-void launch_attention(int head_dim, bool fp8, const CUtensorMap& tmQ, const CUtensorMap& tmK,
+void launch_attention(int head_dim, int precision, const CUtensorMap& tmQ, const CUtensorMap& tmK,
                       const CUtensorMap& tmV, const AttnArgs& a, cudaStream_t s) {
   using Kern = void (*)(const CUtensorMap, const CUtensorMap, const CUtensorMap, const AttnArgs);
   const bool split = a.kv_splits > 1;
   Kern kern;
   int smem;
-  if (head_dim == 128 && fp8) {
+  if (head_dim == 128 && precision == FK_ATTN_FP8) {
+    kern = split ? attn_kernel<128, true, true, true> : attn_kernel<128, false, true, true>;
+    smem = Layout<128, true, true>::kSmem;
+  } else if (head_dim == 128 && precision == FK_ATTN_FP8_QK) {
     kern = split ? attn_kernel<128, true, true> : attn_kernel<128, false, true>;
     smem = Layout<128, true>::kSmem;
   } else if (head_dim == 128) {

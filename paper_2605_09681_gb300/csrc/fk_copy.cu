@@ -7,8 +7,9 @@
 // frame; attention does not depend on the order of the keys, so a view holds them as
 // [sinks | anchor | kept-segment ring] and incremental compaction only appends).
 // All of them are HBM-bound: every byte is read once and written once in 16-byte accesses.
-// Under FP8_QK attention each of them also writes the E4M3 codes of every view K row it writes
-// (8 bytes per 16-byte granule), so the attention's key operand is ready without another pass.
+// Under FP8 attention each of them also writes the E4M3 codes of every view K row it writes
+// (8 bytes per 16-byte granule), and of every view V row under FP8 P V, so the attention's
+// operands are ready without another pass.
 #include "fk_internal.h"
 
 namespace fk {
@@ -142,12 +143,14 @@ __global__ void __launch_bounds__(256, 4) current_kernel(const CurrentArgs a) {
         st_v4(a.viewK[h] + so, ko[i]);
         st_v4(a.viewV[h] + so, vo[i]);
         if (a.viewK8[h]) *reinterpret_cast<uint2*>(a.viewK8[h] + so) = e4m3x8(ko[i], 1.0f);
+        if (a.viewV8[h]) *reinterpret_cast<uint2*>(a.viewV8[h] + so) = e4m3x8(vo[i], 1.0f);
       }
       if (a.srcK) {
         const int64_t vof = (int64_t)(r * a.F + p) * D + c * 8;
         st_v4(a.viewK[h] + vof, kn[i]);
         st_v4(a.viewV[h] + vof, vn[i]);
         if (a.viewK8[h]) *reinterpret_cast<uint2*>(a.viewK8[h] + vof) = e4m3x8(kn[i], 1.0f);
+        if (a.viewV8[h]) *reinterpret_cast<uint2*>(a.viewV8[h] + vof) = e4m3x8(vn[i], 1.0f);
       }
     }
     if (scoring) {
@@ -211,7 +214,11 @@ __global__ void __launch_bounds__(256) scatter_kernel(const ScatterArgs a) {
       st_v4(a.dstK[h] + dst_off, k);
       if (a.dstK8[h]) *reinterpret_cast<uint2*>(a.dstK8[h] + dst_off) = e4m3x8(k, 1.0f);
     }
-    if (a.dstV[h]) st_v4(a.dstV[h] + dst_off, ld_stream(a.srcV + (size_t)g * 8));
+    if (a.dstV[h]) {
+      const uint4 v = ld_stream(a.srcV + (size_t)g * 8);
+      st_v4(a.dstV[h] + dst_off, v);
+      if (a.dstV8[h]) *reinterpret_cast<uint2*>(a.dstV8[h] + dst_off) = e4m3x8(v, 1.0f);
+    }
   }
 }
 
@@ -256,6 +263,7 @@ __global__ void __launch_bounds__(256) compact_kernel(const CompactArgs a) {
     uint4* dK = reinterpret_cast<uint4*>(it.viewK + dst_off);
     uint4* dV = reinterpret_cast<uint4*>(it.viewV + dst_off);
     uint2* dK8 = it.viewK8 ? reinterpret_cast<uint2*>(it.viewK8 + dst_off) : nullptr;
+    uint2* dV8 = it.viewV8 ? reinterpret_cast<uint2*>(it.viewV8 + dst_off) : nullptr;
 #pragma unroll
     for (int r = 0; r < kPer; ++r) {
       const int64_t i = g0 + threadIdx.x + r * 256;
@@ -271,6 +279,7 @@ __global__ void __launch_bounds__(256) compact_kernel(const CompactArgs a) {
         st_v4(dK + i, k[r]);
         st_v4(dV + i, v[r]);
         if (dK8) dK8[i] = e4m3x8(k[r], 1.0f);
+        if (dV8) dV8[i] = e4m3x8(v[r], 1.0f);
       }
     }
     return;
@@ -299,6 +308,7 @@ __global__ void __launch_bounds__(256) compact_kernel(const CompactArgs a) {
       st_v4(dK[r], k[r]);
       st_v4(dV[r], v[r]);
       if (it.viewK8) *reinterpret_cast<uint2*>(it.viewK8 + e8[r]) = e4m3x8(k[r], 1.0f);
+      if (it.viewV8) *reinterpret_cast<uint2*>(it.viewV8 + e8[r]) = e4m3x8(v[r], 1.0f);
     }
   }
 }

@@ -141,7 +141,9 @@ struct fk_handle {
   int selection = FK_SELECT_SIMILARITY;
   uint32_t select_seed = 0;
   bool drop_anchor = false;        // static heads keep sink + current chunk only
-  bool fp8 = false;                // FK_ATTN_FP8_QK
+  bool fp8 = false;                // FK_ATTN_FP8_QK or FK_ATTN_FP8: Q K^T on E4M3
+  bool fp8pv = false;              // FK_ATTN_FP8: P V on E4M3 too
+  int precision = FK_ATTN_BF16;
   std::vector<HeadBuf> heads;      // [L*H]
   std::vector<LayerState> layers;  // [L]
   // device memory
@@ -184,8 +186,10 @@ struct fk_handle {
   int max_run = 0;
   int score_ctas = 0;
   CUtensorMap tmK{}, tmV{};
-  uint8_t* viewK8 = nullptr;       // FP8_QK: E4M3 codes of the K view arena
+  uint8_t* viewK8 = nullptr;       // FP8: E4M3 codes of the K view arena
   CUtensorMap tmK8{};
+  uint8_t* viewV8 = nullptr;       // FP8 P V: E4M3 codes of the V view arena
+  CUtensorMap tmV8{};
   const void* q_cached[2] = {};   // two cached Q maps (the two Q staging slots alternate)
   CUtensorMap tmQ[2]{};
   int q_next = 0;
@@ -413,6 +417,7 @@ fk_status push_history(fk_handle* h, int layer, const bf16* tokK, const bf16* to
         va.dstK[hd] = hb.viewK + row * h->D;
         va.dstV[hd] = hb.viewV + row * h->D;
         if (h->fp8) va.dstK8[hd] = h->viewK8 + (hb.row_base + row) * h->D;
+        if (h->fp8pv) va.dstV8[hd] = h->viewV8 + (hb.row_base + row) * h->D;
         any_v = true;
       }
     }
@@ -507,6 +512,7 @@ fk_status update_current(fk_handle* h, int layer, bool retire, const void* K, co
     a.pageK[hd] = hb.retains ? hb.pageK : nullptr;
     a.pageV[hd] = hb.retains ? hb.pageV : nullptr;
     a.viewK8[hd] = h->fp8 ? h->viewK8 + hb.row_base * h->D : nullptr;
+    a.viewV8[hd] = h->fp8pv ? h->viewV8 + hb.row_base * h->D : nullptr;
     a.is_static[hd] = hb.is_static ? 1 : 0;
   }
   if (retire) plan_fused_scoring(h, layer, a);
@@ -672,8 +678,10 @@ fk_status fk_validate_config(const fk_config* c) {
   if (c->selection < FK_SELECT_SIMILARITY || c->selection > FK_SELECT_RANDOM) return FK_ERR_CONFIG;
   if (c->selection == FK_SELECT_UNIFORM && c->select_scope != FK_SCOPE_PER_FRAME) return FK_ERR_CONFIG;
   if (c->static_drop_anchor != 0 && c->static_drop_anchor != 1) return FK_ERR_CONFIG;
-  if (c->attn_precision != FK_ATTN_BF16 && c->attn_precision != FK_ATTN_FP8_QK) return FK_ERR_CONFIG;
-  if (c->attn_precision == FK_ATTN_FP8_QK && c->head_dim != 128) return FK_ERR_CONFIG;
+  if (c->attn_precision != FK_ATTN_BF16 && c->attn_precision != FK_ATTN_FP8_QK &&
+      c->attn_precision != FK_ATTN_FP8)
+    return FK_ERR_CONFIG;
+  if (c->attn_precision != FK_ATTN_BF16 && c->head_dim != 128) return FK_ERR_CONFIG;
   const int64_t cf = (int64_t)c->frames_per_chunk * c->tokens_per_frame;
   if (cf > (1 << 24) || (int64_t)c->tokens_per_frame * c->head_dim > (1 << 28)) return FK_ERR_CONFIG;
   // 16-byte granules of one chunk (all heads) are indexed with 32-bit integers
@@ -716,7 +724,9 @@ fk_status fk_create(const fk_config* cfg, fk_handle** out) {
   h->selection = cfg->selection;
   h->select_seed = cfg->select_seed;
   h->drop_anchor = cfg->static_drop_anchor != 0;
-  h->fp8 = cfg->attn_precision == FK_ATTN_FP8_QK;
+  h->precision = cfg->attn_precision;
+  h->fp8 = cfg->attn_precision != FK_ATTN_BF16;
+  h->fp8pv = cfg->attn_precision == FK_ATTN_FP8;
   h->k_frame = h->selection == FK_SELECT_ALL ? h->n : (h->b * h->n) / 1000;
   h->kmax = std::max(1, keep_total(h, h->cap_nonsink - 1));
   h->chunks = (h->seg + kScoreTokensPerCta - 1) / kScoreTokensPerCta;
@@ -783,6 +793,10 @@ fk_status fk_create(const fk_config* cfg, fk_handle** out) {
   h->viewK = static_cast<bf16*>(p);
   if ((st = dev_alloc(h, view_bytes, &p)) != FK_OK) return fail(st);
   h->viewV = static_cast<bf16*>(p);
+  if (h->fp8pv) {
+    if ((st = dev_alloc(h, view_bytes / 2, &p)) != FK_OK) return fail(st);
+    h->viewV8 = static_cast<uint8_t*>(p);
+  }
   if (h->fp8) {
     if ((st = dev_alloc(h, view_bytes / 2, &p)) != FK_OK) return fail(st);
     h->viewK8 = static_cast<uint8_t*>(p);
@@ -876,7 +890,8 @@ fk_status fk_create(const fk_config* cfg, fk_handle** out) {
       const HeadBuf& hb = h->heads[l * h->H + hd];
       if (hb.is_static) continue;
       h->compact_items.push_back({hb.pageK, hb.pageV, hb.viewK, hb.viewV, l, hb.target,
-                                  h->fp8 ? h->viewK8 + hb.row_base * h->D : nullptr});
+                                  h->fp8 ? h->viewK8 + hb.row_base * h->D : nullptr,
+                                  h->fp8pv ? h->viewV8 + hb.row_base * h->D : nullptr});
     }
   auto upload = [&](const void* src, size_t bytes, void** dst) -> fk_status {
     fk_status s2 = dev_alloc(h, std::max<size_t>(bytes, 16), dst);
@@ -897,6 +912,8 @@ fk_status fk_create(const fk_config* cfg, fk_handle** out) {
   if ((st = encode_2d(&h->tmK, h->viewK, h->view_rows_total, h->D)) != FK_OK) return fail(st);
   if ((st = encode_2d(&h->tmV, h->viewV, h->view_rows_total, h->D)) != FK_OK) return fail(st);
   if (h->fp8 && (st = encode_2d(&h->tmK8, h->viewK8, h->view_rows_total, h->D, true)) != FK_OK)
+    return fail(st);
+  if (h->fp8pv && (st = encode_2d(&h->tmV8, h->viewV8, h->view_rows_total, h->D, true)) != FK_OK)
     return fail(st);
   if (cudaDeviceSynchronize() != cudaSuccess) return fail(FK_ERR_CUDA);
   for (int l = 0; l < h->L; ++l) update_lengths(h, l);
@@ -1197,10 +1214,12 @@ fk_status fk_attend(fk_handle* h, int layer, const void* Q, void* O, void* strea
   a.part_o = h->part_o;
   a.part_ml = h->part_ml;
   const int D = h->D;
-  // FP8_QK: the E4M3 keys come from the view arena's E4M3 copy; the kernel quantizes Q
+  // FP8: the E4M3 keys (and, for P V, values) come from the view arenas' E4M3 copies; the kernel
+  // quantizes Q
   const CUtensorMap& tk = h->fp8 ? h->tmK8 : h->tmK;
+  const CUtensorMap& tv = h->fp8pv ? h->tmV8 : h->tmV;
   if ((st = launch(h, s, FK_KERNEL_ATTEND, [&] {
-         launch_attention(D, h->fp8, h->tmQ[qm], tk, h->tmV, a, s);
+         launch_attention(D, h->precision, h->tmQ[qm], tk, tv, a, s);
          if (a.kv_splits > 1) launch_merge(D, a, s);
        })) != FK_OK)
     return st;
@@ -1233,7 +1252,7 @@ size_t fk_cache_bytes(const fk_handle* h) {
       const HeadBuf& hb = h->heads[l * h->H + hd];
       if (hb.retains) bytes += (size_t)live_frames * frame_bytes;
       const int rows = hb.is_static ? ls.len_static : ls.len_dynamic;
-      bytes += (size_t)rows * h->D * (h->fp8 ? 5 : 4);   // K and V bf16 (+ E4M3 K)
+      bytes += (size_t)rows * h->D * (4 + (h->fp8 ? 1 : 0) + (h->fp8pv ? 1 : 0));   // bf16 K, V (+ E4M3)
     }
   }
   bytes += h->targets.size() * ((size_t)h->ring_slots * h->n * sizeof(float) + h->kmax * sizeof(int));

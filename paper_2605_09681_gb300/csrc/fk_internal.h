@@ -117,7 +117,8 @@ struct CurrentArgs {
   bf16* viewV[kMaxHeads];
   bf16* pageK[kMaxHeads];       // page rings (nullptr: head keeps no history pages)
   bf16* pageV[kMaxHeads];
-  uint8_t* viewK8[kMaxHeads];   // FP8_QK: E4M3 copies of the K views, same rows (else nullptr)
+  uint8_t* viewK8[kMaxHeads];   // FP8 attention: E4M3 copies of the K views, same rows (else nullptr)
+  uint8_t* viewV8[kMaxHeads];   // FP8 P V: E4M3 copies of the V views (else nullptr)
   unsigned char is_static[kMaxHeads];   // static: sink / anchor slots live in the view
   // in-kernel scoring of the retired chunk (requires retire; every retired frame and the frame
   // before the chunk are non-sink window frames, and C <= kFuseMaxFrames)
@@ -140,7 +141,8 @@ struct ScatterArgs {            // token-major [rows][H][D] -> per-head row-majo
   int head_dim;
   bf16* dstK[kMaxHeads];        // nullptr = skip this head
   bf16* dstV[kMaxHeads];
-  uint8_t* dstK8[kMaxHeads];    // FP8_QK view rows: E4M3 copy of dstK (else nullptr)
+  uint8_t* dstK8[kMaxHeads];    // FP8 attention view rows: E4M3 copy of dstK (else nullptr)
+  uint8_t* dstV8[kMaxHeads];    // FP8 P V view rows: E4M3 copy of dstV (else nullptr)
 };
 void launch_scatter(const ScatterArgs& a, cudaStream_t s);
 
@@ -212,7 +214,8 @@ struct CompactItem {            // one dynamic (layer, head)
   bf16* viewV;
   int layer;
   int target;                   // kept list
-  uint8_t* viewK8;              // FP8_QK: E4M3 copy of the K view, same rows (else nullptr)
+  uint8_t* viewK8;              // FP8 attention: E4M3 copy of the K view, same rows (else nullptr)
+  uint8_t* viewV8;              // FP8 P V: E4M3 copy of the V view (else nullptr)
 };
 
 struct CompactArgs {
@@ -253,10 +256,11 @@ struct AttnArgs {
   int n_keys[kMaxHeads];        // keys the head attends to
 };
 // tmQ: 3D map over Q [Nq][H][D]; tmK/tmV: 2D maps over the view arenas [rows][D].
-// fp8: Q K^T on E4M3 operands (head_dim 128): tmK then maps the E4M3 key arena (box 128 x 128,
-// one 128-byte swizzle atom per row); tmQ still maps the bf16 queries, which the kernel
-// quantizes itself.
-void launch_attention(int head_dim, bool fp8, const CUtensorMap& tmQ, const CUtensorMap& tmK,
+// precision FK_ATTN_FP8_QK: Q K^T on E4M3 operands (head_dim 128): tmK then maps the E4M3 key
+// arena (box 128 x 128, one 128-byte swizzle atom per row); tmQ still maps the bf16 queries,
+// which the kernel quantizes itself.  FK_ATTN_FP8: P V on E4M3 operands too: tmV maps the
+// E4M3 value arena the same way.
+void launch_attention(int head_dim, int precision, const CUtensorMap& tmQ, const CUtensorMap& tmK,
                       const CUtensorMap& tmV, const AttnArgs& a, cudaStream_t s);
 cudaError_t attention_prepare(int head_dim);   // sets the dynamic shared-memory limits
 // combine the key splits of every (row, head) into O (bf16)

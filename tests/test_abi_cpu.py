@@ -63,7 +63,8 @@ def test_abi_version(lib):
     dict(score_source=5), dict(incremental=2), dict(window_frames=-1), dict(n_sink_frames=-1),
     dict(window_frames=0, max_history_frames=0), dict(selection=4), dict(selection=-1),
     dict(selection=2, select_scope=1, n_segments=1), dict(static_drop_anchor=2),
-    dict(attn_precision=2), dict(attn_precision=-1), dict(attn_precision=1, head_dim=64),
+    dict(attn_precision=3), dict(attn_precision=-1), dict(attn_precision=1, head_dim=64),
+    dict(attn_precision=2, head_dim=64),
 ])
 def test_validate_rejects_bad_configs(lib, bad):
     c, _keep = _cfg(**bad)
@@ -79,7 +80,7 @@ def test_validate_accepts_paper_configs(lib):
                dict(selection=1, n_sink_frames=3, window_frames=4),
                dict(selection=1, window_frames=2, static_drop_anchor=1),
                dict(selection=2, n_segments=60), dict(selection=3, select_seed=7, n_segments=60),
-               dict(attn_precision=1, head_dim=128)]:
+               dict(attn_precision=1, head_dim=128), dict(attn_precision=2, head_dim=128)]:
         c, _keep = _cfg(**kw)
         assert lib.fk_validate_config(ctypes.byref(c)) == 0, kw
 
@@ -198,3 +199,14 @@ def test_noalloc_rejects_bad_arguments_on_the_host(lib):
     assert f(K, 1, 64, 128, 8, S, None, None) == 1
     assert f(K, 256, 64, 128, 32, S, None, None) == 1             # frames x segments
     assert f(K, 4, 60, 128, 8, S, None, None) == 1                # segments must divide F
+
+
+def test_stream_read_rejects_bad_arguments_on_the_host(lib):
+    # null, misaligned or non-multiple-of-16 requests are refused before any CUDA call; zero
+    # bytes is a no-op
+    f = lib.fk_stream_read
+    assert f(None, 64, None) == 2
+    assert f(1 << 20 | 8, 64, None) == 2
+    assert f(1 << 20, 60, None) == 2
+    assert f(1 << 20, 0, None) == 0
+

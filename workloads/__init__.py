@@ -31,7 +31,7 @@ __all__ = [
     "Workload", "TINY", "TINY_PER_FRAME", "P480_LAYER", "P480_STACK", "ROLLING",
     "P1080_LAYER", "WORKLOADS", "normals", "uniforms", "to_bf16_bits", "bf16_bits_to_f32",
     "profile_inputs", "FULL_KV_480P", "STREAMINGLLM_480P", "DUMMY_FORCING_480P", "UNIFORM_TOKENS_480P",
-    "RANDOM_TOKENS_480P",
+    "RANDOM_TOKENS_480P", "P480_LAYER_FP8PV", "P1080_LAYER_FP8PV", "TINY_FP8PV",
     "head_map", "FrameStream", "snapshot_inputs", "queries", "step_kv", "stream_key",
 ]
 
@@ -132,7 +132,7 @@ class Workload:
     selection: str = "similarity"        # "similarity" | "all" | "uniform" | "random"
     select_seed: int = 0
     static_drop_anchor: bool = False
-    attn_precision: str = "bf16"         # "bf16" | "fp8_qk" (Q K^T on e4m3 operands)
+    attn_precision: str = "bf16"         # "bf16" | "fp8_qk" (Q K^T on e4m3 operands) | "fp8" (P V too)
     seed: int = 0
     description: str = ""
 
@@ -235,11 +235,22 @@ P1080_LAYER_FP8 = P1080_LAYER.with_(
 TINY_FP8 = TINY_PER_FRAME.with_(
     name="tiny_fp8", head_dim=128, attn_precision="fp8_qk",
     description="tiny per-frame case at head_dim 128 with Q K^T on FP8 E4M3 operands")
+# both products on e4m3 operands (P scaled by 2^6 relative to the running row max, V unscaled)
+P480_LAYER_FP8PV = P480_LAYER.with_(
+    name="480p_layer_fp8pv", attn_precision="fp8",
+    description="the 480P layer with Q K^T and P V on FP8 E4M3 operands")
+P1080_LAYER_FP8PV = P1080_LAYER.with_(
+    name="1080p_layer_fp8pv", attn_precision="fp8",
+    description="the 1080P layer with Q K^T and P V on FP8 E4M3 operands")
+TINY_FP8PV = TINY_PER_FRAME.with_(
+    name="tiny_fp8pv", head_dim=128, attn_precision="fp8",
+    description="tiny per-frame case at head_dim 128 with both products on FP8 E4M3 operands")
 
 WORKLOADS = {w.name: w for w in (TINY, TINY_PER_FRAME, P480_LAYER, P480_STACK, ROLLING, P1080_LAYER,
                                  FULL_KV_480P, STREAMINGLLM_480P, DUMMY_FORCING_480P,
                                  UNIFORM_TOKENS_480P, RANDOM_TOKENS_480P, P480_LAYER_FP8,
-                                 P1080_LAYER_FP8, TINY_FP8)}
+                                 P1080_LAYER_FP8, TINY_FP8, P480_LAYER_FP8PV, P1080_LAYER_FP8PV,
+                                 TINY_FP8PV)}
 
 
 def head_map(w: Workload) -> np.ndarray:
