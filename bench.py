@@ -36,6 +36,7 @@ sys.path.insert(0, ROOT)
 METRIC = "compressed chunk-attention TFLOP/s + compaction GB/s (% roofline); attn frames/s"
 DIT_LAYERS, DENOISE_STEPS = 30, 4      # attention calls per generated chunk in the 30-block, 4-step DiT
 L2_FLUSH_BYTES = 512 << 20
+E2E_MIN_STEPS = 100                    # end-to-end steps timed in one interval (at least)
 
 
 def _peaks():
@@ -312,9 +313,10 @@ def measure_layer(args, w, hm, inp, flush, stream, world, local_rank, peaks, cal
         step(i, host=True)
     torch.cuda.synchronize()
     barrier(world)
+    e2e_steps = max(args.steps, E2E_MIN_STEPS)
     e_begin, e_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e_begin.record(stream)
-    for i in range(args.steps):
+    for i in range(e2e_steps):
         step(i, host=True)
     cache.wait_outputs()                 # every step's output copy-back inside the interval
     e_end.record(stream)
@@ -343,12 +345,13 @@ def measure_layer(args, w, hm, inp, flush, stream, world, local_rank, peaks, cal
         "keys": keys, "alg": alg, "prof": prof, "launches": int(launches),
         "ms_step": total_ms / args.steps,
         "value": world * alg["attn_flops"] * args.steps / (total_ms * 1e-3) / 1e12,
-        "e2e": {"value": round(world * alg["attn_flops"] * args.steps / (e2e_ms * 1e-3) / 1e12, 3),
-                "unit": "TFLOP/s", "ms_per_step": round(e2e_ms / args.steps, 4),
+        "e2e": {"value": round(world * alg["attn_flops"] * e2e_steps / (e2e_ms * 1e-3) / 1e12, 3),
+                "unit": "TFLOP/s", "ms_per_step": round(e2e_ms / e2e_steps, 4), "steps": e2e_steps,
                 "h2d_bytes_per_step": 3 * nbytes, "d2h_bytes_per_step": nbytes,
                 "note": "pinned host K, V, Q in and O out every step through the C ABI; host copies "
                         "overlap queued work (fk_set_host_overlap, outputs joined by fk_wait_outputs "
-                        "before the end event); one continuous interval over all steps",
+                        "before the end event); one continuous interval over all steps (at least "
+                        "%d, so that one slow host interval does not dominate)" % E2E_MIN_STEPS,
                 "l2": "not flushed between steps (each step touches more inputs, views and pages than "
                       "the L2 holds); the device-timed value flushes before every step"},
         "roofline": {
@@ -373,6 +376,7 @@ def measure_layer(args, w, hm, inp, flush, stream, world, local_rank, peaks, cal
                        "peak": peaks["hbm_gbs"], "unit": "GB/s",
                        "frac": round(alg["append_bytes"] / (per_launch("append") * 1e-3) / 1e9 / peaks["hbm_gbs"], 4),
                        "bytes": alg["append_bytes"], "us": round(per_launch("append") * 1e3, 2),
+                       "traffic": traffic.get("append"),
                        "scores_retired_chunk": alg["score_fused"]},
             "peak_source": peaks["source"] + " HBM copy bandwidth",
             "traffic_source": TRAFFIC_SOURCE if traffic else None,
@@ -624,7 +628,7 @@ def run_fp8(args, w, hm, local_rank, hk, hv, dK, dV, dQ, dO, flush, stream, worl
     # half the flops run at each rate (peak 4/3 of the measured bf16 peak), with both products
     # on E4M3 all of them (peak 2x)
     mixed_peak = peaks["bf16_tflops"] * (2.0 if precision == "fp8" else 4.0 / 3.0)
-    traffic = _traffic("480p_layer") if w.name == "480p_layer" and precision == "fp8_qk" else {}
+    traffic = _traffic("480p_layer") if w.name == "480p_layer" else {}
     per_step = lambda p, k: round(p[k][0] / args.steps * 1e3, 2)
     return {
         "workload": w.name + " (%s)" % precision,
@@ -639,7 +643,7 @@ def run_fp8(args, w, hm, local_rank, hk, hv, dK, dV, dQ, dO, flush, stream, worl
                                      % ("2" if precision == "fp8" else "4/3"),
                       "frac": round(attn_tflops / mixed_peak, 4),
                       "speedup_vs_bf16_kernel": round(bf16_attn_ms / attn_ms, 3),
-                      "traffic": traffic.get("attend_fp8")},
+                      "traffic": traffic.get("attend_fp8" if precision == "fp8_qk" else "attend_fp8pv")},
         "e4m3_key_writes_us_per_step": round(per_step(prof, "append") + per_step(prof, "compact")
                                              - per_step(bf16_prof, "append") - per_step(bf16_prof, "compact"), 2),
         "note": "same algorithmic FLOPs as the bf16 step; Q K^T on E4M3 (kind::f8f6f4)%s; E4M3 copies "
@@ -757,16 +761,18 @@ def run_stack(local_rank, attn_precision="bf16"):
 # is reported only while that source is unchanged.
 NCU_TRAFFIC = {
     "480p_layer": {
-        "attend": ("fk_attn.cu", "da6b58031078", 119412117),
-        "attend_fp8": ("fk_attn.cu", "da6b58031078", 92557994),
-        "compact": ("fk_copy.cu", "e373e101c0f6", 73879072),
-        "score": ("fk_score.cu", "8a76e34bff85", 43158016),
+        "attend": ("fk_attn.cu", "99a3095cd302", 118640000),
+        "attend_fp8": ("fk_attn.cu", "99a3095cd302", 91760000),
+        "attend_fp8pv": ("fk_attn.cu", "99a3095cd302", 65810000),
+        "append": ("fk_copy.cu", "2690c64c569f", 54140000),
+        "compact": ("fk_copy.cu", "2690c64c569f", 58300000),
+        "score": ("fk_score.cu", "c31614e0df7f", 35970000),
     },
 }
 
 
-TRAFFIC_SOURCE = ("stored DRAM bytes per launch from an earlier ncu capture of the same kernel "
-                  "source (profiles/hbm_kernels_480p_layer.md, profiles/attn_kernel_480p_layer.md); "
+TRAFFIC_SOURCE = ("stored DRAM bytes per launch (read + write, median over the launches) from an "
+                  "earlier ncu capture of the same kernel source (profiles/launches_480p_layer.md); "
                   "reported only while the source hash matches, not observed in this run")
 
 
