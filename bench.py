@@ -129,6 +129,8 @@ class Clocks:
         self.index, self.proc = index, None
 
     def __enter__(self):
+        import threading
+        self.lines = []
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.FIELDS,
@@ -136,6 +138,15 @@ class Clocks:
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
         except OSError:
             self.proc = None
+        if self.proc:
+            # collect samples in a thread; the timed region starts only once the sampler has
+            # produced its first sample (its start-up can stall launches on a fresh box)
+            self.reader = threading.Thread(target=lambda: self.lines.extend(iter(self.proc.stdout.readline, "")),
+                                           daemon=True)
+            self.reader.start()
+            t0 = time.time()
+            while not self.lines and time.time() - t0 < 15.0 and self.proc.poll() is None:
+                time.sleep(0.05)
         time.sleep(0.3)
         return self
 
@@ -145,9 +156,11 @@ class Clocks:
             time.sleep(0.2)
             self.proc.terminate()
             try:
-                self.out, _ = self.proc.communicate(timeout=5)
+                self.proc.wait(timeout=5)
             except subprocess.TimeoutExpired:
                 self.proc.kill()
+            self.reader.join(timeout=5)
+            self.out = "".join(self.lines)
 
     def summary(self):
         sm, mx, reasons = [], [], set()
