@@ -570,6 +570,76 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
         uint32_t sv[64];
         FK_TMEM_LD64(tS + half * 64, sv);
         tmem_wait_ld();
+        if constexpr (!kFp8PV) {
+          // Full tile after the first (every row has a finite running max m): P = exp2(S*c - m)
+          // straight away; m has to move only if some P exceeds 2^8 (an element more than 8
+          // above m), which the packed bf16 maximum of the half's P shows.  Otherwise the
+          // half is done without a separate max pass; if it does, the path below redoes it.
+          if (full && j > 0) {
+            uint32_t pk[32];
+            float2 ah[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) ah[i] = make_float2(0.0f, 0.0f);
+            const float2 nm2 = make_float2(-m, -m);
+#pragma unroll
+            for (int q = 0; q < 32; ++q) {
+              const float2 x = ffma2(make_float2(__uint_as_float(sv[2 * q]), __uint_as_float(sv[2 * q + 1])),
+                                     sc2, nm2);
+              float2 e;
+              e.x = fast_exp2(x.x);
+              e.y = fast_exp2(x.y);
+              ah[q & 3] = fadd2(ah[q & 3], e);
+              pk[q] = pack_bf16(e.x, e.y);
+            }
+            __nv_bfloat162 pm[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) pm[i] = *reinterpret_cast<const __nv_bfloat162*>(&pk[i]);
+#pragma unroll
+            for (int q = 4; q < 32; ++q)
+              pm[q & 3] = __hmax2(pm[q & 3], *reinterpret_cast<const __nv_bfloat162*>(&pk[q]));
+            const __nv_bfloat162 p2 = __hmax2(__hmax2(pm[0], pm[1]), __hmax2(pm[2], pm[3]));
+            const float pmax = fmaxf(__low2float(p2), __high2float(p2));
+            if (!__any_sync(0xffffffffu, pmax > 256.0f)) {               // warp-uniform
+#pragma unroll
+              for (int i = 0; i < 4; ++i) acc[i] = fadd2(acc[i], ah[i]);
+              FK_TMEM_ST32(tS + half * 32, pk);
+              continue;
+            }
+          }
+        } else {
+          // FP8 P V, the same idea with the integer reference: a numerator above 2^8 (y more than
+          // 2 above m) shows as an e4m3 code above 0x78; codes are non-negative and at most 0x7E,
+          // so adding 7 to each byte sets its top bit exactly then, without carries between bytes
+          if (full && j > 0) {
+            uint32_t pk[16], ov = 0;
+            float2 ah[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) ah[i] = make_float2(0.0f, 0.0f);
+            const float2 nm2 = make_float2(kPShift - m, kPShift - m);
+#pragma unroll
+            for (int q = 0; q < 16; ++q) {
+              const float2 x0 = ffma2(make_float2(__uint_as_float(sv[4 * q]), __uint_as_float(sv[4 * q + 1])),
+                                      sc2, nm2);
+              const float2 x1 = ffma2(make_float2(__uint_as_float(sv[4 * q + 2]), __uint_as_float(sv[4 * q + 3])),
+                                      sc2, nm2);
+              float2 e0, e1;
+              e0.x = fast_exp2(x0.x);
+              e0.y = fast_exp2(x0.y);
+              e1.x = fast_exp2(x1.x);
+              e1.y = fast_exp2(x1.y);
+              ah[(2 * q) & 3] = fadd2(ah[(2 * q) & 3], e0);
+              ah[(2 * q + 1) & 3] = fadd2(ah[(2 * q + 1) & 3], e1);
+              pk[q] = e4m3x2(e0.x, e0.y) | (e4m3x2(e1.x, e1.y) << 16);
+              ov |= pk[q] + 0x07070707u;
+            }
+            if (!__any_sync(0xffffffffu, (ov & 0x80808080u) != 0)) {   // warp-uniform
+#pragma unroll
+              for (int i = 0; i < 4; ++i) acc[i] = fadd2(acc[i], ah[i]);
+              FK_TMEM_ST16(tS + half * 16, pk);
+              continue;
+            }
+          }
+        }
         float mxa[8];
 #pragma unroll
         for (int i = 0; i < 8; ++i) mxa[i] = -INFINITY;
