@@ -591,15 +591,20 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
               ah[q & 3] = fadd2(ah[q & 3], e);
               pk[q] = pack_bf16(e.x, e.y);
             }
-            __nv_bfloat162 pm[4];
+            // the half's sum bounds each of its numerators: only a sum above 2^8 needs the max
+            const float2 hs2 = fadd2(fadd2(ah[0], ah[1]), fadd2(ah[2], ah[3]));
+            bool over = false;
+            if (__any_sync(0xffffffffu, hs2.x + hs2.y > 256.0f)) {
+              __nv_bfloat162 pm[4];
 #pragma unroll
-            for (int i = 0; i < 4; ++i) pm[i] = *reinterpret_cast<const __nv_bfloat162*>(&pk[i]);
+              for (int i = 0; i < 4; ++i) pm[i] = *reinterpret_cast<const __nv_bfloat162*>(&pk[i]);
 #pragma unroll
-            for (int q = 4; q < 32; ++q)
-              pm[q & 3] = __hmax2(pm[q & 3], *reinterpret_cast<const __nv_bfloat162*>(&pk[q]));
-            const __nv_bfloat162 p2 = __hmax2(__hmax2(pm[0], pm[1]), __hmax2(pm[2], pm[3]));
-            const float pmax = fmaxf(__low2float(p2), __high2float(p2));
-            if (!__any_sync(0xffffffffu, pmax > 256.0f)) {               // warp-uniform
+              for (int q = 4; q < 32; ++q)
+                pm[q & 3] = __hmax2(pm[q & 3], *reinterpret_cast<const __nv_bfloat162*>(&pk[q]));
+              const __nv_bfloat162 p2 = __hmax2(__hmax2(pm[0], pm[1]), __hmax2(pm[2], pm[3]));
+              over = fmaxf(__low2float(p2), __high2float(p2)) > 256.0f;
+            }
+            if (!__any_sync(0xffffffffu, over)) {                          // warp-uniform
 #pragma unroll
               for (int i = 0; i < 4; ++i) acc[i] = fadd2(acc[i], ah[i]);
               FK_TMEM_ST32(tS + half * 32, pk);
