@@ -774,9 +774,9 @@ def run_stack(local_rank, attn_precision="bf16"):
 # is reported only while that source is unchanged.
 NCU_TRAFFIC = {
     "480p_layer": {
-        "attend": ("fk_attn.cu", "99a3095cd302", 118640000),
-        "attend_fp8": ("fk_attn.cu", "99a3095cd302", 91760000),
-        "attend_fp8pv": ("fk_attn.cu", "99a3095cd302", 65810000),
+        "attend": ("fk_attn.cu", "74c0df6bf474", 118470000),
+        "attend_fp8": ("fk_attn.cu", "74c0df6bf474", 91820000),
+        "attend_fp8pv": ("fk_attn.cu", "74c0df6bf474", 65810000),
         "append": ("fk_copy.cu", "2690c64c569f", 54140000),
         "compact": ("fk_copy.cu", "2690c64c569f", 58300000),
         "score": ("fk_score.cu", "c31614e0df7f", 35970000),
