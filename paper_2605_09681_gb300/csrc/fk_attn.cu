@@ -482,15 +482,14 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
       for (int j = 0; j < nt && ok; ++j) {
         const int st = j & 1;
         const bool more = j + 1 < nt;
-        if (!wait_phase(&bar->p_full[0], j & 1, bar, a.status) ||
-            !wait_phase(&bar->v_full[st], (j >> 1) & 1, bar, a.status)) { ok = false; break; }
+        // V_j and K_{j+1} are waited for before P_0(j): neither depends on the softmax, and
+        // PV0(j), S0(j+1) then go to the tensor pipe back to back once P_0(j) is in TMEM
+        if (!wait_phase(&bar->v_full[st], (j >> 1) & 1, bar, a.status) ||
+            (more && !wait_phase(&bar->k_full[(j + 1) & 1], ((j + 1) >> 1) & 1, bar, a.status)) ||
+            !wait_phase(&bar->p_full[0], j & 1, bar, a.status)) { ok = false; break; }
         tc_fence_after();
         pv(j, 0);
-        if (more) {
-          if (!wait_phase(&bar->k_full[(j + 1) & 1], ((j + 1) >> 1) & 1, bar, a.status)) { ok = false; break; }
-          tc_fence_after();
-          qk(j + 1, 0);
-        }
+        if (more) qk(j + 1, 0);
         if (!wait_phase(&bar->p_full[1], j & 1, bar, a.status)) { ok = false; break; }
         tc_fence_after();
         pv(j, 1);
@@ -960,10 +959,43 @@ profile_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
           if (lane == 0) mbar_arrive(&bar->p_full[st]);
         }
         if (valid <= 0) continue;
-        float mx = -INFINITY;
+        // key classes are contiguous ranges in the order generated, sink, other, transition
+        const int last = kb + valid - 1;
+        const int cls_first = kb < a.g_end ? 0 : kb < a.s_end ? 1 : kb >= a.t_begin ? 3 : 2;
+        const int cls_last = last < a.g_end ? 0 : last < a.s_end ? 1 : last >= a.t_begin ? 3 : 2;
+        // A full half of one key class after the first half (every row then has a finite
+        // running max m): the exponentials with m straight away.  The half's sum bounds each
+        // term, so only a sum above 2^8 (possibly a key more than 8 above m in log2 units)
+        // needs the max pass and lazy rescale below, which then redoes the half.
+        if (valid == 64 && cls_first == cls_last && (j > 0 || half > 0)) {   // CTA-uniform
+          const float2 sc2 = make_float2(a.scale_log2, a.scale_log2), nm2 = make_float2(-m, -m);
+          float2 a2[4];
+#pragma unroll
+          for (int i = 0; i < 4; ++i) a2[i] = make_float2(0.0f, 0.0f);
+#pragma unroll
+          for (int q = 0; q < 32; ++q) {
+            const float2 x = ffma2(make_float2(__uint_as_float(sv[2 * q]), __uint_as_float(sv[2 * q + 1])),
+                                   sc2, nm2);
+            a2[q & 3] = fadd2(a2[q & 3], make_float2(fast_exp2(x.x), fast_exp2(x.y)));
+          }
+          const float2 s2 = fadd2(fadd2(a2[0], a2[1]), fadd2(a2[2], a2[3]));
+          const float sum = s2.x + s2.y;
+          if (!__any_sync(0xffffffffu, sum > 256.0f)) {                  // warp-uniform
+            l += sum;
+            if (cls_first == 0) cg += sum;
+            else if (cls_first == 1) cs += sum;
+            else if (cls_first == 3) ct += sum;
+            continue;
+          }
+        }
+        float mxa[8];                                // eight independent max chains
+#pragma unroll
+        for (int i = 0; i < 8; ++i) mxa[i] = -INFINITY;
 #pragma unroll
         for (int c = 0; c < 64; ++c)
-          if (c < valid) mx = fmaxf(mx, __uint_as_float(sv[c]));
+          if (c < valid) mxa[c & 7] = fmaxf(mxa[c & 7], __uint_as_float(sv[c]));
+        const float mx = fmaxf(fmaxf(fmaxf(mxa[0], mxa[1]), fmaxf(mxa[2], mxa[3])),
+                               fmaxf(fmaxf(mxa[4], mxa[5]), fmaxf(mxa[6], mxa[7])));
         const float m_new = fmaxf(m, mx * a.scale_log2);
         if (__any_sync(0xffffffffu, m_new > m + kRescaleThreshold)) {   // warp-uniform
           const float alpha = fast_exp2(m - m_new);  // 0 when m = -inf
@@ -973,10 +1005,6 @@ profile_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
           ct *= alpha;
           m = m_new;
         }
-        // key classes are contiguous ranges in the order generated, sink, other, transition
-        const int last = kb + valid - 1;
-        const int cls_first = kb < a.g_end ? 0 : kb < a.s_end ? 1 : kb >= a.t_begin ? 3 : 2;
-        const int cls_last = last < a.g_end ? 0 : last < a.s_end ? 1 : last >= a.t_begin ? 3 : 2;
         if (cls_first == cls_last) {
           float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll
