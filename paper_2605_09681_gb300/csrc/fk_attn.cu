@@ -827,7 +827,11 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
 // [generated | sink | other history | transition].  S = Q K^T runs on the tensor cores
 // (tcgen05, S double-buffered in 256 TMEM columns); no P V product is needed.  Per row the
 // softmax statistics are kept online (running max, total sum, and the three class sums,
-// rescaled together); the per-row fractions are summed per head in double.
+// rescaled together); the per-row fractions are summed per head in double.  A cluster of two
+// CTAs handles one (head, 128-row query tile), each CTA half of the key tiles (so the grid
+// fills the SMs in about three even waves instead of two, the second half empty); the
+// second CTA writes its row statistics into the first's shared memory (distributed shared
+// memory, one cluster barrier), and the first merges the two ranges.
 //   warps 0-3  statistics of rows 0..127 (TMEM lanes), one thread per row;
 //   warp 4     TMA: the query tile once, key tiles into a two-stage ring;
 //   warp 5     tcgen05.mma: S_b = Q K_j^T for b = j mod 2, once the statistics warps have
@@ -843,11 +847,12 @@ struct ProfLayout {
   static constexpr int kOffQ = 0;
   static constexpr int kOffK = kOffQ + kQ;
   static constexpr int kOffBar = kOffK + 2 * kK;
-  static constexpr int kSmem = kOffBar + 256 + 1024;   // + alignment slack; two CTAs per SM
+  static constexpr int kOffPart = kOffBar + 256;      // the cluster peer's row statistics
+  static constexpr int kSmem = kOffPart + kAttnBM * 8 * 4 + 1024;   // + alignment slack; two CTAs per SM
 };
 
 template <int D>
-__global__ void __launch_bounds__(kProfThreads, 2)
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kProfThreads, 2)
 profile_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                const ProfArgs a) {
   using Lay = ProfLayout<D>;
@@ -862,11 +867,24 @@ profile_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
   // barrier use: q_full, k_full/k_empty (key ring), s_full[b] (S_b written), p_full[b]
   // (S_b read by the four statistics warps), fin
 
+  float* part = reinterpret_cast<float*>(smem + Lay::kOffPart);   // [row][8]: m l cg cs ct ok
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int head = blockIdx.x / a.n_qtiles;
-  const int q0 = (blockIdx.x - head * a.n_qtiles) * kAttnBM;
+  const int row = warp * 32 + lane;                 // query row of a statistics thread
+  // A cluster of two CTAs = one (head, query tile); CTA r of the cluster takes key tiles
+  // [j0, j0 + nt) of the head's window (r = 0 the first half, r = 1 the rest).
+  uint32_t rank;
+  asm("mov.u32 %0, %%cluster_ctarank;" : "=r"(rank));
+  const int pair = blockIdx.x >> 1;
+  const int head = pair / a.n_qtiles;
+  const int q0 = (pair - head * a.n_qtiles) * kAttnBM;
   const int nk = a.Nk;
-  const int nt = (nk + kAttnBN - 1) / kAttnBN;
+  const int nt_all = (nk + kAttnBN - 1) / kAttnBN;
+  const int j0 = rank ? nt_all / 2 : 0;
+  const int nt = rank ? nt_all - nt_all / 2 : nt_all / 2;   // may be 0 (one key tile in all)
+  // row statistics of this CTA's keys (statistics warps): running max (log2 domain), total
+  // sum and the class sums, all relative to m
+  float m = -INFINITY, l = 0.0f, cg = 0.0f, cs = 0.0f, ct = 0.0f;
+  bool ok = true;
 
   if (threadIdx.x == 0) {
     mbar_init(&bar->q_full, 1);
@@ -903,7 +921,7 @@ profile_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         mbar_expect_tx(&bar->k_full[st], Lay::kK);
         for (int h = 0; h < kHalves; ++h)
           tma_load_3d(sK + st * Lay::kK + h * 16384, &tmK, &bar->k_full[st], h * 64, head,
-                      j * kAttnBN);
+                      (j0 + j) * kAttnBN);
         lastK[st] = u;
       }
       if (!ok) {   // drain every load this thread issued before the CTA exits
@@ -938,17 +956,14 @@ profile_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
     __syncwarp();
   } else {
     const int wq = warp;
-    const int row = wq * 32 + lane;
     const uint32_t lane_base = (uint32_t)(wq * 32) << 16;
-    float m = -INFINITY, l = 0.0f, cg = 0.0f, cs = 0.0f, ct = 0.0f;
-    bool ok = true;
     for (int j = 0; j < nt; ++j) {
       const int st = j & 1;
       if (!warp_wait(&bar->s_full[st], (j >> 1) & 1, bar, a.status)) { ok = false; break; }
       tc_fence_after();
 #pragma unroll
       for (int half = 0; half < 2; ++half) {
-        const int kb = j * kAttnBN + half * 64;      // first key of this half
+        const int kb = (j0 + j) * kAttnBN + half * 64;   // first key of this half
         const int valid = min(64, nk - kb);          // uniform over the CTA
         uint32_t sv[64];
         FK_TMEM_LD64(tmem + lane_base + (uint32_t)(st * kAttnBN + half * 64), sv);
@@ -1030,6 +1045,38 @@ profile_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
         }
       }
     }
+    if (rank == 1) {
+      // this CTA's row statistics go to the same row slot in the first CTA's shared memory
+      uint32_t dst;
+      asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(dst) : "r"(su32(part + row * 8)), "r"(0u));
+      asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" :: "r"(dst), "f"(m), "f"(l),
+                   "f"(cg), "f"(cs) : "memory");
+      asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" :: "r"(dst + 16u), "f"(ct),
+                   "f"(ok ? 1.0f : 0.0f) : "memory");
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == kWarpProfMma) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" :: "r"(tmem),
+                 "r"(kTmemCols) : "memory");
+  }
+  // every thread of both CTAs: the second CTA's statistics have landed (release / acquire)
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+  if (rank == 0 && warp < kWarpProfTma) {
+    // merge the two key ranges: with M = max(m0, m1), every sum s = s0 2^(m0 - M) + s1 2^(m1 - M)
+    const float* pp = part + row * 8;
+    const float pm = pp[0];
+    ok = ok && pp[5] != 0.0f;                       // warp-uniform: one warp of each CTA per row block
+    const float M = fmaxf(m, pm);
+    const float w0 = m == -INFINITY ? 0.0f : fast_exp2(m - M);
+    const float w1 = pm == -INFINITY ? 0.0f : fast_exp2(pm - M);
+    l = l * w0 + pp[1] * w1;
+    cg = cg * w0 + pp[2] * w1;
+    cs = cs * w0 + pp[3] * w1;
+    ct = ct * w0 + pp[4] * w1;
     if (ok) {
       const bool in = q0 + row < a.Nq;
       float fg = in ? cg / l : 0.0f, fs = in ? cs / l : 0.0f, ft = in ? ct / l : 0.0f;
@@ -1050,21 +1097,13 @@ profile_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ 
       }
     }
   }
-
-  tc_fence_before();
-  __syncthreads();
-  if (warp == kWarpProfMma) {
-    tc_fence_after();
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" :: "r"(tmem),
-                 "r"(kTmemCols) : "memory");
-  }
 }
 
 }  // namespace
 
 cudaError_t launch_head_profile(int head_dim, const CUtensorMap& tmQ, const CUtensorMap& tmK,
                                 const ProfArgs& a, cudaStream_t s) {
-  const unsigned grid = (unsigned)(a.n_qtiles * a.H);
+  const unsigned grid = (unsigned)(2 * a.n_qtiles * a.H);   // clusters of two CTAs
   cudaError_t e;
   if (head_dim == 128) {
     e = cudaFuncSetAttribute(profile_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,

@@ -545,7 +545,7 @@ fk_status fk_head_profile(const void* Q, const void* K, int n_queries, int n_key
       (int64_t)n_generate + n_sink + n_transition > n_keys)
     return FK_ERR_CONFIG;
   const int64_t n_qtiles = (n_queries + kAttnBM - 1) / kAttnBM;
-  if (n_qtiles * n_heads >= ((int64_t)1 << 31)) return FK_ERR_CONFIG;
+  if (2 * n_qtiles * n_heads >= ((int64_t)1 << 31)) return FK_ERR_CONFIG;
   if (!is_device_ptr(Q) || !is_device_ptr(K) || !is_device_ptr(mass) || !is_device_ptr(status))
     return FK_ERR_ARG;
   if (!get_encode()) return FK_ERR_CUDA;

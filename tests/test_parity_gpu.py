@@ -284,10 +284,12 @@ def test_480p_stack_full():
     assert run_stream(w, track_layers=(0, 13, 29), compare_every=3, step_filter=(0, 3)) > 0
 
 
-@pytest.mark.parametrize("head_dim,F,hist", [(128, 260, 8), (64, 100, 5)])
+@pytest.mark.parametrize("head_dim,F,hist", [(128, 260, 8), (64, 100, 5), (128, 24, 2), (64, 40, 2)])
 def test_head_profile_matches_oracle(head_dim, F, hist):
     # Eq. 1 masses from the tcgen05 profiling kernel vs the fp64 oracle on the same bf16
     # inputs; 3-frame chunk, ragged query and key tiles, class boundaries inside key tiles.
+    # The two CTAs of a cluster split the key tiles: 27 (13 + 14), 8, a single tile (the
+    # first CTA has none) and two tiles (one each, the second ragged).
     # A second call adds to the same accumulator.
     from paper_2605_09681_gb300 import classify_heads, head_profile
     H = 8
