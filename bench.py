@@ -774,19 +774,20 @@ def run_stack(local_rank, attn_precision="bf16"):
 # is reported only while that source is unchanged.
 NCU_TRAFFIC = {
     "480p_layer": {
-        "attend": ("fk_attn.cu", "74c0df6bf474", 118470000),
-        "attend_fp8": ("fk_attn.cu", "74c0df6bf474", 91820000),
-        "attend_fp8pv": ("fk_attn.cu", "74c0df6bf474", 65810000),
-        "append": ("fk_copy.cu", "2690c64c569f", 54140000),
-        "compact": ("fk_copy.cu", "2690c64c569f", 58300000),
+        "attend": ("fk_attn.cu", "45283c8250ca", 118870000),
+        "attend_fp8": ("fk_attn.cu", "45283c8250ca", 91970000),
+        "attend_fp8pv": ("fk_attn.cu", "45283c8250ca", 65860000),
+        "append": ("fk_copy.cu", "2690c64c569f", 53940000),
+        "compact": ("fk_copy.cu", "2690c64c569f", 58110000),
         "score": ("fk_score.cu", "c31614e0df7f", 35970000),
     },
 }
 
 
-TRAFFIC_SOURCE = ("stored DRAM bytes per launch (read + write, median over the launches) from an "
-                  "earlier ncu capture of the same kernel source (profiles/launches_480p_layer.md); "
-                  "reported only while the source hash matches, not observed in this run")
+TRAFFIC_SOURCE = ("stored DRAM bytes per launch (read + write, median of three launches) from an "
+                  "earlier ncu capture of the same kernel source, one kernel per capture "
+                  "(profiles/launches_480p_layer.md); reported only while the source hash matches, "
+                  "not observed in this run")
 
 
 def _traffic(workload):
