@@ -456,6 +456,8 @@ def run_fk(args, rank, world, local_rank):
                              inp["dQ"], inp["dO"], flush, stream, world, peaks, prof, precision="fp8")
     if args.workload == "480p_layer":
         out["compress_30_layers"] = run_compress_layers(args, w, hm, local_rank, inp, flush, stream, peaks)
+        out["compress_30_layers_incremental"] = run_compress_layers(args, w, hm, local_rank, inp, flush,
+                                                                    stream, peaks, incremental=True)
     del inp
     if not args.no_1080p and args.workload == "480p_layer":
         out["p1080"] = run_1080p(args, world, local_rank, flush, stream, peaks, calib)
@@ -501,20 +503,23 @@ def run_1080p(args, world, local_rank, flush, stream, peaks, calib=None):
     }
 
 
-def run_compress_layers(args, w, hm, local_rank, inp, flush, stream, peaks, n_layers=30):
+def run_compress_layers(args, w, hm, local_rank, inp, flush, stream, peaks, n_layers=30,
+                        incremental=False):
     """Compression of a whole model: the 480P layer workload (per-head scoring, whole-window
     rescoring, full rebuild) in each of n_layers layers with the same head map, every layer
     appended with its chunk, then one fk_compress whose scoring, selection and compaction
     launches cover all layers at once (n_layers x 35.9 MB of keys scored, n_layers x 108.6 MB of
     kept K/V gathered).  Per-kernel event times (L2 flushed before each step) give those
     kernels' HBM fractions at the size of one model step's compression, where the launch and
-    first-access latency that bounds a single layer's 36 MB scoring launch is amortised."""
+    first-access latency that bounds a single layer's 36 MB scoring launch is amortised.  With
+    incremental set, the ring mode: the append kernels form the new pairs' sums (no scoring
+    launch) and the compaction copies only the newly decided segments (n_layers x 19.2 MB)."""
     import numpy as np
     import torch
 
     from paper_2605_09681_gb300 import ForcingKVCache
 
-    wl = w.with_(n_layers=n_layers)
+    wl = w.with_(n_layers=n_layers, incremental=incremental)
     hml = np.repeat(np.asarray(hm)[:1], n_layers, axis=0)
     n_pool = len(inp["dK"])
     cache = ForcingKVCache.from_workload(wl, hml, device=local_rank)
@@ -548,6 +553,12 @@ def run_compress_layers(args, w, hm, local_rank, inp, flush, stream, peaks, n_la
     reserved = cache.reserved_bytes()
     cache.close()
     alg = _algorithmic(w, keys)
+    if incremental:   # C x k new segments per dynamic head, K and V, read and written
+        D, F, C = w.head_dim, w.tokens_per_frame, w.frames_per_chunk
+        n_dyn = sum(1 for st in _workload_static(w) if not st)
+        k_frame = w.keep_budget_permille * w.n_segments // 1000
+        alg = dict(alg, score_bytes=0,
+                   compact_bytes=n_dyn * 2 * 2 * C * k_frame * (F // w.n_segments) * D * 2)
 
     def kern(kind, nbytes):
         ms, n = prof[kind]
@@ -560,15 +571,17 @@ def run_compress_layers(args, w, hm, local_rank, inp, flush, stream, peaks, n_la
 
     return {
         "layers": n_layers,
+        "mode": "incremental" if incremental else "whole-window rescoring, full rebuild",
         "score": kern("score", n_layers * alg["score_bytes"]),
         "compact": kern("compact", n_layers * alg["compact_bytes"]),
         "select_us": round(prof["select"][0] / max(1, prof["select"][1]) * 1e3, 2),
         "append_us_per_layer": round(prof["append"][0] / max(1, prof["append"][1]) * 1e3, 2),
         "compress_us": round((prof["score"][0] + prof["select"][0] + prof["compact"][0]) / args.steps * 1e3, 2),
         "reserved_gb": round(reserved / 1e9, 2),
-        "note": "one fk_compress over %d layers of the 480P layer workload (per-head scoring, "
-                "whole-window rescoring, full rebuild); each kernel launch covers every layer; "
-                "per-launch CUDA-event times, L2 flushed before each step" % n_layers,
+        "note": "one fk_compress over %d layers of the 480P layer workload (per-head scoring); "
+                "each kernel launch covers every layer; per-launch CUDA-event times, L2 flushed "
+                "before each step%s" % (n_layers, "; the append kernels form the new pairs' sums, "
+                                        "so no scoring kernel runs" if incremental else ""),
     }
 
 
