@@ -240,7 +240,9 @@ def _read_floor(args, nbytes, calib, flush, stream):
     from paper_2605_09681_gb300 import stream_read
     if not nbytes or calib is None:
         return None
-    nbytes = min(int(nbytes) // 16 * 16, calib.numel())
+    if nbytes > calib.numel():
+        return None
+    nbytes = int(nbytes) // 16 * 16
     reps = max(3, min(args.steps, 50))
     evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(reps)]
     torch.cuda.synchronize()
@@ -317,6 +319,8 @@ def measure_layer(args, w, hm, inp, flush, stream, world, local_rank, peaks, cal
         raise SystemExit("device status %d during the timed region (%s)" % (st, w.name))
     total_ms = reduce_max(total_ms, world)
     floor = _read_floor(args, alg["score_bytes"], calib, flush, stream)
+    floor_append = _read_floor(args, alg["append_bytes"], calib, flush, stream)
+    floor_compact = _read_floor(args, alg["compact_bytes"], calib, flush, stream)
 
     # end to end: pinned host inputs copied (on the handle's copy stream, overlapping the work
     # already queued) and the output copied back every step; one continuous timed interval over
@@ -378,7 +382,9 @@ def measure_layer(args, w, hm, inp, flush, stream, world, local_rank, peaks, cal
         "roofline_hbm": {
             "compact": {"achieved": round(compact_gbs, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
                         "frac": round(compact_gbs / peaks["hbm_gbs"], 4), "bytes": alg["compact_bytes"],
-                        "us": round(compact_ms * 1e3, 2), "traffic": traffic.get("compact")},
+                        "us": round(compact_ms * 1e3, 2), "traffic": traffic.get("compact"),
+                        "read_floor_us": round(floor_compact, 2) if floor_compact else None,
+                        "frac_of_read_floor": round(floor_compact / (compact_ms * 1e3), 4) if floor_compact else None},
             "score": ({"achieved": round(score_gbs, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
                        "frac": round(score_gbs / peaks["hbm_gbs"], 4), "bytes": alg["score_bytes"],
                        "us": round(score_ms * 1e3, 2), "traffic": traffic.get("score"),
@@ -390,12 +396,15 @@ def measure_layer(args, w, hm, inp, flush, stream, world, local_rank, peaks, cal
                        "frac": round(alg["append_bytes"] / (per_launch("append") * 1e-3) / 1e9 / peaks["hbm_gbs"], 4),
                        "bytes": alg["append_bytes"], "us": round(per_launch("append") * 1e3, 2),
                        "traffic": traffic.get("append"),
+                       "read_floor_us": round(floor_append, 2) if floor_append else None,
+                       "frac_of_read_floor": round(floor_append / (per_launch("append") * 1e3), 4) if floor_append else None,
                        "scores_retired_chunk": alg["score_fused"]},
             "peak_source": peaks["source"] + " HBM copy bandwidth",
             "traffic_source": TRAFFIC_SOURCE if traffic else None,
-            "read_floor_note": "read_floor_us: event-timed fk_stream_read of the scoring kernel's bytes "
-                               "after the same L2 flush (a plain streaming read: the floor for any "
-                               "launch that reads those bytes); frac_of_read_floor = floor / kernel time",
+            "read_floor_note": "read_floor_us: event-timed fk_stream_read of as many bytes as the kernel "
+                               "moves, after the same L2 flush (a plain streaming read: the floor for any "
+                               "single launch that moves those bytes; the append and compaction also "
+                               "write half of theirs); frac_of_read_floor = floor / kernel time",
         },
         "kernels_us_per_step": {k: round(prof[k][0] / args.steps * 1e3, 2) for k in prof},
         "attn_fps_extrapolated": round(attn_fps, 2),
@@ -416,7 +425,7 @@ def run_fk(args, rank, world, local_rank):
     flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream(dev)
     peaks = _peaks()
-    calib = torch.ones(256 << 20, dtype=torch.uint8, device=dev)   # read-floor calibration data
+    calib = torch.ones(768 << 20, dtype=torch.uint8, device=dev)   # read-floor calibration data
 
     w = _workload(args.workload)
     hm = W.head_map(w)
