@@ -189,6 +189,18 @@ def test_stream_layer0_pooled_small():
     assert run_stream(w, track_layers=(0, 1, 2)) == 5 * 2 * 3
 
 
+@pytest.mark.parametrize("incremental", [False, True])
+def test_stream_per_head_scoring_many_layers(incremental):
+    # per-head scoring in every layer, each layer with its own keys: one compress scores and
+    # compacts all layers in single launches (the flattened per-layer ranges of the scoring
+    # kernel, the multi-layer item list of the compaction); every layer's scores, kept sets and
+    # attention are compared with its own oracle, whole-window and incremental
+    w = W.P480_STACK.with_(name="layers_per_head_small", n_layers=5, n_heads=4, head_dim=128,
+                           tokens_per_frame=60, n_chunks=6, denoise_steps=1,
+                           score_source="per_head", incremental=incremental, window_frames=4)
+    assert run_stream(w, track_layers=(0, 1, 2, 3, 4)) == 6 * 5
+
+
 # ------------------------------------------------------------------ error paths (host-side)
 def test_state_errors():
     from paper_2605_09681_gb300 import ForcingKVCache, FkError
