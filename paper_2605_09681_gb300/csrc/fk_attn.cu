@@ -45,8 +45,9 @@ constexpr int kAttnThreads = 320;
 
 struct AttnBarriers {
   uint64_t q_full;
-  uint64_t k_full[2], k_empty[2];
-  uint64_t v_full[2], v_empty[2];
+  uint64_t k_full[2], k_empty[2];   // profiling: the key ring
+  uint64_t k0_full, k0_empty;       // attention: key tile 0 (stage 0)
+  uint64_t vk_full[2], vk_empty[2]; // attention, b = j mod 2: V_j (V stage b) with K_{j+1} (K stage 1-b)
   uint64_t s_full[2], p_full[2];
   uint64_t o_done, fin;
   uint64_t q8_ready;            // FP8_QK: the 256 softmax threads have written the E4M3 Q rows
@@ -350,11 +351,11 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
 
   if (threadIdx.x == 0) {
     mbar_init(&bar->q_full, 1);
+    mbar_init(&bar->k0_full, 1);
+    mbar_init(&bar->k0_empty, 1);
     for (int i = 0; i < 2; ++i) {
-      mbar_init(&bar->k_full[i], 1);
-      mbar_init(&bar->k_empty[i], 1);
-      mbar_init(&bar->v_full[i], 1);
-      mbar_init(&bar->v_empty[i], 1);
+      mbar_init(&bar->vk_full[i], 1);
+      mbar_init(&bar->vk_empty[i], 1);
       mbar_init(&bar->s_full[i], 1);
       mbar_init(&bar->p_full[i], 4);
     }
@@ -377,8 +378,8 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
   if (warp == kWarpTma) {
     // ------------------------------------------------------------------ TMA producer
     if (lane == 0) {
-      int lastK[2] = {-1, -1}, lastV[2] = {-1, -1};
-      bool ok = true;
+      int lastVK[2] = {-1, -1};
+      bool ok = true, k0 = false;
       // Q, K and V may have been written by the previous kernel of the stream
       asm volatile("griddepcontrol.wait;" ::: "memory");
       // bf16 query tiles: the MMA operand, or (FP8) the softmax threads' quantization input
@@ -389,35 +390,42 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
         for (int h = 0; h < kHalves; ++h)
           tma_load_3d(q_dst + t * kQBytes + h * 16384, &tmQ, &bar->q_full, h * 64, head,
                       q0 + t * kAttnBM);
-      for (int j = 0; j < nt && ok; ++j) {
-        const int st = j & 1, u = j >> 1;
-        if (j >= 2 && !wait_phase(&bar->k_empty[st], (u - 1) & 1, bar, a.status)) { ok = false; break; }
-        mbar_expect_tx(&bar->k_full[st], Lay::kK);
+      auto load_k = [&](int j, uint64_t* b) {         // key tile j into K stage j mod 2
+        const int st = j & 1;
         if constexpr (kFp8) {
-          tma_load_2d(sK + st * Lay::kK, &tmK, &bar->k_full[st], 0, row0 + j * kAttnBN);
+          tma_load_2d(sK + st * Lay::kK, &tmK, b, 0, row0 + j * kAttnBN);
         } else {
           for (int h = 0; h < kHalves; ++h)
-            tma_load_2d(sK + st * Lay::kK + h * 16384, &tmK, &bar->k_full[st], h * 64,
-                        row0 + j * kAttnBN);
+            tma_load_2d(sK + st * Lay::kK + h * 16384, &tmK, b, h * 64, row0 + j * kAttnBN);
         }
-        lastK[st] = u;
-        if (j >= 2 && !wait_phase(&bar->v_empty[st], (u - 1) & 1, bar, a.status)) { ok = false; break; }
-        mbar_expect_tx(&bar->v_full[st], Lay::kKV);
+      };
+      mbar_expect_tx(&bar->k0_full, Lay::kK);
+      load_k(0, &bar->k0_full);
+      k0 = true;
+      // then per key tile j: V_j together with K_{j+1} on one barrier (b = j mod 2).  Their
+      // stages were last used by V_{j-2} and K_{j-1}, released together by vk_empty[b] after
+      // iteration j-2's MMAs (K_2 reuses K_0's stage: k0_empty)
+      for (int j = 0; j < nt && ok; ++j) {
+        const int bb = j & 1, u = j >> 1;
+        const bool more = j + 1 < nt;
+        if (j >= 2 && !wait_phase(&bar->vk_empty[bb], (u - 1) & 1, bar, a.status)) { ok = false; break; }
+        if (j == 1 && more && !wait_phase(&bar->k0_empty, 0, bar, a.status)) { ok = false; break; }
+        mbar_expect_tx(&bar->vk_full[bb], Lay::kKV + (more ? Lay::kK : 0));
         if constexpr (kFp8PV) {
-          tma_load_2d(sV + st * Lay::kKV, &tmV, &bar->v_full[st], 0, row0 + j * kAttnBN);
+          tma_load_2d(sV + bb * Lay::kKV, &tmV, &bar->vk_full[bb], 0, row0 + j * kAttnBN);
         } else {
           for (int h = 0; h < kHalves; ++h)
-            tma_load_2d(sV + st * Lay::kKV + h * 16384, &tmV, &bar->v_full[st], h * 64,
+            tma_load_2d(sV + bb * Lay::kKV + h * 16384, &tmV, &bar->vk_full[bb], h * 64,
                         row0 + j * kAttnBN);
         }
-        lastV[st] = u;
+        if (more) load_k(j + 1, &bar->vk_full[bb]);
+        lastVK[bb] = u;
       }
       if (!ok) {   // drain every load this thread issued before the CTA exits
         wait_phase(&bar->q_full, 0, bar, a.status, false);
-        for (int st = 0; st < 2; ++st) {
-          if (lastK[st] >= 0) wait_phase(&bar->k_full[st], lastK[st] & 1, bar, a.status, false);
-          if (lastV[st] >= 0) wait_phase(&bar->v_full[st], lastV[st] & 1, bar, a.status, false);
-        }
+        if (k0) wait_phase(&bar->k0_full, 0, bar, a.status, false);
+        for (int bb = 0; bb < 2; ++bb)
+          if (lastVK[bb] >= 0) wait_phase(&bar->vk_full[bb], lastVK[bb] & 1, bar, a.status, false);
       }
     }
     __syncwarp();
@@ -472,20 +480,19 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
         }
       };
       bool ok = wait_phase(kFp8 ? &bar->q8_ready : &bar->q_full, 0, bar, a.status) &&
-                wait_phase(&bar->k_full[0], 0, bar, a.status);
+                wait_phase(&bar->k0_full, 0, bar, a.status);
       if (ok) {
         tc_fence_after();
         qk(0, 0);
         qk(0, 1);
-        umma_commit(&bar->k_empty[0]);
+        umma_commit(&bar->k0_empty);
       }
       for (int j = 0; j < nt && ok; ++j) {
-        const int st = j & 1;
+        const int bb = j & 1;
         const bool more = j + 1 < nt;
-        // V_j and K_{j+1} are waited for before P_0(j): neither depends on the softmax, and
+        // V_j and K_{j+1} (one barrier) before P_0(j): neither depends on the softmax, and
         // PV0(j), S0(j+1) then go to the tensor pipe back to back once P_0(j) is in TMEM
-        if (!wait_phase(&bar->v_full[st], (j >> 1) & 1, bar, a.status) ||
-            (more && !wait_phase(&bar->k_full[(j + 1) & 1], ((j + 1) >> 1) & 1, bar, a.status)) ||
+        if (!wait_phase(&bar->vk_full[bb], (j >> 1) & 1, bar, a.status) ||
             !wait_phase(&bar->p_full[0], j & 1, bar, a.status)) { ok = false; break; }
         tc_fence_after();
         pv(j, 0);
@@ -493,11 +500,8 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
         if (!wait_phase(&bar->p_full[1], j & 1, bar, a.status)) { ok = false; break; }
         tc_fence_after();
         pv(j, 1);
-        umma_commit(&bar->v_empty[st]);
-        if (more) {
-          qk(j + 1, 1);
-          umma_commit(&bar->k_empty[(j + 1) & 1]);
-        }
+        if (more) qk(j + 1, 1);
+        umma_commit(&bar->vk_empty[bb]);             // V_j and K_{j+1} consumed
       }
       if (ok) umma_commit(&bar->o_done);
       umma_commit(&bar->fin);                       // completes once every MMA above is done
