@@ -100,6 +100,16 @@ __device__ __forceinline__ bool mbar_test(uint64_t* b, uint32_t parity) {
   return ok != 0;
 }
 
+// Non-blocking test of the phase of parity `parity` (acquire when it has completed).
+__device__ __forceinline__ bool mbar_peek(uint64_t* b, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok) : "r"(su32(b)), "r"(parity) : "memory");
+  return ok != 0;
+}
+
 // Bounded wait for the phase of parity `parity`.  Returns false when the CTA is
 // aborting or the limit expired (which starts the abort).  Inlined: a call would save and
 // restore the caller's live registers on every wait, even when the phase is complete.
@@ -487,19 +497,24 @@ attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
         qk(0, 1);
         umma_commit(&bar->k0_empty);
       }
+      // barriers found complete by a test made while the pipe was busy with the group just issued
+      // need no wait afterwards (each wait costs ~100 cycles where the pipe would drain)
+      bool vk_ready = false;
       for (int j = 0; j < nt && ok; ++j) {
         const int bb = j & 1;
         const bool more = j + 1 < nt;
         // V_j and K_{j+1} (one barrier) before P_0(j): neither depends on the softmax, and
         // PV0(j), S0(j+1) then go to the tensor pipe back to back once P_0(j) is in TMEM
-        if (!wait_phase(&bar->vk_full[bb], (j >> 1) & 1, bar, a.status) ||
+        if (!(vk_ready || wait_phase(&bar->vk_full[bb], (j >> 1) & 1, bar, a.status)) ||
             !wait_phase(&bar->p_full[0], j & 1, bar, a.status)) { ok = false; break; }
         tc_fence_after();
         pv(j, 0);
+        const bool p1_ready = mbar_peek(&bar->p_full[1], j & 1);
         if (more) qk(j + 1, 0);
-        if (!wait_phase(&bar->p_full[1], j & 1, bar, a.status)) { ok = false; break; }
+        if (!(p1_ready || wait_phase(&bar->p_full[1], j & 1, bar, a.status))) { ok = false; break; }
         tc_fence_after();
         pv(j, 1);
+        vk_ready = more && mbar_peek(&bar->vk_full[(j + 1) & 1], ((j + 1) >> 1) & 1);
         if (more) qk(j + 1, 1);
         umma_commit(&bar->vk_empty[bb]);             // V_j and K_{j+1} consumed
       }
