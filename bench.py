@@ -869,9 +869,9 @@ def run_stack(local_rank, attn_precision="bf16"):
 # is reported only while that source is unchanged.
 NCU_TRAFFIC = {
     "480p_layer": {
-        "attend": ("fk_attn.cu", "f44ee3bd8b6b", 118520000),
-        "attend_fp8": ("fk_attn.cu", "f44ee3bd8b6b", 91930000),
-        "attend_fp8pv": ("fk_attn.cu", "f44ee3bd8b6b", 65860000),
+        "attend": ("fk_attn.cu", "58646e428577", 118530000),
+        "attend_fp8": ("fk_attn.cu", "58646e428577", 91830000),
+        "attend_fp8pv": ("fk_attn.cu", "58646e428577", 65870000),
         "append": ("fk_copy.cu", "2690c64c569f", 53940000),
         "compact": ("fk_copy.cu", "2690c64c569f", 58110000),
         "score": ("fk_score.cu", "c31614e0df7f", 35970000),
