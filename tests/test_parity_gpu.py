@@ -102,6 +102,17 @@ def test_stream_window_small():
     assert run_stream(w) == 12
 
 
+@pytest.mark.parametrize("precision", ["bf16", "fp8_qk", "fp8"])
+def test_heads_of_one_key_tile(precision):
+    # every view fits one 128-key tile (60 current keys at the first chunk, then 100 static and
+    # 120 dynamic): the attention's path with key tile 0 alone and a ragged (half-empty) tile,
+    # in each precision, through appends, compressions and a sliding window
+    w = W.ROLLING.with_(name="one_tile_" + precision, head_dim=128, tokens_per_frame=20, n_heads=4,
+                        n_segments=4, window_frames=3, n_chunks=5, keep_budget_permille=500,
+                        attn_precision=precision)
+    assert run_stream(w) == 5
+
+
 def test_incremental_compaction_matches_rebuild():
     # Incremental mode appends only newly decided segments into a ring of kept-segment slots;
     # the rebuild copies every kept segment each time.  The views hold the same keys in a
