@@ -307,16 +307,12 @@ def test_480p_stack_full():
     assert run_stream(w, track_layers=(0, 13, 29), compare_every=3, step_filter=(0, 3)) > 0
 
 
-@pytest.mark.parametrize("head_dim,F,hist", [(128, 260, 8), (64, 100, 5), (128, 24, 2), (64, 40, 2)])
-def test_head_profile_matches_oracle(head_dim, F, hist):
-    # Eq. 1 masses from the tcgen05 profiling kernel vs the fp64 oracle on the same bf16
-    # inputs; 3-frame chunk, ragged query and key tiles, class boundaries inside key tiles.
-    # The two CTAs of a cluster split the key tiles: 27 (13 + 14), 8, a single tile (the
-    # first CTA has none) and two tiles (one each, the second ragged).
-    # A second call adds to the same accumulator.
+def _check_head_profile(q, k, g, s, t):
+    """Eq. 1 masses of the GPU kernel vs the fp64 oracle on the same bf16 inputs; the
+    classification of every head not within 1e-3 of the threshold; a second call adds to the
+    same accumulator."""
     from paper_2605_09681_gb300 import classify_heads, head_profile
-    H = 8
-    q, k, (g, s, t) = W.profile_inputs(11 + head_dim, H, head_dim, F, 3, 1, hist)
+    H = q.shape[1]
     Qd, Kd = to_dev(q), to_dev(k)
     mass, status = head_profile(Qd, Kd, g, s, t)
     torch.cuda.synchronize()
@@ -334,6 +330,28 @@ def test_head_profile_matches_oracle(head_dim, F, hist):
     head_profile(Qd, Kd, g, s, t, mass=mass, status=status)
     torch.cuda.synchronize()
     assert np.allclose(mass.cpu().numpy(), 2 * got, rtol=1e-12, atol=0)
+
+
+@pytest.mark.parametrize("head_dim,F,hist", [(128, 260, 8), (64, 100, 5), (128, 24, 2), (64, 40, 2)])
+def test_head_profile_matches_oracle(head_dim, F, hist):
+    # 3-frame chunk, ragged query and key tiles, class boundaries inside key tiles.  The two
+    # CTAs of a cluster split the key tiles: 27 (13 + 14), 8, a single tile (the first CTA has
+    # none) and two tiles (one each, the second ragged).
+    q, k, (g, s, t) = W.profile_inputs(11 + head_dim, 8, head_dim, F, 3, 1, hist)
+    _check_head_profile(q, k, g, s, t)
+
+
+@pytest.mark.parametrize("i", range(16))
+def test_head_profile_sweep(i):
+    # seeded draws of heads (1-12), head_dim, tokens per frame (8-300), chunk frames (1-3),
+    # sink frames (0-2, so an empty sink class too) and other history frames (0-7): query
+    # tiles, key tiles, the cluster's key split and the class boundaries land anywhere
+    rng = np.random.default_rng(3571 * (i + 1))
+    H, D = int(rng.integers(1, 13)), int(rng.choice([64, 128]))
+    F, C, S = int(rng.integers(8, 301)), int(rng.integers(1, 4)), int(rng.integers(0, 3))
+    hist = S + 1 + int(rng.integers(0, 8))
+    q, k, (g, s, t) = W.profile_inputs(200 + i, H, D, F, C, S, hist)
+    _check_head_profile(q, k, g, s, t)
 
 
 def test_host_inputs_and_overlap_match_device_inputs():
