@@ -85,6 +85,24 @@ def test_validate_accepts_paper_configs(lib):
         assert lib.fk_validate_config(ctypes.byref(c)) == 0, kw
 
 
+def test_validate_accepts_every_sweep_config(lib):
+    # the seeded configurations of the GPU parity sweep, built the way the binding builds them
+    from paper_2605_09681_gb300._lib import FK_ATTN, FK_SELECT, FkConfig
+    import workloads as W
+    from sweep_cases import N_CASES, N_LARGE, sweep_case
+    cases = [sweep_case(i) for i in range(N_CASES)] + [sweep_case(i, True) for i in range(N_LARGE)]
+    for w in cases:
+        hm = np.ascontiguousarray(W.head_map(w).reshape(-1))
+        c = FkConfig(w.n_layers, w.n_heads, w.head_dim, w.tokens_per_frame, w.frames_per_chunk,
+                     w.n_sink_frames, w.window_frames, w.n_segments, w.keep_budget_permille,
+                     {"per_frame": 0, "pooled": 1}[w.select_scope],
+                     {"per_head": 0, "layer0_pooled": 1}[w.score_source], int(w.incremental),
+                     max(1, w.max_history_frames()), 0,
+                     hm.ctypes.data_as(ctypes.POINTER(ctypes.c_uint8)), FK_SELECT[w.selection],
+                     w.select_seed, int(w.static_drop_anchor), FK_ATTN[w.attn_precision])
+        assert lib.fk_validate_config(ctypes.byref(c)) == 0, w.name
+
+
 def test_null_config_and_status_strings(lib):
     assert lib.fk_validate_config(None) == 2
     for s in range(9):
