@@ -405,6 +405,9 @@ def measure_layer(args, w, hm, inp, flush, stream, world, local_rank, peaks, cal
                                "moves, after the same L2 flush (a plain streaming read: the floor for any "
                                "single launch that moves those bytes; the append and compaction also "
                                "write half of theirs); frac_of_read_floor = floor / kernel time",
+            "write_note": "the append's and the compaction's view writes mostly stay in L2, where the "
+                          "attention that follows reads them: their DRAM write bytes (in traffic) "
+                          "understate the writes, and the write-back lands in later kernels of the step",
         },
         "kernels_us_per_step": {k: round(prof[k][0] / args.steps * 1e3, 2) for k in prof},
         "attn_fps_extrapolated": round(attn_fps, 2),
