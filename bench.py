@@ -868,32 +868,41 @@ def run_stack(local_rank, attn_precision="bf16"):
 
 
 # DRAM bytes (read + write) per launch from one ncu capture of each kernel on the 480P
-# workload, with the SHA-1 prefix of the kernel source the capture was taken on: a figure
-# is reported only while that source is unchanged.
+# workload, with the SHA-1 prefix of the kernel source's code (comments and blank lines
+# removed) the capture was taken on: a figure is reported only while that code is unchanged.
 NCU_TRAFFIC = {
     "480p_layer": {
-        "attend": ("fk_attn.cu", "58646e428577", 118530000),
-        "attend_fp8": ("fk_attn.cu", "58646e428577", 91830000),
-        "attend_fp8pv": ("fk_attn.cu", "58646e428577", 65870000),
-        "append": ("fk_copy.cu", "2690c64c569f", 53940000),
-        "compact": ("fk_copy.cu", "2690c64c569f", 58110000),
-        "score": ("fk_score.cu", "c31614e0df7f", 35970000),
+        "attend": ("fk_attn.cu", "3f055d216605", 118530000),
+        "attend_fp8": ("fk_attn.cu", "3f055d216605", 91830000),
+        "attend_fp8pv": ("fk_attn.cu", "3f055d216605", 65870000),
+        "append": ("fk_copy.cu", "bd1364854f34", 53940000),
+        "compact": ("fk_copy.cu", "bd1364854f34", 58110000),
+        "score": ("fk_score.cu", "02ad1f1c1247", 35970000),
     },
 }
 
 
 TRAFFIC_SOURCE = ("stored DRAM bytes per launch (read + write, median of three launches) from an "
                   "earlier ncu capture of the same kernel source, one kernel per capture "
-                  "(profiles/launches_480p_layer.md); reported only while the source hash matches, "
-                  "not observed in this run")
+                  "(profiles/launches_480p_layer.md); reported only while the code hash (comments "
+                  "excluded) matches, not observed in this run")
+
+
+def _code_hash(path):
+    """SHA-1 prefix of a CUDA source without its comments and blank lines."""
+    import hashlib
+    import re
+    src = re.sub(r"/\*.*?\*/", "", open(path).read(), flags=re.S)
+    src = re.sub(r"//[^\n]*", "", src)
+    lines = [line.rstrip() for line in src.splitlines() if line.strip()]
+    return hashlib.sha1("\n".join(lines).encode()).hexdigest()[:12]
 
 
 def _traffic(workload):
-    import hashlib
     out = {}
     for kind, (src, sha, nbytes) in NCU_TRAFFIC.get(workload, {}).items():
         path = os.path.join(ROOT, "paper_2605_09681_gb300", "csrc", src)
-        cur = hashlib.sha1(open(path, "rb").read()).hexdigest()[:12] if os.path.exists(path) else ""
+        cur = _code_hash(path) if os.path.exists(path) else ""
         out[kind] = nbytes if cur == sha else None
     return out
 

@@ -5,13 +5,21 @@
 // in tiles of 128 keys, on the 5th-generation tensor cores:
 //   warp 8 (one lane)  TMA: both Q tiles once (3D map over [Nq][H][D]), K and V tiles (2D
 //                      maps over the view arenas) into two-stage rings, 128-byte swizzle;
-//   warp 9 (one lane)  tcgen05.mma: S_t = Q_t K^T into TMEM (t = 0, 1), then
-//                      O_t += P_t V with P_t read from TMEM; completion via tcgen05.commit;
+//                      key tile 0 on its own barrier, then V_j together with K_{j+1} on one
+//                      barrier per stage pair (one wait and one release per key tile);
+//   warp 9 (one lane)  tcgen05.mma, per key tile j: P_0 V_j, S_0(j+1), P_1 V_j, S_1(j+1)
+//                      (S_t = Q_t K^T into TMEM, O_t += P_t V with P_t read from TMEM);
+//                      completion via tcgen05.commit; the barriers of the next group are
+//                      tested without blocking while the tensor pipe still runs this one;
 //   warps 0-3 / 4-7    softmax of query tile 0 / 1 (ping-pong: one warpgroup's softmax
 //                      overlaps the other tile's MMAs): thread r owns row r = TMEM lane r,
 //                      reads S with tcgen05.ld, online softmax in the log2 domain with a
 //                      lazily rescaled running max, writes P as bf16 pairs over S's first
 //                      64 columns with tcgen05.st, and finally normalises O and stores it.
+//                      After the first key tile a 64-key half computes P with the running
+//                      max at once; its sum (at most 2^8) or the packed maximum of its P
+//                      shows that no numerator exceeds the rescale bound, else the half is
+//                      redone with a max pass.
 // TMEM columns: S0 0-127, S1 128-255, O0 256.., O1 256+D.. (512 allocated).
 // FP8_QK variant (D = 128): the K tiles hold E4M3 codes (one 128-byte swizzle atom per row,
 // from the view arena's E4M3 copy); the bf16 Q tiles are loaded as usual and each softmax
@@ -19,6 +27,10 @@
 // 2^-e_row, written in the 128-byte swizzle pattern) before the first MMA; S = Q K^T runs as
 // tcgen05.mma kind::f8f6f4 (K = 32 per instruction) and the thread scales its row's logits by
 // 2^e_row along with 1/sqrt(D); P V is unchanged (bf16).
+// FP8 variant (P V too): the V tiles hold E4M3 codes of the V arena's E4M3 copy, P is stored
+// as E4M3 codes of 2^6 exp2(S c - m) (four per TMEM column) with m an integer running
+// reference, and P V runs as kind::f8f6f4; O and the row sum are rescaled by exact powers of
+// two when the reference moves.
 // Every mbarrier wait is bounded (%globaltimer); on expiry the CTA records
 // FK_ERR_TIMEOUT in the status word, drains its own TMA loads and MMAs and frees TMEM.
 // The kernel is launched with programmatic dependent launch: its setup (barriers, TMEM) may
