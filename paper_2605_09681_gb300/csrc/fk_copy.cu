@@ -5,7 +5,7 @@
 // it retires), the prefill scatter of history frames, and the gather of kept segments into the
 // packed per-head views of dynamic heads (Sec. 4.3, Eq. 4: sink, kept segments and the anchor
 // frame; attention does not depend on the order of the keys, so a view holds them as
-// [sinks | anchor | kept-segment ring] and incremental compaction only appends).
+// [current chunk | sinks | anchor | kept-segment ring] and incremental compaction only appends).
 // All of them are HBM-bound: every byte is read once and written once in 16-byte accesses.
 // Under FP8 attention each of them also writes the E4M3 codes of every view K row it writes
 // (8 bytes per 16-byte granule), and of every view V row under FP8 P V, so the attention's
