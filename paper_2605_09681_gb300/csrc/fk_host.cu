@@ -16,9 +16,10 @@
 //                int64 scoring sums (scratch); status word;
 //                host staging (two slots of K, V and Q; O) and the attention key-split
 //                scratch (fp32 partial outputs and row statistics of two splits).
-//   FP8_QK only  the E4M3 copy of the K view arena ([rows][D] bytes, written by the copy
-//                kernels together with every bf16 view K row; the attention kernel
-//                quantizes its query tiles itself).
+//   FP8 only     the E4M3 copy of the K view arena ([rows][D] bytes, written by the copy
+//                kernels together with every bf16 view K row) and, when P V also runs on
+//                E4M3 (FK_ATTN_FP8), of the V view arena; the attention kernel quantizes
+//                its query tiles itself.
 #include <algorithm>
 #include <cmath>
 #include <cstdio>
